@@ -59,6 +59,8 @@ import numpy as np
 # Quantizer ids: the value is the number of storage bits per code.
 BINARY = 1
 TERNARY = 2
+# |entry| below this in the fp64 encode table is fp64 noise on an exact zero.
+ZERO_FLUSH = 2.0 ** -46
 # alpha modes.
 ALPHA_MAXABS = 0
 ALPHA_MEANABS = 1
@@ -164,6 +166,11 @@ def encode_table(block: int, n_b: int, signs=None, hadamard: bool = True) -> np.
     _check_geometry(block, n_b)
     had = hadamard_matrix(block, signs, hadamard)
     a64 = (had @ resample_matrix(block, n_b)).T
+    # Entries that are exactly zero in real arithmetic (e.g. the interpolating
+    # property of Resample at integer OSR, and cancellations of the Hadamard
+    # rows) come out of fp64 as +-1e-16 noise; they are set to exact zero so
+    # that the fp32 table does not depend on how the fp64 value was computed.
+    a64[np.abs(a64) < ZERO_FLUSH] = 0.0
     return a64.astype(np.float32)
 
 
