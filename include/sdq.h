@@ -1,0 +1,192 @@
+/*
+ * sdq.h -- C ABI of the GB300 (sm_103a) Sigma-Delta-quantized linear layer.
+ *
+ * SDQ-LLM (arXiv 2510.03275) stores each linear layer's weights as
+ * Sigma-Delta codes of the Hadamard-smoothed, OSR-times upsampled weight rows
+ * (section 3, Algorithm 1).  This library implements, on one GPU:
+ *
+ *   sdq_encode_rows      Algorithm 1 (SDQuant + Resample) per output row:
+ *                        randomised Hadamard smoothing (eq. 13), band-limited
+ *                        upsampling, per-row scale, first-order Sigma-Delta
+ *                        scan (eqs. 7-8) with the binary (eqs. 3-4) or ternary
+ *                        (eqs. 5-6) quantizer.  GPTQ block compensation is
+ *                        not applied (no calibration data; blocks independent).
+ *   sdq_pack/sdq_unpack  plain <-> tiled code layouts (bit-exact).
+ *   sdq_prep_activations x_tilde = G x per block of B inputs, G = D^T Had^T:
+ *                        the exact adjoint of the decimation and Hadamard
+ *                        reconstruction, i.e. the activation upsampling of
+ *                        section 3.5 (Fig. 5) that makes the inner product of
+ *                        eq. (12) equal x . W_hat^T.
+ *   sdq_contract         y[m,r] = alpha_r * sum_j c[r,j] x_tilde[m,j]
+ *                        (decode path for M <= 64, tensor-core prefill path
+ *                        above).
+ *   sdq_linear_forward   sdq_prep_activations + sdq_contract.
+ *
+ * Conventions
+ *  - Every entry point returns an int: SDQ_OK (0) or a negative sdq_status.
+ *    Nothing throws across the ABI.
+ *  - Device pointers are caller-owned device memory; host pointers are
+ *    marked "host".  No entry point allocates device memory except
+ *    sdq_plan_create (its tables) -- hot calls take a caller workspace.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream).  Launches are asynchronous; launch-configuration errors are
+ *    reported as SDQ_ERR_CUDA.  A plan is immutable after creation and may be
+ *    used from several host threads and streams at once, provided every
+ *    concurrent call has its own workspace.
+ *  - bf16 activations are passed as their 16-bit patterns (uint16_t).
+ *
+ * Code values.  Ternary codes are {-1, 0, +1}; binary codes are {-1, +1}.
+ * The real weight block the codes stand for is
+ *   W_hat[r, bB:(b+1)B] = alpha_r * Resample(c[r, b*n_b:(b+1)*n_b], B) . Had^T
+ * with Had = diag(d) . H_B / sqrt(B) (H_B Sylvester, d the sign vector given
+ * to sdq_plan_create) and Resample the FFT resampler of Algorithm 1.
+ *
+ * Plain layout (canonical; output of sdq_encode_rows): b bits per code
+ * (b = 2 ternary, 1 binary).  Row r occupies words_per_row =
+ * 4 * ceil(K_eff * b / 128) uint32 words starting at word r * words_per_row;
+ * code j of the row sits at bit b * (j % (32/b)) of word j / (32/b).
+ * Ternary fields: 00 = 0, 01 = +1, 11 = -1 (10 is invalid).  Binary: 1 = +1,
+ * 0 = -1.  Padding bits are 0.
+ *
+ * Tiled layout (input of sdq_contract; built by sdq_pack):  rows are grouped
+ * by 16 (row group G) and codes by kc = 128 (ternary) or 256 (binary)
+ * (chunk c).  Tile (G, c) holds rows [16G, 16G+16) x codes [kc c, kc c + kc)
+ * in 128 consecutive uint32 words starting at word 128 * (G * C + c),
+ * C = ceil(K_eff / kc).  Word 32 q + L (q = 0..3, L = 0..31, g = L / 4,
+ * t = L % 4) holds these codes, field f at bits [b f, b f + b):
+ *   ternary: j = 3 - f % 4, i = f / 4,
+ *            row = 16G + g + 8 (j % 2),  k = 128c + 32q + 16 (j / 2) + 4t + i
+ *   binary:  j = 7 - f % 8, i = f / 8,
+ *            row = 16G + g + 8 (j % 2),
+ *            k = 256c + 64q + 32 (j / 4) + 16 ((j / 2) % 2) + 4t + i
+ * Codes past n_out or K_eff are padding with field value 0.  With this map,
+ * (word << 2j) & 0xC0C0C0C0 (ternary) and ((~word << j) & 0x80808080) |
+ * 0x40404040 (binary) are directly the fp8 (e4m3) A-operand registers of a
+ * 16x8x32 warp MMA, each byte +-2.0 or 0.
+ */
+#ifndef SDQ_H_
+#define SDQ_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SDQ_OK = 0,
+  SDQ_ERR_INVALID_ARG = -1,  /* bad descriptor, size, null or misaligned pointer */
+  SDQ_ERR_UNSUPPORTED = -2,  /* valid but not implemented (e.g. device not sm_103) */
+  SDQ_ERR_WORKSPACE = -3,    /* workspace smaller than sdq_workspace_bytes() */
+  SDQ_ERR_CUDA = -4,         /* a CUDA runtime call or launch failed */
+  SDQ_ERR_TIMEOUT = -5,      /* a bounded device-side wait gave up */
+  SDQ_ERR_BAD_CODE = -6,     /* invalid ternary pattern 10 found */
+  SDQ_ERR_ALLOC = -7         /* host or device allocation failed in plan creation */
+} sdq_status;
+
+typedef enum { SDQ_BINARY = 1, SDQ_TERNARY = 2 } sdq_quantizer; /* value = bits per code */
+typedef enum { SDQ_ALPHA_MAXABS = 0, SDQ_ALPHA_MEANABS = 1 } sdq_alpha_mode;
+
+/* One quantized linear layer.  OSR = osr_num / osr_den (section 3.2; a
+ * fractional OSR such as 2.5 is allowed) with n_b = block * OSR an integer.
+ *   n_out     N, output rows (d_row), 1 .. 2^24
+ *   k_in      K, input columns (d_col), a positive multiple of block
+ *   block     B, Hadamard / resampling block, a power of two in [2, 1024]
+ *   osr_num, osr_den  OSR >= 1, block * osr_num divisible by osr_den,
+ *             n_b = block * osr_num / osr_den <= 4096
+ *   quantizer SDQ_BINARY or SDQ_TERNARY
+ *   hadamard  1: Had = diag(d) H_B / sqrt(B); 0: Had = I
+ *   alpha_mode SDQ_ALPHA_MAXABS (max |x_up| over the row, default) or
+ *             SDQ_ALPHA_MEANABS (mean |x_up|, section 3.1's "mean(|W|)")
+ */
+typedef struct {
+  int32_t n_out;
+  int32_t k_in;
+  int32_t block;
+  int32_t osr_num;
+  int32_t osr_den;
+  int32_t quantizer;
+  int32_t hadamard;
+  int32_t alpha_mode;
+} sdq_layer_desc;
+
+typedef struct sdq_plan_s* sdq_plan;
+
+/* Validate `desc`, build the fp64-derived tables (encode table
+ * A_enc = fp32(U Had^T), activation table G = D^T Had^T) and upload them to
+ * the current device.  `had_signs` (host, `block` entries, each +1 or -1) is
+ * the sign vector d of the randomised Hadamard; NULL means all +1.  The plan
+ * owns its device tables until sdq_plan_destroy.  Errors: INVALID_ARG,
+ * UNSUPPORTED (current device is not compute capability 10.3), ALLOC, CUDA. */
+int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_signs, sdq_plan* out);
+int sdq_plan_destroy(sdq_plan plan);
+
+/* Geometry (host only, no device work).  Return 0 for an invalid descriptor. */
+int64_t sdq_k_eff(const sdq_layer_desc* desc);         /* K * OSR */
+size_t sdq_plain_bytes(const sdq_layer_desc* desc);    /* plain layout size */
+size_t sdq_tiled_bytes(const sdq_layer_desc* desc);    /* tiled layout size */
+/* Workspace needed by sdq_linear_forward / sdq_prep_activations /
+ * sdq_contract at batch M (1 <= M <= 2^20).  0 on invalid input. */
+size_t sdq_workspace_bytes(sdq_plan plan, int32_t M);
+
+/* Host-only table builder used by sdq_plan_create, exposed for checking:
+ * writes A_enc (n_b x block, row-major, fp32) and G (n_b x block, row-major,
+ * fp32) to host buffers (either may be NULL).  Same error codes as
+ * sdq_plan_create minus CUDA/UNSUPPORTED. */
+int sdq_build_tables(const sdq_layer_desc* desc, const int8_t* had_signs,
+                     float* a_enc_host, float* g_host);
+
+/* Algorithm 1 without compensation, on every row of W (device, fp32,
+ * n_out x k_in row-major).  Writes codes in the plain layout
+ * (sdq_plain_bytes) and alpha (device, fp32[n_out]).  Bit-exact contract:
+ * x_up[j] = fl(...fl(fl(A[j,0] w_0) + fl(A[j,1] w_1))...) in ascending k,
+ * i = fl(fl(i + x_up[j]) - y_prev), no FMA contraction; alpha exact max
+ * (MAXABS) or fp32 sequential (block, index)-order sum / K_eff (MEANABS);
+ * ternary: +1 if i > alpha/2, -1 if i < -alpha/2, else 0; binary: +1 if
+ * i >= 0 else -1; y_prev = code * alpha.  Integrator reset every block.
+ * Needs no workspace.  Pointers must be 16-byte aligned. */
+int sdq_encode_rows(sdq_plan plan, const float* W, uint32_t* codes_plain, float* alpha,
+                    void* stream);
+
+/* Plain -> tiled (sdq_tiled_bytes).  Input and output must not overlap. */
+int sdq_pack(sdq_plan plan, const uint32_t* codes_plain, uint32_t* codes_tiled, void* stream);
+/* Tiled -> plain.  If `bad_count` (device, one uint32) is not NULL, the
+ * number of invalid ternary fields (pattern 10) seen is ADDED to it; they
+ * decode to 0.  The caller reads it after the stream completes and treats a
+ * non-zero count as SDQ_ERR_BAD_CODE. */
+int sdq_unpack(sdq_plan plan, const uint32_t* codes_tiled, uint32_t* codes_plain,
+               uint32_t* bad_count, void* stream);
+
+/* x_tilde = G x_b for every block b of every row of x (device, bf16 bits,
+ * M x k_in row-major), written into the workspace `ws` for sdq_contract.
+ * For M <= 64 x_tilde is kept in fp32 (the decode path re-encodes it as a
+ * three-/two-term fp8 expansion inside the contraction kernel); for M > 64
+ * it is written in bf16 in the permuted K order the prefill kernel reads. */
+int sdq_prep_activations(sdq_plan plan, const uint16_t* x, int32_t M,
+                         void* ws, size_t ws_bytes, void* stream);
+
+/* Contraction against the tiled codes: y (device, fp32, M x n_out row-major)
+ * = alpha_r * sum_j c[r,j] x_tilde[m,j], reading the x_tilde that
+ * sdq_prep_activations left in `ws` for the same M.  M <= 64: decode kernel
+ * (fp8 warp MMAs on register-expanded codes, split-K over CTAs with a
+ * deterministic last-CTA reduction).  M > 64: tcgen05 prefill kernel. */
+int sdq_contract(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha, int32_t M,
+                 float* y, void* ws, size_t ws_bytes, void* stream);
+
+/* sdq_prep_activations followed by sdq_contract on the same stream. */
+int sdq_linear_forward(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha,
+                       const uint16_t* x, int32_t M, float* y, void* ws, size_t ws_bytes,
+                       void* stream);
+
+/* Copy x_tilde for M <= 64 out of the workspace as fp32 (M x K_eff,
+ * device), for checking sdq_prep_activations. */
+int sdq_read_prep(sdq_plan plan, int32_t M, const void* ws, float* xt_out, void* stream);
+
+/* Static string for a status code. */
+const char* sdq_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SDQ_H_ */

@@ -1,0 +1,202 @@
+// C ABI of libsdq (declarations and contracts in include/sdq.h).
+#include <cstdlib>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "common.cuh"
+
+namespace sdq {
+
+namespace {
+
+inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+uint16_t host_bf16(double v) {
+  float f = (float)v;
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  u += 0x7FFFu + ((u >> 16) & 1u);
+  return (uint16_t)(u >> 16);
+}
+double host_bf16_value(uint16_t b) {
+  uint32_t u = (uint32_t)b << 16;
+  float f;
+  std::memcpy(&f, &u, 4);
+  return f;
+}
+
+int cuda_status(cudaError_t e) { return e == cudaSuccess ? SDQ_OK : SDQ_ERR_CUDA; }
+
+}  // namespace
+
+WsLayout workspace_layout(const sdq_plan_s* pl, int M) {
+  const Geometry& g = pl->geo;
+  WsLayout L{};
+  size_t off = 0;
+  L.xt = off;
+  if (M <= kMaxDecodeM) {
+    const DecodeConfig& dc = pl->dcfg[M];
+    off = align_up(off + sizeof(float) * (size_t)M * g.k_eff_pad, 256);
+    L.pmax = off;
+    off = align_up(off + sizeof(float) * (size_t)M * dc.P, 256);
+    L.part = off;
+    off = align_up(off + (dc.S > 1 ? sizeof(float) * (size_t)dc.S * M * g.ng * 16 : 0), 256);
+    L.cnt = off;
+    off = align_up(off + sizeof(uint32_t) * (size_t)dc.R, 256);
+  } else {
+    off = align_up(off + sizeof(uint16_t) * (size_t)M * g.k_eff_pad, 256);
+    L.pmax = L.part = L.cnt = off;
+  }
+  L.total = off;
+  return L;
+}
+
+}  // namespace sdq
+
+using namespace sdq;
+
+extern "C" int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_signs, sdq_plan* out) {
+  if (!desc || !out) return SDQ_ERR_INVALID_ARG;
+  *out = nullptr;
+  Geometry g;
+  int st = validate(desc, &g);
+  if (st != SDQ_OK) return st;
+  int dev = 0, major = 0, minor = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return SDQ_ERR_CUDA;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return SDQ_ERR_CUDA;
+  if (major != 10 || minor != 3) return SDQ_ERR_UNSUPPORTED;
+
+  const size_t tab = (size_t)g.n_b * g.block;
+  std::vector<float> a_enc(tab), gm(tab), at(tab);
+  st = build_tables(desc, had_signs, a_enc.data(), gm.data());
+  if (st != SDQ_OK) return st;
+  for (int j = 0; j < g.n_b; ++j)
+    for (int k = 0; k < g.block; ++k) at[(size_t)k * g.n_b + j] = a_enc[(size_t)j * g.block + k];
+  std::vector<uint16_t> ghi(tab), glo(tab);
+  for (size_t i = 0; i < tab; ++i) {
+    ghi[i] = host_bf16(gm[i]);
+    glo[i] = host_bf16((double)gm[i] - host_bf16_value(ghi[i]));
+  }
+
+  sdq_plan_s* p = new (std::nothrow) sdq_plan_s();
+  if (!p) return SDQ_ERR_ALLOC;
+  p->desc = *desc;
+  p->geo = g;
+  p->device = dev;
+  p->sm_count = sms;
+  if (cudaMalloc(&p->d_at, sizeof(float) * tab) != cudaSuccess ||
+      cudaMalloc(&p->d_g_hi, sizeof(uint16_t) * tab) != cudaSuccess ||
+      cudaMalloc(&p->d_g_lo, sizeof(uint16_t) * tab) != cudaSuccess) {
+    sdq_plan_destroy(p);
+    return SDQ_ERR_ALLOC;
+  }
+  if (cudaMemcpy(p->d_at, at.data(), sizeof(float) * tab, cudaMemcpyHostToDevice) != cudaSuccess ||
+      cudaMemcpy(p->d_g_hi, ghi.data(), sizeof(uint16_t) * tab, cudaMemcpyHostToDevice) != cudaSuccess ||
+      cudaMemcpy(p->d_g_lo, glo.data(), sizeof(uint16_t) * tab, cudaMemcpyHostToDevice) != cudaSuccess) {
+    sdq_plan_destroy(p);
+    return SDQ_ERR_CUDA;
+  }
+  for (int M = 1; M <= kMaxDecodeM; ++M) p->dcfg[M] = decode_config_search(p, M);
+  *out = p;
+  return SDQ_OK;
+}
+
+extern "C" int sdq_plan_destroy(sdq_plan p) {
+  if (!p) return SDQ_ERR_INVALID_ARG;
+  cudaError_t e = cudaSuccess, e2;
+  if (p->d_at && (e2 = cudaFree(p->d_at)) != cudaSuccess) e = e2;
+  if (p->d_g_hi && (e2 = cudaFree(p->d_g_hi)) != cudaSuccess) e = e2;
+  if (p->d_g_lo && (e2 = cudaFree(p->d_g_lo)) != cudaSuccess) e = e2;
+  delete p;
+  return cuda_status(e);
+}
+
+extern "C" size_t sdq_workspace_bytes(sdq_plan p, int32_t M) {
+  if (!p || M < 1 || M > (1 << 20)) return 0;
+  return workspace_layout(p, M).total;
+}
+
+extern "C" int sdq_encode_rows(sdq_plan p, const float* W, uint32_t* codes_plain, float* alpha,
+                               void* stream) {
+  if (!p || !W || !codes_plain || !alpha) return SDQ_ERR_INVALID_ARG;
+  if (!aligned16(W) || !aligned16(codes_plain) || !aligned16(alpha)) return SDQ_ERR_INVALID_ARG;
+  return cuda_status(launch_encode(p, W, codes_plain, alpha, (cudaStream_t)stream));
+}
+
+extern "C" int sdq_pack(sdq_plan p, const uint32_t* plain, uint32_t* tiled, void* stream) {
+  if (!p || !plain || !tiled || !aligned16(plain) || !aligned16(tiled)) return SDQ_ERR_INVALID_ARG;
+  return cuda_status(launch_pack(p, plain, tiled, (cudaStream_t)stream));
+}
+
+extern "C" int sdq_unpack(sdq_plan p, const uint32_t* tiled, uint32_t* plain, uint32_t* bad_count,
+                          void* stream) {
+  if (!p || !plain || !tiled || !aligned16(plain) || !aligned16(tiled)) return SDQ_ERR_INVALID_ARG;
+  return cuda_status(launch_unpack(p, tiled, plain, bad_count, (cudaStream_t)stream));
+}
+
+static int check_ws(sdq_plan p, int32_t M, const void* ws, size_t ws_bytes) {
+  if (!p || M < 1 || M > 65535) return SDQ_ERR_INVALID_ARG;
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u)) return SDQ_ERR_INVALID_ARG;
+  if (ws_bytes < workspace_layout(p, M).total) return SDQ_ERR_WORKSPACE;
+  return SDQ_OK;
+}
+
+extern "C" int sdq_prep_activations(sdq_plan p, const uint16_t* x, int32_t M, void* ws,
+                                    size_t ws_bytes, void* stream) {
+  int st = check_ws(p, M, ws, ws_bytes);
+  if (st != SDQ_OK) return st;
+  if (!x || !aligned16(x)) return SDQ_ERR_INVALID_ARG;
+  return cuda_status(launch_prep(p, x, M, ws, (cudaStream_t)stream));
+}
+
+extern "C" int sdq_contract(sdq_plan p, const uint32_t* codes_tiled, const float* alpha, int32_t M,
+                            float* y, void* ws, size_t ws_bytes, void* stream) {
+  int st = check_ws(p, M, ws, ws_bytes);
+  if (st != SDQ_OK) return st;
+  if (!codes_tiled || !alpha || !y || !aligned16(codes_tiled) || !aligned16(y)) return SDQ_ERR_INVALID_ARG;
+  if (M <= kMaxDecodeM)
+    return cuda_status(launch_decode(p, codes_tiled, alpha, M, y, ws, (cudaStream_t)stream));
+  cudaError_t e = launch_prefill(p, codes_tiled, alpha, M, y, ws, (cudaStream_t)stream);
+  if (e == cudaErrorNotSupported) return SDQ_ERR_UNSUPPORTED;
+  return cuda_status(e);
+}
+
+extern "C" int sdq_linear_forward(sdq_plan p, const uint32_t* codes_tiled, const float* alpha,
+                                  const uint16_t* x, int32_t M, float* y, void* ws, size_t ws_bytes,
+                                  void* stream) {
+  int st = sdq_prep_activations(p, x, M, ws, ws_bytes, stream);
+  if (st != SDQ_OK) return st;
+  return sdq_contract(p, codes_tiled, alpha, M, y, ws, ws_bytes, stream);
+}
+
+extern "C" int sdq_read_prep(sdq_plan p, int32_t M, const void* ws, float* xt_out, void* stream) {
+  if (!p || M < 1 || M > kMaxDecodeM || !ws || !xt_out) return SDQ_ERR_INVALID_ARG;
+  return cuda_status(launch_read_prep(p, M, ws, xt_out, (cudaStream_t)stream));
+}
+
+namespace sdq {
+
+namespace {
+__global__ void read_prep_kernel(const float* xt, float* out, int M, int64_t k_eff, int64_t kpad) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (int64_t)M * k_eff) return;
+  const int64_t m = i / k_eff, k = i - m * k_eff;
+  out[i] = xt[m * kpad + k];
+}
+}  // namespace
+
+cudaError_t launch_read_prep(const sdq_plan_s* p, int M, const void* ws, float* out, cudaStream_t st) {
+  const WsLayout L = workspace_layout(p, M);
+  const float* xt = reinterpret_cast<const float*>(static_cast<const uint8_t*>(ws) + L.xt);
+  const int64_t n = (int64_t)M * p->geo.k_eff;
+  read_prep_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(xt, out, M, p->geo.k_eff, p->geo.k_eff_pad);
+  return cudaGetLastError();
+}
+
+}  // namespace sdq

@@ -1,0 +1,101 @@
+"""Host-side checks of the C ABI: no GPU needed (no kernel is launched)."""
+import ctypes
+import os
+import re
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2510_03275_gb300 import workloads as W
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    with open(os.path.join(ROOT, "include", "sdq.h")) as f:
+        txt = f.read()
+    return sorted(set(re.findall(r"^\s*(?:[\w\s\*]+?)\b(sdq_\w+)\s*\(", txt, re.M)))
+
+
+def test_exports_every_declared_symbol(sdq):
+    names = _declared()
+    assert "sdq_linear_forward" in names and "sdq_encode_rows" in names and len(names) >= 15
+    L = sdq.lib()
+    for n in names:
+        assert hasattr(L, n), n
+
+
+def test_status_strings(sdq):
+    for st in range(0, -8, -1):
+        s = sdq.sdq_status_string(st)
+        assert s.startswith("SDQ_")
+    assert "unknown" in sdq.sdq_status_string(-99)
+
+
+@pytest.mark.parametrize("n,k,b,osr,q,keff,plain,tiled", [
+    (256, 512, 512, Fraction(2), 2, 1024, 256 * 64 * 4, 16 * 8 * 512),
+    (768, 768, 128, Fraction(5, 2), 1, 1920, 768 * 60 * 4, 48 * 8 * 512),
+    (17, 20, 4, Fraction(5, 2), 2, 50, 17 * 4 * 4, 2 * 1 * 512),
+])
+def test_geometry(sdq, n, k, b, osr, q, keff, plain, tiled):
+    d = sdq.LayerDesc(n, k, b, osr, q)
+    assert sdq.sdq_k_eff(d) == keff
+    assert sdq.sdq_plain_bytes(d) == plain
+    assert sdq.sdq_tiled_bytes(d) == tiled
+    assert O.plain_words_per_row(keff, q) * 4 * n == plain
+
+
+@pytest.mark.parametrize("bad", [
+    dict(n_out=0), dict(k_in=100), dict(block=96), dict(block=2048), dict(osr=Fraction(1, 2)),
+    dict(osr=Fraction(7, 3)), dict(quantizer=3), dict(hadamard=2), dict(alpha_mode=5),
+])
+def test_invalid_descriptors(sdq, bad):
+    base = dict(n_out=64, k_in=256, block=128, osr=Fraction(2), quantizer=2, hadamard=1, alpha_mode=0)
+    base.update(bad)
+    d = sdq.LayerDesc(**base)
+    with pytest.raises(sdq.SdqError) as e:
+        sdq.sdq_build_tables(d)
+    assert e.value.status == -1
+    h = ctypes.c_void_p()
+    assert sdq.lib().sdq_plan_create(ctypes.byref(d.c()), None, ctypes.byref(h)) == -1
+    assert sdq.sdq_k_eff(d) == 0 and sdq.sdq_plain_bytes(d) == 0
+
+
+def test_bad_signs_rejected(sdq):
+    d = sdq.LayerDesc(16, 8, 8, Fraction(2))
+    with pytest.raises(sdq.SdqError):
+        sdq.sdq_build_tables(d, np.array([1, -1, 0, 1, 1, 1, 1, 1]))
+
+
+def test_null_pointers_rejected(sdq):
+    L = sdq.lib()
+    assert L.sdq_plan_create(None, None, None) == -1
+    assert L.sdq_encode_rows(None, None, None, None, None) == -1
+    assert L.sdq_linear_forward(None, None, None, None, 1, None, None, 0, None) == -1
+    assert L.sdq_workspace_bytes(None, 1) == 0
+
+
+def _cfg_tables():
+    seen = {}
+    for ci in range(5):
+        cfg = W.config(ci)
+        for lin in cfg.linears:
+            s = W.hadamard_signs(lin, cfg.block)
+            seen[(cfg.block, lin.osr, s.tobytes())] = (cfg.block, lin.osr, s)
+    return list(seen.values())
+
+
+@pytest.mark.parametrize("block,osr,signs", _cfg_tables()[:6] + [(4, Fraction(5, 2), None),
+                                                                  (4, Fraction(2), None),
+                                                                  (8, Fraction(9, 4), None)])
+@pytest.mark.parametrize("had", [1, 0])
+def test_tables_match_oracle(sdq, block, osr, signs, had):
+    """The library's fp64-built encode table equals the oracle's bit for bit
+    (both are the fp32 rounding of the same real table); G within 1e-6."""
+    d = sdq.LayerDesc(16, block, block, osr, 2, had)
+    a, g = sdq.sdq_build_tables(d, signs)
+    nb = d.n_b
+    assert np.array_equal(a, O.encode_table(block, nb, signs, bool(had)))
+    assert np.abs(g - O.decode_table(block, nb, signs, bool(had))).max() < 1e-6
