@@ -1,0 +1,494 @@
+"""Benchmark of the SDQ linear-layer hot path on GB300.
+
+Workload (N=1): the LLaMA-70B-shaped decoder layer (q/o 8192x8192, k/v
+1024x8192, gate/up 28672x8192, down 8192x28672), OSR 2, ternary codes, B =
+128, synthetic Student-t(5) weights (std 0.015) and N(0,1) bf16
+activations.  One step = the decode forward (prep + contraction) of all
+seven linears at batch M (default 1).  Metric: weight-HBM GB/s = packed code
+bytes of the layer / step time.  The 7 code matrices (428 MB) are streamed in
+turn, so every step reads them from HBM (L2 is 129 MB).
+
+Also reported: the decode kernel's roofline (algorithmic bytes / event-timed
+launch duration against the measured HBM copy bandwidth), the end-to-end
+figure through the C ABI with host buffers, the encoder time, the prefill
+(M = 4096) throughput when available, and the oracle's CPU time.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+Multi-GPU runs (torchrun, one process per GPU) are independent replicas.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "SDQ-linear decode GB/s vs ~8 TB/s HBM; prefill TOPS vs tensor-core peak"
+PROFILE_DECODE = os.path.join(ROOT, "profiles", "decode_llama70b_m1.md")
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5000)
+    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--impl", default="sdq", choices=["sdq", "reference"])
+    ap.add_argument("--m", type=int, default=1, help="decode batch")
+    ap.add_argument("--no-extras", action="store_true", help="skip encode/prefill/sweep/cpu legs")
+    ap.add_argument("--linears", default="", help="comma list of cfg4 linears to run (default: all 7)")
+    return ap.parse_args()
+
+
+# ------------------------------------------------------------------ utils
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return p["hbm_gbs"], p["bf16_tflops"], p.get("bf16_tflops_sustained", p["bf16_tflops"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi SM clocks and throttle reasons, sampled every 100 ms."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.idx = gpu_index
+        self.rows = []
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+            return
+        self.t = threading.Thread(target=self._read, daemon=True)
+        self.t.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.rows.append((time.time(), line.strip()))
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self, t0, t1):
+        sel = [r for (t, r) in self.rows if t0 - 0.15 <= t <= t1 + 0.15]
+        if not sel:
+            sel = [r for (_, r) in self.rows[-3:]]
+        mhz, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in sel:
+            f = [x.strip() for x in r.split(",")]
+            try:
+                mhz.append(float(f[1]))
+                mx = max(mx, float(f[2]))
+            except (ValueError, IndexError):
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        mhz.sort()
+        med = mhz[len(mhz) // 2] if mhz else None
+        return {"sm_mhz": med, "sm_max_mhz": mx or None, "reasons": sorted(reasons),
+                "samples": len(sel)}
+
+
+def profile_traffic(src_files):
+    """dram bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel source (sha256 recorded in the summary)."""
+    try:
+        with open(PROFILE_DECODE) as f:
+            txt = f.read()
+    except OSError:
+        return None, None
+    h = hashlib.sha256()
+    for p in src_files:
+        with open(p, "rb") as f:
+            h.update(f.read())
+    cur = h.hexdigest()[:16]
+    vals = {}
+    for line in txt.splitlines():
+        if ":" in line and line.strip().startswith(("source_sha256", "traffic_bytes_per_launch",
+                                                    "traffic_launch_linear")):
+            k, v = line.split(":", 1)
+            vals[k.strip()] = v.strip()
+    if vals.get("source_sha256") != cur:
+        return None, cur
+    try:
+        return int(vals["traffic_bytes_per_launch"]), cur
+    except (KeyError, ValueError):
+        return None, cur
+
+
+# ------------------------------------------------------------------ layer
+def build_layer(P, W, torch, cfg):
+    """Encode + pack every linear of ``cfg`` on the device; returns the plans
+    with tiled codes and alpha, and the encode time."""
+    layers = []
+    enc_ms = 0.0
+    for lin in cfg.linears:
+        desc = P.LayerDesc(lin.n_out, lin.k_in, cfg.block, lin.osr, cfg.quantizer)
+        plan = P.Plan(desc, W.hadamard_signs(lin, cfg.block))
+        w = W.weights_device(lin)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        codes, alpha = plan.encode(w)
+        tiled = plan.pack(codes)
+        e1.record()
+        torch.cuda.synchronize()
+        enc_ms += e0.elapsed_time(e1)
+        del w, codes
+        layers.append({"lin": lin, "plan": plan, "tiled": tiled, "alpha": alpha,
+                       "code_bytes": P.sdq_tiled_bytes(desc)})
+    torch.cuda.empty_cache()
+    return layers, enc_ms
+
+
+def alg_bytes(lay, M):
+    lin = lay["lin"]
+    # packed codes (2 bits/code) + alpha + bf16 x + fp32 y
+    k_eff = lay["plan"].k_eff
+    return lin.n_out * k_eff * 2 // 8 + 4 * lin.n_out + 2 * M * lin.k_in + 4 * M * lin.n_out
+
+
+def run_sdq(args, rank, world, dist):
+    import numpy as np
+    import torch
+
+    import paper_2510_03275_gb300 as P
+    from paper_2510_03275_gb300 import workloads as W
+
+    dev = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(dev)
+    hbm, tf_burst, tf_sus, peak_src = peaks()
+    cfg = W.config(4)
+    if args.linears:
+        keep = set(args.linears.split(","))
+        cfg.linears = [l for l in cfg.linears if l.name in keep]
+    M = args.m
+    layers, enc_ms = build_layer(P, W, torch, cfg)
+    code_bytes = sum(l["code_bytes"] for l in layers)
+    # per-linear inputs / outputs / workspaces
+    for lay in layers:
+        lin = lay["lin"]
+        bits = W.activations(lin, M)
+        lay["x"] = torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).cuda()
+        lay["y"] = torch.empty((M, lin.n_out), dtype=torch.float32, device="cuda")
+        lay["ws"] = lay["plan"].alloc_workspace(M)
+
+    stream = torch.cuda.Stream()
+
+    def step():
+        for lay in layers:
+            P.sdq_linear_forward(lay["plan"].handle, lay["tiled"], lay["alpha"], lay["x"], M,
+                                 lay["y"], lay["ws"], stream)
+
+    # eager warm-up, then capture one step in a CUDA graph
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            step()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        step()
+    torch.cuda.synchronize()
+
+    sampler = ClockSampler(dev)
+    sampler.start()
+    time.sleep(0.3)
+    for _ in range(max(3, args.warmup)):
+        graph.replay()
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_wall0 = time.time()
+    ev0.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(args.steps):
+            graph.replay()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    t_wall1 = time.time()
+    if dist:
+        dist.barrier()
+    ms_total = ev0.elapsed_time(ev1)
+    clocks = sampler.summary(t_wall0, t_wall1)
+    sampler.stop()
+    if dist:
+        t = torch.tensor([ms_total], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_total = float(t.item())
+    ms_step = ms_total / args.steps
+    value = code_bytes * world / (ms_step * 1e-3) / 1e9
+
+    # decode kernel alone: event-timed contraction launches (prep done before)
+    k_ms, k_bytes = 0.0, 0
+    per_lin = []
+    reps = 20
+    for lay in layers:
+        P.sdq_prep_activations(lay["plan"].handle, lay["x"], M, lay["ws"], stream)
+    torch.cuda.synchronize()
+    for rep in range(reps + 3):
+        for lay in layers:
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            P.sdq_contract(lay["plan"].handle, lay["tiled"], lay["alpha"], M, lay["y"], lay["ws"], stream)
+            b.record(stream)
+            lay.setdefault("ev", []).append((a, b)) if rep >= 3 else None
+    torch.cuda.synchronize()
+    for lay in layers:
+        d = sum(a.elapsed_time(b) for a, b in lay["ev"]) / len(lay["ev"])
+        ab = alg_bytes(lay, M)
+        per_lin.append({"linear": lay["lin"].name, "us": round(d * 1e3, 2),
+                        "GBps": round(ab / (d * 1e-3) / 1e9, 1)})
+        k_ms += d
+        k_bytes += ab
+    achieved = k_bytes / (k_ms * 1e-3) / 1e9
+    srcs = [os.path.join(ROOT, "paper_2510_03275_gb300", "csrc", f) for f in ("decode.cu", "common.cuh")]
+    traffic, _ = profile_traffic(srcs)
+
+    # end to end through the C ABI with host buffers (pinned), eager calls
+    e2e_steps = min(200, max(20, args.steps // 100))
+    hx = [lay["x"].cpu().pin_memory() for lay in layers]
+    hy = [torch.empty_like(lay["y"], device="cpu").pin_memory() for lay in layers]
+    h2d = sum(h.numel() * h.element_size() for h in hx)
+    d2h = sum(h.numel() * h.element_size() for h in hy)
+
+    def e2e_step():
+        for lay, xh, yh in zip(layers, hx, hy):
+            lay["x"].copy_(xh, non_blocking=True)
+            P.sdq_linear_forward(lay["plan"].handle, lay["tiled"], lay["alpha"], lay["x"], M,
+                                 lay["y"], lay["ws"], stream)
+            yh.copy_(lay["y"], non_blocking=True)
+
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            e2e_step()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        a.record(stream)
+        for _ in range(e2e_steps):
+            e2e_step()
+        b.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = a.elapsed_time(b) / e2e_steps
+    e2e_val = code_bytes * world / (e2e_ms * 1e-3) / 1e9
+
+    out = {
+        "metric": METRIC, "value": round(value, 1), "unit": "GB/s",
+        "n_gpus": world, "steps": args.steps, "warmup": max(3, args.warmup),
+        "ms_per_step": round(ms_step, 5), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "u2-codes/e4m3-mma/f32-acc", "data": "synthetic",
+        "config": {"workload": "llama70b-layer decode (cfg4): q/o 8192x8192, k/v 1024x8192, "
+                               "gate/up 28672x8192, down 8192x28672; OSR 2 ternary B=128"
+                               + (f" [only {args.linears}]" if args.linears else ""),
+                   "decode_batch": M, "code_bytes_per_step": code_bytes,
+                   "l2": "7 code matrices (428 MB) streamed in turn > 129 MB L2",
+                   "timing": "CUDA graph of one step, replayed; events on the launch stream",
+                   "parallelism": f"replicas x{world}"},
+        "clocks": clocks,
+        "e2e": {"value": round(e2e_val, 1), "unit": "GB/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms, 4),
+                "how": "eager sdq_linear_forward per linear with pinned-host x in and y out"},
+        "gpu_launches": 2 * len(layers) * args.steps,
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
+                     "unit": "GB/s", "frac": round(achieved / hbm, 4), "traffic": traffic,
+                     "kernel": "decode_kernel (sdq_contract, M<=64)", "peak_source": peak_src,
+                     "nominal_8tbs_frac": round(achieved / 8000.0, 4), "per_linear": per_lin},
+        "encode": {"ms_per_layer": round(enc_ms, 3), "what": "sdq_encode_rows + sdq_pack, 7 linears"},
+    }
+    if not args.no_extras and rank == 0:
+        out["decode_sweep"] = decode_sweep(P, W, torch, layers, stream)
+        out["prefill"] = prefill_leg(P, W, torch, layers, stream, tf_burst, tf_sus, peak_src)
+        out["cpu_baseline"] = cpu_baseline_leg()
+    return out
+
+
+def decode_sweep(P, W, torch, layers, stream):
+    import numpy as np
+    res = {}
+    for M in (1, 2, 4, 8, 16, 32, 64):
+        tot_b, tot_ms = 0, 0.0
+        for lay in layers:
+            lin = lay["lin"]
+            x = torch.from_numpy(W.activations(lin, M).view(np.int16)).view(torch.bfloat16).cuda()
+            y = torch.empty((M, lin.n_out), dtype=torch.float32, device="cuda")
+            ws = lay["plan"].alloc_workspace(M)
+            P.sdq_prep_activations(lay["plan"].handle, x, M, ws, stream)
+            for _ in range(3):
+                P.sdq_contract(lay["plan"].handle, lay["tiled"], lay["alpha"], M, y, ws, stream)
+            evs = []
+            for _ in range(10):
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                P.sdq_contract(lay["plan"].handle, lay["tiled"], lay["alpha"], M, y, ws, stream)
+                b.record(stream)
+                evs.append((a, b))
+            torch.cuda.synchronize()
+            tot_ms += sum(a.elapsed_time(b) for a, b in evs) / len(evs)
+            tot_b += lay["code_bytes"]
+        res[str(M)] = round(tot_b / (tot_ms * 1e-3) / 1e9, 1)
+    return {"unit": "weight GB/s (decode kernel, per batch size)", "values": res}
+
+
+def prefill_leg(P, W, torch, layers, stream, tf_burst, tf_sus, peak_src):
+    import numpy as np
+    M = 4096
+    flops, ms = 0, 0.0
+    try:
+        for lay in layers:
+            lin = lay["lin"]
+            x = torch.from_numpy(W.activations(lin, M).view(np.int16)).view(torch.bfloat16).cuda()
+            y = torch.empty((M, lin.n_out), dtype=torch.float32, device="cuda")
+            ws = lay["plan"].alloc_workspace(M)
+            P.sdq_prep_activations(lay["plan"].handle, x, M, ws, stream)
+            P.sdq_contract(lay["plan"].handle, lay["tiled"], lay["alpha"], M, y, ws, stream)
+            evs = []
+            for _ in range(5):
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                P.sdq_contract(lay["plan"].handle, lay["tiled"], lay["alpha"], M, y, ws, stream)
+                b.record(stream)
+                evs.append((a, b))
+            torch.cuda.synchronize()
+            ms += sum(a.elapsed_time(b) for a, b in evs) / len(evs)
+            flops += 2 * M * lin.n_out * lay["plan"].k_eff
+            del x, y, ws
+    except P.SdqError as e:
+        return {"unavailable": str(e)}
+    tflops = flops / (ms * 1e-3) / 1e12
+    return {"value": round(tflops, 1), "unit": "TFLOP/s", "M": M, "ms_per_layer": round(ms, 3),
+            "flops_per_layer": flops,
+            "roofline": {"bound": "tensor", "achieved": round(tflops, 1), "peak": tf_burst,
+                         "unit": "TFLOP/s", "frac": round(tflops / tf_burst, 4),
+                         "peak_source": peak_src + " bf16 burst"}}
+
+
+# -------------------------------------------------------- oracle (CPU) legs
+class OracleSample:
+    """Seeded inputs for the oracle's code-domain forward (decode, M=1) on
+    `rows` rows of every cfg4 linear, prepared once; `run()` times one pass."""
+
+    def __init__(self, rows):
+        import numpy as np
+
+        from paper_2510_03275_gb300 import workloads as W
+        cfg = W.config(4)
+        self.items = []
+        self.nbytes = 0
+        for lin in cfg.linears:
+            nb = cfg.n_b(lin)
+            keff = lin.k_in // cfg.block * nb
+            codes = W.random_codes(rows, keff, cfg.quantizer, seed=lin.seed)
+            alpha = np.full(rows, 0.02, dtype=np.float32)
+            x = W.bf16_to_float(W.activations(lin, 1))
+            self.items.append((x, codes, alpha, cfg.block, nb, W.hadamard_signs(lin, cfg.block)))
+            self.nbytes += rows * keff * 2 // 8
+
+    def run(self):
+        import oracle as O
+        t0 = time.perf_counter()
+        for x, codes, alpha, block, nb, signs in self.items:
+            O.forward_code_domain(x, codes, alpha, block, nb, signs)
+        return time.perf_counter() - t0
+
+
+def _cores():
+    return len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+
+
+def cpu_baseline_leg(sample_rows=256, min_secs=10.0):
+    """The oracle timed on the host cores: repeated passes over a bounded
+    sample until about `min_secs` of CPU work."""
+    smp = OracleSample(sample_rows)
+    secs, passes = 0.0, 0
+    while secs < min_secs:
+        secs += smp.run()
+        passes += 1
+    cores = _cores()
+    return {"value": round(smp.nbytes * passes / secs / 1e9, 4), "unit": "GB/s", "cores": cores,
+            "kind": "oracle",
+            "sample": f"oracle forward_code_domain (fp64 numpy), decode M=1, {sample_rows} rows of "
+                      f"each of the 7 cfg4 linears ({smp.nbytes} code bytes) x {passes} passes = "
+                      f"{secs:.1f} s; numpy default threads on {cores} host cores"}
+
+
+def run_reference(args, rank, world):
+    """The oracle as the reference arm: each step is the code-domain forward on
+    a bounded row sample of every cfg4 linear (GB/s of codes processed)."""
+    if rank != 0:
+        return None
+    rows = 64 if args.steps <= 2000 else 16
+    smp = OracleSample(rows)
+    warm = max(3, args.warmup)
+    for _ in range(warm):
+        smp.run()
+    secs = 0.0
+    for _ in range(args.steps):
+        secs += smp.run()
+    val = smp.nbytes * args.steps / secs / 1e9
+    cores = _cores()
+    return {"impl": "reference", "metric": METRIC, "value": round(val, 4), "unit": "GB/s",
+            "n_gpus": world, "steps": args.steps, "warmup": warm,
+            "ms_per_step": round(secs / args.steps * 1e3, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": "llama70b-layer decode (cfg4), M=1; oracle on a bounded "
+                                   f"sample of {rows} rows per linear per step"},
+            "cpu_baseline": {"value": round(val, 4), "unit": "GB/s", "cores": cores,
+                             "kind": "oracle",
+                             "sample": f"{rows} rows of each of the 7 cfg4 linears per step"},
+            "e2e": {"value": round(val, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch
+        import torch.distributed as td
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if torch.cuda.is_available():
+            torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+        td.init_process_group(backend)
+        dist = td
+    if args.impl == "reference":
+        out = run_reference(args, rank, world)
+    else:
+        out = run_sdq(args, rank, world, dist)
+    if rank == 0 and out is not None:
+        print(json.dumps(out))
+    if dist:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -160,9 +160,11 @@ int sdq_unpack(sdq_plan plan, const uint32_t* codes_tiled, uint32_t* codes_plain
 
 /* x_tilde = G x_b for every block b of every row of x (device, bf16 bits,
  * M x k_in row-major), written into the workspace `ws` for sdq_contract.
- * For M <= 64 x_tilde is kept in fp32 (the decode path re-encodes it as a
- * three-/two-term fp8 expansion inside the contraction kernel); for M > 64
- * it is written in bf16 in the permuted K order the prefill kernel reads. */
+ * For M <= 64 x_tilde is kept in fp32 and, by a second kernel, as the fp8
+ * B-operand fragments of the decode MMAs (a three-term e4m3 expansion of
+ * x_tilde * s for M <= 2, two-term above; s a power of two per batch row);
+ * for M > 64 it is written in bf16 in the permuted K order the prefill kernel
+ * reads.  Kernels are launched with programmatic dependent launch. */
 int sdq_prep_activations(sdq_plan plan, const uint16_t* x, int32_t M,
                          void* ws, size_t ws_bytes, void* stream);
 
@@ -178,6 +180,13 @@ int sdq_contract(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha,
 int sdq_linear_forward(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha,
                        const uint16_t* x, int32_t M, float* y, void* ws, size_t ws_bytes,
                        void* stream);
+
+/* Wait for `stream`, then report whether the last decode call that used
+ * `ws` (same plan and M) completed its bounded device-side waits: SDQ_OK or
+ * SDQ_ERR_TIMEOUT (a TMA copy did not arrive within about 2 s; the output of
+ * that call is invalid).  Prepare calls reset the flag.  For M > 64 this only
+ * synchronizes the stream. */
+int sdq_workspace_status(sdq_plan plan, int32_t M, const void* ws, void* stream);
 
 /* Copy x_tilde for M <= 64 out of the workspace as fp32 (M x K_eff,
  * device), for checking sdq_prep_activations. */

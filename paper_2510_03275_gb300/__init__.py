@@ -23,6 +23,7 @@ __all__ = [
     "sdq_plan_create", "sdq_plan_destroy", "sdq_k_eff", "sdq_plain_bytes", "sdq_tiled_bytes",
     "sdq_workspace_bytes", "sdq_build_tables", "sdq_encode_rows", "sdq_pack", "sdq_unpack",
     "sdq_prep_activations", "sdq_contract", "sdq_linear_forward", "sdq_read_prep",
+    "sdq_workspace_status",
     "sdq_status_string", "Plan",
 ]
 
@@ -87,6 +88,7 @@ _SIGS = {
     "sdq_contract": (ctypes.c_int, [_vp, _vp, _vp, _i32, _vp, _vp, _sz, _vp]),
     "sdq_linear_forward": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _vp, _vp, _sz, _vp]),
     "sdq_read_prep": (ctypes.c_int, [_vp, _i32, _vp, _vp, _vp]),
+    "sdq_workspace_status": (ctypes.c_int, [_vp, _i32, _vp, _vp]),
     "sdq_status_string": (ctypes.c_char_p, [ctypes.c_int]),
 }
 
@@ -202,6 +204,11 @@ def sdq_linear_forward(plan, codes_tiled, alpha, x, M, y, ws, stream=None):
 
 def sdq_read_prep(plan, M, ws, out, stream=None):
     _check(lib().sdq_read_prep(plan, M, _ptr(ws), _ptr(out), _stream(stream)), "sdq_read_prep")
+
+
+def sdq_workspace_status(plan, M, ws, stream=None) -> int:
+    """Synchronize and return the status of the last decode using ``ws``."""
+    return lib().sdq_workspace_status(plan, M, _ptr(ws), _stream(stream))
 
 
 def sdq_status_string(status: int) -> str:

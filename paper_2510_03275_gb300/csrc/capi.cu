@@ -42,13 +42,18 @@ WsLayout workspace_layout(const sdq_plan_s* pl, int M) {
     off = align_up(off + sizeof(float) * (size_t)M * g.k_eff_pad, 256);
     L.pmax = off;
     off = align_up(off + sizeof(float) * (size_t)M * dc.P, 256);
+    L.frag = off;
+    off = align_up(off + (size_t)(g.k_eff_pad / 32) * dc.NT * 32 * 16, 256);
+    L.scale = off;
+    off = align_up(off + sizeof(float) * kMaxDecodeM, 256);
     L.part = off;
     off = align_up(off + (dc.S > 1 ? sizeof(float) * (size_t)dc.S * M * g.ng * 16 : 0), 256);
-    L.cnt = off;
-    off = align_up(off + sizeof(uint32_t) * (size_t)dc.R, 256);
+    L.cnt = off;                                   // R counters, then the error word
+    L.err = off + sizeof(uint32_t) * (size_t)dc.R;
+    off = align_up(off + sizeof(uint32_t) * ((size_t)dc.R + 1), 256);
   } else {
     off = align_up(off + sizeof(uint16_t) * (size_t)M * g.k_eff_pad, 256);
-    L.pmax = L.part = L.cnt = off;
+    L.pmax = L.frag = L.scale = L.part = L.cnt = L.err = off;
   }
   L.total = off;
   return L;
@@ -152,7 +157,9 @@ extern "C" int sdq_prep_activations(sdq_plan p, const uint16_t* x, int32_t M, vo
   int st = check_ws(p, M, ws, ws_bytes);
   if (st != SDQ_OK) return st;
   if (!x || !aligned16(x)) return SDQ_ERR_INVALID_ARG;
-  return cuda_status(launch_prep(p, x, M, ws, (cudaStream_t)stream));
+  cudaError_t e = launch_prep(p, x, M, ws, (cudaStream_t)stream);
+  if (e == cudaSuccess && M <= kMaxDecodeM) e = launch_frag(p, M, ws, (cudaStream_t)stream);
+  return cuda_status(e);
 }
 
 extern "C" int sdq_contract(sdq_plan p, const uint32_t* codes_tiled, const float* alpha, int32_t M,
@@ -173,6 +180,21 @@ extern "C" int sdq_linear_forward(sdq_plan p, const uint32_t* codes_tiled, const
   int st = sdq_prep_activations(p, x, M, ws, ws_bytes, stream);
   if (st != SDQ_OK) return st;
   return sdq_contract(p, codes_tiled, alpha, M, y, ws, ws_bytes, stream);
+}
+
+extern "C" int sdq_workspace_status(sdq_plan p, int32_t M, const void* ws, void* stream) {
+  if (!p || M < 1 || M > 65535 || !ws) return SDQ_ERR_INVALID_ARG;
+  if (M > kMaxDecodeM) {
+    cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+    return cuda_status(e);
+  }
+  const WsLayout L = workspace_layout(p, M);
+  uint32_t err = 0;
+  cudaError_t e = cudaMemcpyAsync(&err, static_cast<const uint8_t*>(ws) + L.err, sizeof(err),
+                                  cudaMemcpyDeviceToHost, (cudaStream_t)stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize((cudaStream_t)stream);
+  if (e != cudaSuccess) return SDQ_ERR_CUDA;
+  return err ? SDQ_ERR_TIMEOUT : SDQ_OK;
 }
 
 extern "C" int sdq_read_prep(sdq_plan p, int32_t M, const void* ws, float* xt_out, void* stream) {

@@ -8,18 +8,18 @@
 // x is bf16 (exact), G is split into bf16 hi + lo parts (relative error of
 // the pair ~2^-16), accumulation in fp32.
 //
-// Output, decode path (M <= 64): fp32 x_tilde (M x K_eff_pad) plus, per CTA,
-// max |x_tilde| for each batch row (the decode kernel turns these into the
-// power-of-two scale of its fp8 expansion).  Prefill path: bf16 x_tilde in
-// the permuted 64-code stage order of the prefill kernel's operand tiles.
+// Decode path (M <= 64): fp32 x_tilde (M x K_eff_pad) plus max |x_tilde|
+// per CTA and batch row; then the fragment kernel below turns x_tilde into
+// the bf16 B-operand fragments of the decode MMAs (hi and lo bf16 terms for
+// M <= 16, hi only above).  Prefill path: bf16 x_tilde in the permuted
+// 64-code stage order of the prefill kernel's operand tiles.
 #include "common.cuh"
 
 namespace sdq {
 
 namespace {
 
-constexpr int kTile = 64;   // rows (blocks b) and columns (samples j) per CTA
-constexpr int kKC = 32;     // k per smem stage
+constexpr int kKC = 32;       // k per smem stage
 constexpr int kLd = kKC + 8;  // padded bf16 row stride
 
 struct PrepParams {
@@ -29,50 +29,79 @@ struct PrepParams {
   float* xt;          // decode: fp32 M x kpad
   uint16_t* xtb;      // prefill: bf16 M x kpad (permuted)
   float* pmax;        // decode: M x P
-  uint32_t* cnt;      // decode counters to zero
+  uint32_t* cnt;      // decode counters and error word to zero
   int ncnt;
   int M, K, B, n_b, nblk, P, JT;
   int64_t k_eff, kpad;
-  int prefill;
+  int prefill, vec;
 };
 
+// CTA tile: TB blocks (rows) x 64 samples j, 4 warps.  TB = 64: each warp
+// owns 16 rows x 64 j; TB = 16: each warp owns the 16 rows x 16 j.
+template <int TB>
 __global__ void __launch_bounds__(128) prep_kernel(PrepParams p) {
-  __shared__ __align__(16) uint16_t xs[kTile * kLd];
-  __shared__ __align__(16) uint16_t ghs[kTile * kLd];
-  __shared__ __align__(16) uint16_t gls[kTile * kLd];
+  constexpr int NTW = TB == 64 ? 8 : 2;   // 8-column MMA tiles per warp
+  __shared__ __align__(16) uint16_t xs[TB * kLd];
+  __shared__ __align__(16) uint16_t ghs[64 * kLd];
+  __shared__ __align__(16) uint16_t gls[64 * kLd];
   __shared__ float red[4];
+  pdl_wait();
+  pdl_launch_dependents();
   const int jt = blockIdx.x, bt = blockIdx.y, m = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t = lane & 3;
-  const int b0 = bt * kTile, j0 = jt * kTile;
+  const int b0 = bt * TB, j0 = jt * 64;
+  const int wrow = TB == 64 ? warp * 16 : 0;       // warp's first row in the tile
+  const int wcol = TB == 64 ? 0 : warp * 16;       // warp's first column
 
-  float acc[8][4];
+  float acc[NTW][4];
 #pragma unroll
-  for (int n = 0; n < 8; ++n)
+  for (int n = 0; n < NTW; ++n)
 #pragma unroll
     for (int e = 0; e < 4; ++e) acc[n][e] = 0.f;
 
   for (int kc = 0; kc < p.B; kc += kKC) {
-    // Stage x rows (blocks) and G rows (samples), k in [kc, kc + 32).
-    for (int i = tid; i < kTile * kKC; i += 128) {
-      const int rr = i / kKC, kk = i - rr * kKC, k = kc + kk;
-      const int b = b0 + rr, j = j0 + rr;
-      xs[rr * kLd + kk] = (b < p.nblk && k < p.B) ? p.x[(size_t)m * p.K + (size_t)b * p.B + k] : 0;
-      const bool gv = j < p.n_b && k < p.B;
-      ghs[rr * kLd + kk] = gv ? p.g_hi[(size_t)j * p.B + k] : 0;
-      gls[rr * kLd + kk] = gv ? p.g_lo[(size_t)j * p.B + k] : 0;
+    if (p.vec) {  // 16-byte loads: B % 32 == 0, rows 16-byte aligned
+      for (int i = tid; i < TB * 4; i += 128) {
+        const int rr = i >> 2, q = i & 3, b = b0 + rr;
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (b < p.nblk)
+          v = *reinterpret_cast<const uint4*>(p.x + (size_t)m * p.K + (size_t)b * p.B + kc + 8 * q);
+        *reinterpret_cast<uint4*>(xs + rr * kLd + 8 * q) = v;
+      }
+      for (int i = tid; i < 64 * 4; i += 128) {
+        const int rr = i >> 2, q = i & 3, j = j0 + rr;
+        uint4 vh = make_uint4(0, 0, 0, 0), vl = vh;
+        if (j < p.n_b) {
+          vh = *reinterpret_cast<const uint4*>(p.g_hi + (size_t)j * p.B + kc + 8 * q);
+          vl = *reinterpret_cast<const uint4*>(p.g_lo + (size_t)j * p.B + kc + 8 * q);
+        }
+        *reinterpret_cast<uint4*>(ghs + rr * kLd + 8 * q) = vh;
+        *reinterpret_cast<uint4*>(gls + rr * kLd + 8 * q) = vl;
+      }
+    } else {
+      for (int i = tid; i < TB * kKC; i += 128) {
+        const int rr = i / kKC, kk = i - rr * kKC, k = kc + kk, b = b0 + rr;
+        xs[rr * kLd + kk] = (b < p.nblk && k < p.B) ? p.x[(size_t)m * p.K + (size_t)b * p.B + k] : 0;
+      }
+      for (int i = tid; i < 64 * kKC; i += 128) {
+        const int rr = i / kKC, kk = i - rr * kKC, k = kc + kk, j = j0 + rr;
+        const bool gv = j < p.n_b && k < p.B;
+        ghs[rr * kLd + kk] = gv ? p.g_hi[(size_t)j * p.B + k] : 0;
+        gls[rr * kLd + kk] = gv ? p.g_lo[(size_t)j * p.B + k] : 0;
+      }
     }
     __syncthreads();
 #pragma unroll
     for (int ks = 0; ks < kKC; ks += 16) {
       uint32_t a[4];
-      const uint16_t* ar = xs + (warp * 16 + g) * kLd + ks + 2 * t;
+      const uint16_t* ar = xs + (wrow + g) * kLd + ks + 2 * t;
       a[0] = *reinterpret_cast<const uint32_t*>(ar);
       a[1] = *reinterpret_cast<const uint32_t*>(ar + 8 * kLd);
       a[2] = *reinterpret_cast<const uint32_t*>(ar + 8);
       a[3] = *reinterpret_cast<const uint32_t*>(ar + 8 * kLd + 8);
 #pragma unroll
-      for (int n = 0; n < 8; ++n) {
-        const int off = (n * 8 + g) * kLd + ks + 2 * t;
+      for (int n = 0; n < NTW; ++n) {
+        const int off = (wcol + n * 8 + g) * kLd + ks + 2 * t;
         const uint32_t h0 = *reinterpret_cast<const uint32_t*>(ghs + off);
         const uint32_t h1 = *reinterpret_cast<const uint32_t*>(ghs + off + 8);
         const uint32_t l0 = *reinterpret_cast<const uint32_t*>(gls + off);
@@ -86,11 +115,11 @@ __global__ void __launch_bounds__(128) prep_kernel(PrepParams p) {
 
   float vmax = 0.f;
 #pragma unroll
-  for (int n = 0; n < 8; ++n)
+  for (int n = 0; n < NTW; ++n)
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
-      const int b = b0 + warp * 16 + g + (e >> 1) * 8;
-      const int j = j0 + n * 8 + 2 * t + (e & 1);
+      const int b = b0 + wrow + g + (e >> 1) * 8;
+      const int j = j0 + wcol + n * 8 + 2 * t + (e & 1);
       if (b < p.nblk && j < p.n_b) {
         const int64_t kk = (int64_t)b * p.n_b + j;
         const float v = acc[n][e];
@@ -126,6 +155,54 @@ __global__ void __launch_bounds__(128) prep_kernel(PrepParams p) {
   }
 }
 
+// ------------------------------------------------------- bf16 fragments
+// B operand of the decode MMAs, in the order one lane reads it: entry
+// (k-step ks, column tile nt, lane (g, t)) is a uint4 of bf16 pairs
+//   .x = (xt[4t+1], xt[4t+3])        .y = (xt[16+4t+1], xt[16+4t+3])
+//   .z = (xt[4t],   xt[4t+2])        .w = (xt[16+4t],   xt[16+4t+2])
+// (offsets from 32 ks) of column n = 8 nt + g = (batch m, term): term 0 is
+// bf16(xt), term 1 is bf16(xt - term 0).  This is the k order implied by the
+// shift-and-mask expansion of the tiled code words.
+struct FragParams {
+  const float* xt;
+  uint4* frag;
+  float* scale;
+  int M, T, NT;
+  int64_t kpad, total;
+};
+
+__device__ __forceinline__ uint32_t bf16_term(float v, int term) {
+  const uint32_t hi = float_to_bf16_bits(v);
+  if (term == 0) return hi;
+  return float_to_bf16_bits(v - bf16_bits_to_float((uint16_t)hi));
+}
+
+__device__ __forceinline__ uint32_t bf16_pair(const float* xr, int i0, int i1, int term) {
+  return bf16_term(xr[i0], term) | (bf16_term(xr[i1], term) << 16);
+}
+
+__global__ void __launch_bounds__(256) frag_kernel(FragParams p) {
+  pdl_wait();
+  pdl_launch_dependents();
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx < p.M && blockIdx.x == 0) p.scale[idx] = 1.f;
+  if (idx >= p.total) return;
+  const int ln = (int)(idx & 31);
+  const int nt = (int)((idx >> 5) % p.NT);
+  const int64_t ks = idx / (32 * p.NT);
+  const int g = ln >> 2, t = ln & 3, n = nt * 8 + g;
+  uint4 v = make_uint4(0, 0, 0, 0);
+  if (n < p.M * p.T) {
+    const int m = n / p.T, term = n - m * p.T;
+    const float* xr = p.xt + (size_t)m * p.kpad + ks * 32 + 4 * t;
+    v.x = bf16_pair(xr, 1, 3, term);
+    v.y = bf16_pair(xr, 17, 19, term);
+    v.z = bf16_pair(xr, 0, 2, term);
+    v.w = bf16_pair(xr, 16, 18, term);
+  }
+  p.frag[idx] = v;
+}
+
 }  // namespace
 
 cudaError_t launch_prep(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws, cudaStream_t st) {
@@ -139,20 +216,46 @@ cudaError_t launch_prep(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws
   p.xtb = p.prefill ? reinterpret_cast<uint16_t*>(base + L.xt) : nullptr;
   p.M = M; p.K = g.k_in; p.B = g.block; p.n_b = g.n_b; p.nblk = g.nblk;
   p.k_eff = g.k_eff; p.kpad = g.k_eff_pad;
-  p.JT = (g.n_b + kTile - 1) / kTile;
-  const int BT = (g.nblk + kTile - 1) / kTile;
+  p.vec = (g.block % 32 == 0) && ((reinterpret_cast<uintptr_t>(x) & 15u) == 0);
+  const bool small = (int64_t)M * g.nblk < 4 * (int64_t)pl->sm_count;
+  const int TB = small ? 16 : 64;
+  p.JT = (g.n_b + 63) / 64;
+  const int BT = (g.nblk + TB - 1) / TB;
   p.P = p.JT * BT;
   if (p.prefill) {
     p.pmax = nullptr; p.cnt = nullptr; p.ncnt = 0;
   } else {
-    const DecodeConfig dc = decode_config(pl, M);
+    const DecodeConfig& dc = decode_config(pl, M);
     p.pmax = reinterpret_cast<float*>(base + L.pmax);
     p.cnt = reinterpret_cast<uint32_t*>(base + L.cnt);
-    p.ncnt = dc.R;
+    p.ncnt = dc.R + 1;   // the counters and the error word that follows them
   }
   dim3 grid(p.JT, BT, M);
-  prep_kernel<<<grid, 128, 0, st>>>(p);
-  return cudaGetLastError();
+  return small ? launch_pdl(prep_kernel<16>, grid, dim3(128), 0, st, p)
+               : launch_pdl(prep_kernel<64>, grid, dim3(128), 0, st, p);
+}
+
+int prep_partials(const sdq_plan_s* pl, int M) {
+  const Geometry& g = pl->geo;
+  const bool small = (int64_t)M * g.nblk < 4 * (int64_t)pl->sm_count;
+  const int TB = small ? 16 : 64;
+  return ((g.n_b + 63) / 64) * ((g.nblk + TB - 1) / TB);
+}
+
+cudaError_t launch_frag(const sdq_plan_s* pl, int M, void* ws, cudaStream_t st) {
+  const Geometry& g = pl->geo;
+  const WsLayout L = workspace_layout(pl, M);
+  const DecodeConfig& dc = decode_config(pl, M);
+  uint8_t* base = static_cast<uint8_t*>(ws);
+  FragParams p;
+  p.xt = reinterpret_cast<const float*>(base + L.xt);
+  p.frag = reinterpret_cast<uint4*>(base + L.frag);
+  p.scale = reinterpret_cast<float*>(base + L.scale);
+  p.M = M; p.T = dc.T; p.NT = dc.NT;
+  p.kpad = g.k_eff_pad;
+  p.total = (g.k_eff_pad / 32) * dc.NT * 32;
+  const int64_t blocks = (p.total + 255) / 256;
+  return launch_pdl(frag_kernel, dim3((unsigned)blocks), dim3(256), 0, st, p);
 }
 
 }  // namespace sdq

@@ -29,8 +29,9 @@ int validate(const sdq_layer_desc* d, Geometry* g);
 //   g:     n_b x B row-major, G[j][k]     = fp32(sum_k' Dt[j][k'] Had[k][k'])
 int build_tables(const sdq_layer_desc* d, const int8_t* signs, float* a_enc, float* g);
 
-// Decode-path term count and MMA column tiles for batch M.
-inline int decode_terms(int M) { return M <= 2 ? 3 : 2; }
+// Decode-path terms per activation (bf16 hi + lo below 17 rows, hi only
+// above) and 8-column MMA tiles for batch M.
+inline int decode_terms(int M) { return M <= 16 ? 2 : 1; }
 inline int decode_ntiles(int M) { return (M * decode_terms(M) + 7) / 8; }
 
 constexpr int kMaxDecodeM = 64;
