@@ -181,11 +181,11 @@ int sdq_linear_forward(sdq_plan plan, const uint32_t* codes_tiled, const float* 
                        const uint16_t* x, int32_t M, float* y, void* ws, size_t ws_bytes,
                        void* stream);
 
-/* Wait for `stream`, then report whether the last decode call that used
+/* Wait for `stream`, then report whether the last contraction that used
  * `ws` (same plan and M) completed its bounded device-side waits: SDQ_OK or
  * SDQ_ERR_TIMEOUT (a TMA copy did not arrive within about 2 s; the output of
- * that call is invalid).  Prepare calls reset the flag.  For M > 64 this only
- * synchronizes the stream. */
+ * that call is invalid).  Prepare calls reset the flag.  Covers both the
+ * decode (M <= 64) and the prefill (M > 64) kernels. */
 int sdq_workspace_status(sdq_plan plan, int32_t M, const void* ws, void* stream);
 
 /* Copy x_tilde for M <= 64 out of the workspace as fp32 (M x K_eff,

@@ -53,7 +53,8 @@ WsLayout workspace_layout(const sdq_plan_s* pl, int M) {
     off = align_up(off + sizeof(uint32_t) * ((size_t)dc.R + 1), 256);
   } else {
     off = align_up(off + sizeof(uint16_t) * (size_t)M * g.k_eff_pad, 256);
-    L.pmax = L.frag = L.scale = L.part = L.cnt = L.err = off;
+    L.pmax = L.frag = L.scale = L.part = L.cnt = L.err = off;   // error word only
+    off = align_up(off + sizeof(uint32_t), 256);
   }
   L.total = off;
   return L;
@@ -184,10 +185,6 @@ extern "C" int sdq_linear_forward(sdq_plan p, const uint32_t* codes_tiled, const
 
 extern "C" int sdq_workspace_status(sdq_plan p, int32_t M, const void* ws, void* stream) {
   if (!p || M < 1 || M > 65535 || !ws) return SDQ_ERR_INVALID_ARG;
-  if (M > kMaxDecodeM) {
-    cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
-    return cuda_status(e);
-  }
   const WsLayout L = workspace_layout(p, M);
   uint32_t err = 0;
   cudaError_t e = cudaMemcpyAsync(&err, static_cast<const uint8_t*>(ws) + L.err, sizeof(err),

@@ -17,7 +17,7 @@
 // epilogue adds the terms and applies alpha / 2.
 //
 // Memory path: every warp streams its own sequence of 512-byte code tiles
-// (16 rows x 128 / 256 codes) through a private ring of kStages shared-memory
+// (16 rows x 128 / 256 codes) through a private ring of shared-memory
 // slots filled with cp.async (16 bytes per lane, one commit group per tile),
 // so each SM keeps ~64 KB of loads in flight without holding them in
 // registers.  The CTA's slice of B-fragments arrives by one 1-D TMA bulk
@@ -36,7 +36,9 @@ namespace sdq {
 
 namespace {
 
-constexpr int kStages = 8;   // cp.async ring slots per warp (512-byte tiles)
+// Occupancy and cp.async ring depth (512-byte tiles per warp) by column tiles.
+__host__ __device__ constexpr int ctas_per_sm(int NT) { return NT == 1 ? 3 : (NT <= 4 ? 2 : 1); }
+__host__ __device__ constexpr int ring_depth(int NT) { return NT == 1 ? 6 : (NT <= 4 ? 8 : 4); }
 
 struct DecodeParams {
   const uint32_t* codes;
@@ -59,7 +61,7 @@ struct DecodeParams {
 // Binary word: ((~w << j) & 0x80008000) | 0x40004000, j = 0..15, four MMAs.
 template <int QT, int NT, int QA>
 __device__ __forceinline__ void mma_tile(float (&acc)[QA][NT][4], const uint32_t (&wq)[4],
-                                         const uint4* bf) {
+                                         const uint4* bf, int lanes, bool active) {
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     const uint32_t w = wq[q];
@@ -71,7 +73,7 @@ __device__ __forceinline__ void mma_tile(float (&acc)[QA][NT][4], const uint32_t
         for (int j = 0; j < 4; ++j) a[j] = (w << (2 * (4 * h + j))) & 0xC000C000u;
 #pragma unroll
         for (int n = 0; n < NT; ++n) {
-          const uint4 b = bf[(q * NT + n) * 32];
+          const uint4 b = active ? bf[(q * NT + n) * lanes] : make_uint4(0, 0, 0, 0);
           mma_bf16_16816(acc[(2 * q + h) % QA][n], a, h ? b.z : b.x, h ? b.w : b.y);
         }
       }
@@ -85,7 +87,7 @@ __device__ __forceinline__ void mma_tile(float (&acc)[QA][NT][4], const uint32_t
 #pragma unroll
         for (int n = 0; n < NT; ++n) {
           // h = 0, 1: odd fields (k-steps 2q, 2q + 1); h = 2, 3: even fields
-          const uint4 b = bf[((2 * q + (h & 1)) * NT + n) * 32];
+          const uint4 b = active ? bf[((2 * q + (h & 1)) * NT + n) * lanes] : make_uint4(0, 0, 0, 0);
           mma_bf16_16816(acc[(4 * q + h) % QA][n], a, (h >> 1) ? b.z : b.x, (h >> 1) ? b.w : b.y);
         }
       }
@@ -101,10 +103,10 @@ template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
 
 template <int QT, int NT>
-__global__ void __launch_bounds__(256, NT <= 4 ? 2 : 1) decode_kernel(DecodeParams p) {
+__global__ void __launch_bounds__(256, ctas_per_sm(NT)) decode_kernel(DecodeParams p) {
   constexpr int KS = QT == 2 ? 4 : 8;                  // 32-code k-steps per chunk
   constexpr int QA = NT == 1 ? 4 : (NT == 2 ? 2 : 1);  // independent accumulator sets
-  constexpr int D = kStages;                           // ring slots per warp
+  constexpr int D = ring_depth(NT);                    // ring slots per warp
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ __align__(8) uint64_t frag_bar;
   __shared__ float scale_s[kMaxDecodeM];
@@ -117,7 +119,9 @@ __global__ void __launch_bounds__(256, NT <= 4 ? 2 : 1) decode_kernel(DecodePara
   const int nc = c1 - c0;                                  // tiles per row group
   uint8_t* ring = smem + (size_t)warp * D * 512;          // [8 warps][D][512 B]
   uint4* bfrag = reinterpret_cast<uint4*>(smem + 8 * D * 512);
-  float* wb = reinterpret_cast<float*>(smem + 8 * D * 512 + (size_t)p.cps * KS * NT * 32 * 16) +
+  // With one column tile only the lanes of the used columns carry fragments.
+  const int flanes = NT == 1 ? 4 * p.M * p.T : 32;
+  float* wb = reinterpret_cast<float*>(smem + 8 * D * 512 + (size_t)p.cps * KS * NT * flanes * 16) +
               (size_t)warp * 16 * 8 * NT;
 
   if (tid == 0) {
@@ -134,16 +138,21 @@ __global__ void __launch_bounds__(256, NT <= 4 ? 2 : 1) decode_kernel(DecodePara
   // grid waits.
   const int n_rg_w = rg1 - rg0 - warp > 0 ? (rg1 - rg0 - warp + 7) / 8 : 0;
   const int total = n_rg_w * nc;
-  const uint8_t* cbase = reinterpret_cast<const uint8_t*>(
+  const uint8_t* src = reinterpret_cast<const uint8_t*>(
       p.codes + ((size_t)(rg0 + warp) * p.n_chunks + c0) * 128) + 16 * lane;
-  const size_t rg_step = (size_t)8 * p.n_chunks * 512;    // bytes between this warp's row groups
-  int ld_rg = 0, ld_ci = 0, ld_t = 0;                      // next tile to request
+  const size_t rg_jump = (size_t)8 * p.n_chunks * 512 - (size_t)nc * 512;
+  uint8_t* dst = ring + 16 * lane;
+  uint8_t* const ring_end = ring + D * 512;
+  int ld_ci = 0, ld_t = 0;                                 // next tile to request
   auto request = [&]() {
     if (ld_t < total) {
-      cp_async16(ring + (ld_t % D) * 512 + 16 * lane, cbase + ld_rg * rg_step + (size_t)ld_ci * 512);
-      if (++ld_ci == nc) { ld_ci = 0; ++ld_rg; }
+      cp_async16(dst, src);
+      src += 512;
+      if (++ld_ci == nc) { ld_ci = 0; src += rg_jump; }
     }
     ++ld_t;
+    dst += 512;
+    if (dst == ring_end + 16 * lane) dst = ring + 16 * lane;
     cp_async_commit();
   };
 #pragma unroll 1
@@ -151,10 +160,10 @@ __global__ void __launch_bounds__(256, NT <= 4 ? 2 : 1) decode_kernel(DecodePara
 
   // bf16 B-fragments (written by the fragment kernel) by one bulk copy.
   pdl_wait();
-  const uint32_t frag_bytes = (uint32_t)(nc * KS * NT * 32 * 16);
+  const uint32_t frag_bytes = (uint32_t)(nc * KS * NT * flanes * 16);
   if (tid == 0) {
     mbar_expect_tx(&frag_bar, frag_bytes);
-    bulk_g2s(bfrag, p.frag + (size_t)c0 * KS * NT * 32, frag_bytes, &frag_bar);
+    bulk_g2s(bfrag, p.frag + (size_t)c0 * KS * NT * flanes, frag_bytes, &frag_bar);
   }
   if (tid < p.M) scale_s[tid] = p.scale[tid];
   const bool ok = mbar_wait(&frag_bar, 0);
@@ -171,15 +180,20 @@ __global__ void __launch_bounds__(256, NT <= 4 ? 2 : 1) decode_kernel(DecodePara
 #pragma unroll
       for (int e = 0; e < 4; ++e) acc[a][n][e] = 0.f;
   int ci = 0, it = 0;
+  const bool active = lane < flanes;
+  const uint32_t* rd = reinterpret_cast<const uint32_t*>(ring) + lane;
+  const uint32_t* const rd_end = reinterpret_cast<const uint32_t*>(ring_end) + lane;
+  const uint4* bfl = bfrag + (active ? lane : 0);
 #pragma unroll 1
   for (int t = 0; t < total; ++t) {
     __syncwarp();        // every lane has consumed the slot refilled next
     request();           // tile t + D - 1 into slot (t - 1) % D
     cp_async_wait<D - 1>();
     __syncwarp();        // the other lanes' copies of tile t are visible
-    const uint32_t* tw = reinterpret_cast<const uint32_t*>(ring + (t % D) * 512) + lane;
-    const uint32_t wq[4] = {tw[0], tw[32], tw[64], tw[96]};
-    mma_tile<QT, NT, QA>(acc, wq, bfrag + (size_t)ci * KS * NT * 32 + lane);
+    const uint32_t wq[4] = {rd[0], rd[32], rd[64], rd[96]};
+    rd += 128;
+    if (rd == rd_end) rd = reinterpret_cast<const uint32_t*>(ring) + lane;
+    mma_tile<QT, NT, QA>(acc, wq, bfl + (size_t)ci * KS * NT * flanes, flanes, active);
     if (++ci == nc) {
       // Row group done: fold, stage in the warp's smem slot, combine the
       // terms of every batch row, write y (or the slice partial).
@@ -266,13 +280,14 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
   dc.WK = 1;
   dc.WR = 8;
   const int KS = g.kc / 32;
-  const size_t frag_per_chunk = (size_t)KS * dc.NT * 32 * 16;
-  const size_t fixed = (size_t)8 * kStages * 512 + (size_t)8 * 16 * 8 * dc.NT * 4 + 1024;
-  const int ctas_per_sm = dc.NT <= 4 ? 2 : 1;   // matches __launch_bounds__
-  const size_t budget = (size_t)(ctas_per_sm == 2 ? 110 : 220) * 1024;
+  const int flanes = dc.NT == 1 ? 4 * M * dc.T : 32;
+  const size_t frag_per_chunk = (size_t)KS * dc.NT * flanes * 16;
+  const int cpsm = ctas_per_sm(dc.NT);
+  const size_t fixed = (size_t)8 * ring_depth(dc.NT) * 512 + (size_t)8 * 16 * 8 * dc.NT * 4 + 1024;
+  const size_t budget = (size_t)(cpsm == 3 ? 72 : cpsm == 2 ? 110 : 220) * 1024;
   int max_cps = (int)((budget - fixed) / frag_per_chunk);
   if (max_cps < 1) max_cps = 1;
-  const int slots = pl->sm_count * ctas_per_sm;
+  const int slots = pl->sm_count * cpsm;
   double best = 1e30;
   for (int S = 1; S <= g.n_chunks && S <= 64; ++S) {
     const int cps = (g.n_chunks + S - 1) / S;
@@ -301,7 +316,7 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
       }
     }
   }
-  dc.smem = (size_t)8 * kStages * 512 + (size_t)dc.cps * frag_per_chunk +
+  dc.smem = (size_t)8 * ring_depth(dc.NT) * 512 + (size_t)dc.cps * frag_per_chunk +
             (size_t)8 * 16 * 8 * dc.NT * 4;
   return dc;
 }

@@ -157,7 +157,8 @@ __global__ void __launch_bounds__(128) prep_kernel(PrepParams p) {
 
 // ------------------------------------------------------- bf16 fragments
 // B operand of the decode MMAs, in the order one lane reads it: entry
-// (k-step ks, column tile nt, lane (g, t)) is a uint4 of bf16 pairs
+// (k-step ks, column tile nt, lane (g, t)) is a uint4 of bf16 pairs (with a
+// single column tile only the lanes of used columns, g < M * T, are stored)
 //   .x = (xt[4t+1], xt[4t+3])        .y = (xt[16+4t+1], xt[16+4t+3])
 //   .z = (xt[4t],   xt[4t+2])        .w = (xt[16+4t],   xt[16+4t+2])
 // (offsets from 32 ks) of column n = 8 nt + g = (batch m, term): term 0 is
@@ -167,7 +168,7 @@ struct FragParams {
   const float* xt;
   uint4* frag;
   float* scale;
-  int M, T, NT;
+  int M, T, NT, lanes;   // lanes per (k-step, tile): 32, or 4 * M * T with one tile
   int64_t kpad, total;
 };
 
@@ -187,9 +188,9 @@ __global__ void __launch_bounds__(256) frag_kernel(FragParams p) {
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx < p.M && blockIdx.x == 0) p.scale[idx] = 1.f;
   if (idx >= p.total) return;
-  const int ln = (int)(idx & 31);
-  const int nt = (int)((idx >> 5) % p.NT);
-  const int64_t ks = idx / (32 * p.NT);
+  const int ln = (int)(idx % p.lanes);
+  const int nt = (int)((idx / p.lanes) % p.NT);
+  const int64_t ks = idx / ((int64_t)p.lanes * p.NT);
   const int g = ln >> 2, t = ln & 3, n = nt * 8 + g;
   uint4 v = make_uint4(0, 0, 0, 0);
   if (n < p.M * p.T) {
@@ -223,7 +224,9 @@ cudaError_t launch_prep(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws
   const int BT = (g.nblk + TB - 1) / TB;
   p.P = p.JT * BT;
   if (p.prefill) {
-    p.pmax = nullptr; p.cnt = nullptr; p.ncnt = 0;
+    p.pmax = nullptr;
+    p.cnt = reinterpret_cast<uint32_t*>(base + L.err);   // the error word
+    p.ncnt = 1;
   } else {
     const DecodeConfig& dc = decode_config(pl, M);
     p.pmax = reinterpret_cast<float*>(base + L.pmax);
@@ -252,8 +255,9 @@ cudaError_t launch_frag(const sdq_plan_s* pl, int M, void* ws, cudaStream_t st) 
   p.frag = reinterpret_cast<uint4*>(base + L.frag);
   p.scale = reinterpret_cast<float*>(base + L.scale);
   p.M = M; p.T = dc.T; p.NT = dc.NT;
+  p.lanes = dc.NT == 1 ? 4 * M * dc.T : 32;
   p.kpad = g.k_eff_pad;
-  p.total = (g.k_eff_pad / 32) * dc.NT * 32;
+  p.total = (g.k_eff_pad / 32) * dc.NT * p.lanes;
   const int64_t blocks = (p.total + 255) / 256;
   return launch_pdl(frag_kernel, dim3((unsigned)blocks), dim3(256), 0, st, p);
 }

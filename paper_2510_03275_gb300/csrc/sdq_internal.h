@@ -5,7 +5,7 @@
 #include <cstddef>
 #include <cstdint>
 
-#include "../../include/sdq.h"
+#include "sdq.h"
 
 namespace sdq {
 

@@ -298,3 +298,33 @@ def test_workspace_too_small_rejected(sdq, torch_cuda):
     with pytest.raises(sdq.SdqError) as e:
         sdq.sdq_linear_forward(plan.handle, tiled, torch.from_numpy(alpha).cuda(), x, 4, y, small)
     assert e.value.status == -3
+
+
+# ---------------------------------------------------------------- prefill
+@pytest.mark.parametrize("q", [O.TERNARY, O.BINARY])
+@pytest.mark.parametrize("m,shape", [(128, (256, 512, 128, 2)), (200, (300, 384, 128, Fraction(5, 2))),
+                                     (65, (17, 20, 4, Fraction(5, 2))), (130, (256, 512, 512, 2)),
+                                     (384, (520, 768, 128, Fraction(3, 2)))])
+def test_forward_prefill_small(sdq, torch_cuda, q, m, shape):
+    """tcgen05 prefill path (M > 64) against the oracle; x_tilde enters the
+    tensor cores as bf16 (one rounding), codes exactly."""
+    n, k, b, osr = shape
+    lay = _setup_layer(sdq, torch_cuda, n, k, b, osr, q, seed=n + k + m)
+    err = _check_forward(*lay, sdq, torch_cuda, m, seed=m)
+    assert err <= TOL, err
+    assert err <= 8e-3, err
+
+
+@pytest.mark.parametrize("ci,name,m", [(4, "q", 4096), (4, "gate", 4096), (4, "down", 4096),
+                                       (3, "l0.gate", 2048), (3, "l3.down", 2048)])
+def test_forward_prefill_full_size_sampled(sdq, torch_cuda, ci, name, m):
+    """Full-size prefill in the bench's launch shape; 32 sampled rows."""
+    from paper_2510_03275_gb300.multiosr import allocate
+    torch = torch_cuda
+    cfg = W.config(ci, multiosr=allocate)
+    lin = [l for l in cfg.linears if l.name == name][0]
+    rows = np.sort(np.random.default_rng(lin.seed + m).choice(lin.n_out, 32, replace=False))
+    lay = _setup_layer(sdq, torch, lin.n_out, lin.k_in, cfg.block, lin.osr, cfg.quantizer,
+                       seed=lin.seed, rows=rows)
+    err = _check_forward(*lay, sdq, torch, m, seed=m + 5, rows=rows)
+    assert err <= min(TOL, 8e-3), err
