@@ -192,6 +192,29 @@ int sdq_workspace_status(sdq_plan plan, int32_t M, const void* ws, void* stream)
  * device), for checking sdq_prep_activations. */
 int sdq_read_prep(sdq_plan plan, int32_t M, const void* ws, float* xt_out, void* stream);
 
+/* Allocation-free decode forward, for callers that may not allocate device
+ * memory or pass a workspace (for example a plugin whose host runtime owns
+ * every device allocation, or a serving loop that forbids allocation after
+ * start-up).  No counterpart in the paper: it is a packaging of
+ * sdq_linear_forward.  Same inputs and outputs as sdq_linear_forward, but
+ * the scratch is a library-owned device array of sdq_noalloc_scratch_bytes()
+ * (16 MiB) per GPU, reserved when the library loads and held until the
+ * process exits.  No cudaMalloc / cudaFree / allocating call is made.
+ *   - M must be 1..64 (the decode path), and sdq_workspace_bytes(plan, M)
+ *     must not exceed the array: otherwise SDQ_ERR_INVALID_ARG or
+ *     SDQ_ERR_WORKSPACE is returned and nothing is launched.
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress, with that device current); make that first call
+ *     before any stream capture.
+ *   - All calls on a device share the array and it keeps the last call's
+ *     contents; each call's prepare kernel re-zeroes what must start at
+ *     zero.  Calls that overlap on the GPU (other streams or host threads)
+ *     race on the array: serialize them.
+ *   - sdq_workspace_status is not available for these calls. */
+int sdq_linear_forward_noalloc(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha,
+                               const uint16_t* x, int32_t M, float* y, void* stream);
+size_t sdq_noalloc_scratch_bytes(void);
+
 /* Static string for a status code. */
 const char* sdq_status_string(int status);
 

@@ -23,7 +23,7 @@ __all__ = [
     "sdq_plan_create", "sdq_plan_destroy", "sdq_k_eff", "sdq_plain_bytes", "sdq_tiled_bytes",
     "sdq_workspace_bytes", "sdq_build_tables", "sdq_encode_rows", "sdq_pack", "sdq_unpack",
     "sdq_prep_activations", "sdq_contract", "sdq_linear_forward", "sdq_read_prep",
-    "sdq_workspace_status",
+    "sdq_workspace_status", "sdq_linear_forward_noalloc", "sdq_noalloc_scratch_bytes",
     "sdq_status_string", "Plan",
 ]
 
@@ -89,6 +89,8 @@ _SIGS = {
     "sdq_linear_forward": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _vp, _vp, _sz, _vp]),
     "sdq_read_prep": (ctypes.c_int, [_vp, _i32, _vp, _vp, _vp]),
     "sdq_workspace_status": (ctypes.c_int, [_vp, _i32, _vp, _vp]),
+    "sdq_linear_forward_noalloc": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _vp, _vp]),
+    "sdq_noalloc_scratch_bytes": (_sz, []),
     "sdq_status_string": (ctypes.c_char_p, [ctypes.c_int]),
 }
 
@@ -209,6 +211,18 @@ def sdq_read_prep(plan, M, ws, out, stream=None):
 def sdq_workspace_status(plan, M, ws, stream=None) -> int:
     """Synchronize and return the status of the last decode using ``ws``."""
     return lib().sdq_workspace_status(plan, M, _ptr(ws), _stream(stream))
+
+
+def sdq_linear_forward_noalloc(plan, codes_tiled, alpha, x, M, y, stream=None):
+    """Decode forward (M <= 64) using the library's own device scratch array
+    instead of a caller workspace; see include/sdq.h for its rules."""
+    _check(lib().sdq_linear_forward_noalloc(plan, _ptr(codes_tiled), _ptr(alpha), _ptr(x), M,
+                                            _ptr(y), _stream(stream)),
+           "sdq_linear_forward_noalloc")
+
+
+def sdq_noalloc_scratch_bytes() -> int:
+    return lib().sdq_noalloc_scratch_bytes()
 
 
 def sdq_status_string(status: int) -> str:
