@@ -10,7 +10,8 @@
 // 128-byte-swizzled operand layout of tcgen05.mma.
 //
 // CTA tile 128 (M) x 256 (N), 64 codes per pipeline stage, kStages stages:
-//   warp 0      TMEM allocation; lane 0 issues the TMA loads of A tiles
+//   warp 0      TMEM allocation; lane 0 issues the TMA loads of the A tile
+//               and of the packed code words of every stage
 //   warp 1      lane 0 issues tcgen05.mma (4 x K=16 per stage), commits to
 //               the stage's "empty" barrier, finally to the accumulator one
 //   warps 2..5  expand the B tile of every stage (one 16-byte smem chunk per
@@ -34,7 +35,8 @@ namespace {
 constexpr int kBM = 128, kBN = 256, kBK = 64, kStages = 4;
 constexpr int kATile = kBM * kBK * 2;     // 16 KB
 constexpr int kBTile = kBN * kBK * 2;     // 32 KB
-constexpr int kSmem = kStages * (kATile + kBTile) + 1024;
+constexpr int kCTile = 16 * 64 * 4;       // packed codes of a stage: 16 row groups x 256 bytes
+constexpr int kSmem = kStages * (kATile + kBTile + kCTile) + 1024;
 constexpr int kThreads = 192;
 
 struct PrefillParams {
@@ -119,7 +121,8 @@ __device__ __forceinline__ void st_chunk(uint8_t* btile, int n, int c8, uint32_t
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-    prefill_kernel(const __grid_constant__ CUtensorMap amap, PrefillParams p) {
+    prefill_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap cmap,
+                   PrefillParams p) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_a[kStages], full_b[kStages], empty[kStages], acc_bar;
   __shared__ uint32_t tmem_base;
@@ -131,6 +134,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* base = smem_raw + (sbase - smem_u32(smem_raw));
   uint8_t* a_tiles = base;
   uint8_t* b_tiles = base + kStages * kATile;
+  const uint32_t* c_tiles = reinterpret_cast<const uint32_t*>(base + kStages * (kATile + kBTile));
+  const int cwords = p.quantizer == SDQ_TERNARY ? 64 : 32;      // words per row group per stage
 
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -156,13 +161,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      // A producer: TMA of x_tilde tiles [m0, m0+128) x [64 ks, 64 ks + 64).
+      // Producer: TMA of the x_tilde tile [m0, m0+128) x [64 ks, 64 ks + 64)
+      // and of the packed code words of the same 64 codes for the CTA's 16
+      // row groups (one 2-D box of the tiled layout; rows past N read 0).
       for (int ks = 0; ks < p.nks && ok; ++ks) {
         const int s = ks % kStages, r = ks / kStages;
         if (r > 0) ok = mbar_wait(&empty[s], (r - 1) & 1);
         if (!ok) break;
-        mbar_expect_tx(&full_a[s], kATile);
+        const int cx = p.quantizer == SDQ_TERNARY ? (ks >> 1) * 128 + 64 * (ks & 1)
+                                                   : (ks >> 2) * 128 + 32 * (ks & 3);
+        mbar_expect_tx(&full_a[s], kATile + 16 * cwords * 4);
         tma_load_2d(a_tiles + s * kATile, &amap, ks * kBK, m0, &full_a[s]);
+        tma_load_2d(base + kStages * (kATile + kBTile) + s * kCTile, &cmap, cx, n0 >> 4, &full_a[s]);
       }
     }
   } else if (warp == 1) {
@@ -189,18 +199,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int ks = 0; ks < p.nks && ok; ++ks) {
       const int s = ks % kStages, r = ks / kStages;
       if (r > 0) ok = mbar_wait(&empty[s], (r - 1) & 1);
+      if (ok) ok = mbar_wait(&full_a[s], r & 1);             // packed codes have landed
       if (!ok) break;
       uint8_t* bt = b_tiles + s * kBTile;
+      const uint32_t* ct = c_tiles + s * (kCTile / 4);
       if (p.quantizer == SDQ_TERNARY) {
-        const int c = ks >> 1, e = ks & 1;
-#pragma unroll 2
+#pragma unroll 4
         for (int u = 0; u < 8; ++u) {
           const int idx = (et >> 5) + 4 * u;            // (row group, word half) pair
           const int rgl = idx >> 1, qh = idx & 1;
-          const int rg = (n0 >> 4) + rgl;
-          uint32_t w = 0;
-          if (rg < p.ng)
-            w = __ldg(p.codes + ((size_t)rg * p.n_chunks + c) * 128 + 32 * (2 * e + qh) + L);
+          const uint32_t w = ct[rgl * 64 + 32 * qh + L];
           uint32_t v[8];
 #pragma unroll
           for (int j = 0; j < 8; ++j) v[j] = (w << (2 * j)) & 0xC000C000u;
@@ -209,15 +217,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           st_chunk(bt, n + 8, c8, v[1], v[3], v[5], v[7]);
         }
       } else {
-        const int c = ks >> 2, q = ks & 3;
 #pragma unroll 2
         for (int u = 0; u < 4; ++u) {
           const int rgl = (et >> 5) + 4 * u;
-          const int rg = (n0 >> 4) + rgl;
-          uint32_t w = 0;
-          if (rg < p.ng)
-            w = __ldg(p.codes + ((size_t)rg * p.n_chunks + c) * 128 + 32 * q + L);
-          const uint32_t nw = ~w;
+          const uint32_t nw = ~ct[rgl * 32 + L];
           uint32_t v[16];
 #pragma unroll
           for (int j = 0; j < 16; ++j) v[j] = ((nw << j) & 0x80008000u) | 0x40004000u;
@@ -306,6 +309,15 @@ cudaError_t launch_prefill(const sdq_plan_s* pl, const uint32_t* codes, const fl
                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
+  // Tiled codes as a 2-D array: one row per row group, n_chunks * 128 words.
+  CUtensorMap cmap;
+  const cuuint64_t cdims[2] = {(cuuint64_t)g.n_chunks * 128, (cuuint64_t)g.ng};
+  const cuuint64_t cstrides[1] = {(cuuint64_t)g.n_chunks * 512};
+  const cuuint32_t cbox[2] = {(cuuint32_t)(pl->desc.quantizer == SDQ_TERNARY ? 64 : 32), 16};
+  cr = enc(&cmap, CU_TENSOR_MAP_DATA_TYPE_UINT32, 2, const_cast<uint32_t*>(codes), cdims, cstrides, cbox,
+           estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
   PrefillParams p;
   p.codes = codes; p.alpha = alpha; p.y = y;
   p.err = reinterpret_cast<uint32_t*>(wbase + L.err);
@@ -315,7 +327,7 @@ cudaError_t launch_prefill(const sdq_plan_s* pl, const uint32_t* codes, const fl
   cudaError_t e = cudaFuncSetAttribute(prefill_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
   if (e != cudaSuccess) return e;
   dim3 grid((g.n_out + kBN - 1) / kBN, (M + kBM - 1) / kBM);
-  return launch_pdl(prefill_kernel, grid, dim3(kThreads), (size_t)kSmem, st, amap, p);
+  return launch_pdl(prefill_kernel, grid, dim3(kThreads), (size_t)kSmem, st, amap, cmap, p);
 }
 
 }  // namespace sdq
