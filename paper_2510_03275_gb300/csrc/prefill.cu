@@ -14,7 +14,7 @@
 //               and of the packed code words of every stage
 //   warp 1      lane 0 issues tcgen05.mma (4 x K=16 per stage), commits to
 //               the stage's "empty" barrier, finally to the accumulator one
-//   warps 2..5  expand the B tile of every stage (one 16-byte smem chunk per
+//   warps 2..9  expand the B tile of every stage (one 16-byte smem chunk per
 //               8 codes of one row; the shift-and-mask expansion of a tiled
 //               word yields its codes in the permuted order the prep kernel
 //               also uses for A), then read the fp32 accumulator out of TMEM
@@ -37,7 +37,8 @@ constexpr int kATile = kBM * kBK * 2;     // 16 KB
 constexpr int kBTile = kBN * kBK * 2;     // 32 KB
 constexpr int kCTile = 16 * 64 * 4;       // packed codes of a stage: 16 row groups x 256 bytes
 constexpr int kSmem = kStages * (kATile + kBTile + kCTile) + 1024;
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;   // 2 control warps + 8 expander / epilogue warps
+constexpr int kExp = 256;       // expander threads
 
 struct PrefillParams {
   const uint32_t* codes;
@@ -140,7 +141,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&full_a[s], 1);
-      mbar_init(&full_b[s], 128);
+      mbar_init(&full_b[s], kExp);
       mbar_init(&empty[s], 1);
     }
     mbar_init(&acc_bar, 1);
@@ -192,7 +193,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       umma_commit(&acc_bar);
     }
   } else {
-    // B expanders: 128 threads.  Lane -> (g = lane % 8, t = lane / 8) so
+    // B expanders: kExp threads.  Lane -> (g = lane % 8, t = lane / 8) so
     // the 8 lanes of each 128-bit store phase hit 8 distinct 16-byte banks.
     const int et = tid - 64;
     const int g = lane & 7, t = lane >> 3, L = 4 * g + t;
@@ -204,9 +205,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint8_t* bt = b_tiles + s * kBTile;
       const uint32_t* ct = c_tiles + s * (kCTile / 4);
       if (p.quantizer == SDQ_TERNARY) {
-#pragma unroll 4
-        for (int u = 0; u < 8; ++u) {
-          const int idx = (et >> 5) + 4 * u;            // (row group, word half) pair
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int idx = (et >> 5) + 8 * u;            // (row group, word half) pair
           const int rgl = idx >> 1, qh = idx & 1;
           const uint32_t w = ct[rgl * 64 + 32 * qh + L];
           uint32_t v[8];
@@ -217,9 +218,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           st_chunk(bt, n + 8, c8, v[1], v[3], v[5], v[7]);
         }
       } else {
-#pragma unroll 2
-        for (int u = 0; u < 4; ++u) {
-          const int rgl = (et >> 5) + 4 * u;
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const int rgl = (et >> 5) + 8 * u;
           const uint32_t nw = ~ct[rgl * 32 + L];
           uint32_t v[16];
 #pragma unroll
@@ -238,9 +239,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (ok) ok = mbar_wait(&acc_bar, 0);
     tc_fence_after();
     if (ok) {
-      const int qd = warp & 3;
+      const int qd = warp & 3;                       // TMEM lane quadrant of this warp
+      const int half = (warp - 2) >> 2;              // warps 2..5 and 6..9 split the columns
       const int row = m0 + 32 * qd + lane;
-      for (int cc = 0; cc < kBN / 16; ++cc) {
+      for (int cc = half * (kBN / 32); cc < (half + 1) * (kBN / 32); ++cc) {
         uint32_t r[16];
         tmem_ld16(tmem + ((uint32_t)(32 * qd) << 16) + 16 * cc, r);
         tmem_ld_wait();
