@@ -431,66 +431,52 @@ def unpack_plain(words, quantizer: int, k_eff: int) -> np.ndarray:
     return np.where(f == 1, 1, -1).astype(np.int8)
 
 
+TILE_ROWS = 128      # rows per tile of the tiled layout
+GROUP_CODES = 64     # codes per k group of the tiled layout
+
+
 def tiled_geometry(n_out: int, k_eff: int, quantizer: int):
-    """(row groups, k chunks per row group, codes per chunk) of the tiled layout."""
-    kc = 128 if quantizer == TERNARY else 256
-    return (n_out + 15) // 16, (k_eff + kc - 1) // kc, kc
+    """(tiles, k groups per tile, words per row per group) of the tiled
+    layout.  K_eff is padded to a multiple of 128 codes."""
+    k_pad = -(-k_eff // 128) * 128
+    wpr = GROUP_CODES * quantizer // 32
+    return -(-n_out // TILE_ROWS), k_pad // GROUP_CODES, wpr
 
 
-def _tiled_position(g_row: int, k: int, quantizer: int, n_chunks: int):
+def _tiled_position(row: int, k: int, quantizer: int, n_groups: int):
     """(word index, bit shift) of code (row, k) in the tiled layout.
 
-    Tile (G, c) = rows [16G, 16G+16) x codes [kc*c, kc*c + kc) occupies 128
-    consecutive uint32 words starting at word ``128 * (G * n_chunks + c)``;
-    word ``32 q + L`` of the tile belongs to lane ``L = 4 g + t``.
-
-    Ternary (kc = 128, 16 two-bit fields f per word):
-        j = 3 - f % 4, b = f // 4,
-        row = 16G + g + 8 (j % 2),  k = 128c + 32q + 16 (j // 2) + 4t + b.
-    Binary (kc = 256, 32 one-bit fields f per word):
-        j = 7 - f % 8, b = f // 8,
-        row = 16G + g + 8 (j % 2),
-        k = 256c + 64q + 32 (j // 4) + 16 ((j // 2) % 2) + 4t + b.
-    This function inverts those maps for one (row, k).
+    Rows are cut into tiles of 128 (T = row // 128, r = row % 128) and codes
+    into groups of 64 (G = k // 64).  Slab (T, G) is 128 * wpr consecutive
+    uint32 words starting at word ``128 * wpr * (T * n_groups + G)``, and row
+    r owns the ``wpr`` words starting at ``wpr * r`` inside it (wpr = 4
+    ternary, 2 binary).  Inside the row's words the codes keep their natural
+    order: ternary word i = (k % 64) // 16 holds k at field f = k % 16 (bits
+    2f, 2f+1); binary word i = (k % 64) // 32 holds k at bit f = k % 32.
     """
-    G, r = divmod(g_row, 16)
-    g, half = r % 8, r // 8
-    if quantizer == TERNARY:
-        c, kk = divmod(k, 128)
-        q, kk = divmod(kk, 32)
-        h, kk = divmod(kk, 16)
-        t, b = divmod(kk, 4)
-        j = 2 * h + half
-        f = 4 * b + (3 - j)
-        shift = 2 * f
-    else:
-        c, kk = divmod(k, 256)
-        q, kk = divmod(kk, 64)
-        u, kk = divmod(kk, 32)
-        h, kk = divmod(kk, 16)
-        t, b = divmod(kk, 4)
-        j = 4 * u + 2 * h + half
-        f = 8 * b + (7 - j)
-        shift = f
-    L = 4 * g + t
-    word = 128 * (G * n_chunks + c) + 32 * q + L
-    return word, shift
+    T, r = divmod(row, TILE_ROWS)
+    G, kk = divmod(k, GROUP_CODES)
+    wpr = GROUP_CODES * quantizer // 32
+    per = 32 // quantizer
+    i, f = divmod(kk, per)
+    word = wpr * (TILE_ROWS * (T * n_groups + G) + r) + i
+    return word, quantizer * f
 
 
 def pack_tiled(codes, quantizer: int) -> np.ndarray:
-    """Tiled layout (see :func:`_tiled_position`), padding codes 0 / -1.
+    """Tiled layout (see :func:`_tiled_position`), padding fields 0.
 
     Pure-Python loop over every code: use on small matrices only.
     """
     codes = np.asarray(codes)
     n, k = codes.shape
-    ng, nc, kc = tiled_geometry(n, k, quantizer)
-    out = [0] * (128 * ng * nc)
+    nt, ng, wpr = tiled_geometry(n, k, quantizer)
+    out = [0] * (nt * ng * TILE_ROWS * wpr)
     for r in range(n):
         for kk in range(k):
             fv = _field(codes[r, kk], quantizer)
             if fv:
-                w, s = _tiled_position(r, kk, quantizer, nc)
+                w, s = _tiled_position(r, kk, quantizer, ng)
                 out[w] |= fv << s
     return np.array(out, dtype=np.uint64).astype(np.uint32)
 
@@ -498,12 +484,12 @@ def pack_tiled(codes, quantizer: int) -> np.ndarray:
 def unpack_tiled(words, quantizer: int, n_out: int, k_eff: int) -> np.ndarray:
     """Inverse of :func:`pack_tiled` (pure-Python loop; small matrices)."""
     words = [int(v) for v in np.asarray(words, dtype=np.uint32)]
-    _, nc, _ = tiled_geometry(n_out, k_eff, quantizer)
+    _, ng, _ = tiled_geometry(n_out, k_eff, quantizer)
     out = np.zeros((n_out, k_eff), dtype=np.int8)
     mask = (1 << quantizer) - 1
     for r in range(n_out):
         for kk in range(k_eff):
-            w, s = _tiled_position(r, kk, quantizer, nc)
+            w, s = _tiled_position(r, kk, quantizer, ng)
             f = (words[w] >> s) & mask
             if quantizer == TERNARY:
                 out[r, kk] = 1 if f == 1 else (-1 if f == 3 else 0)

@@ -41,19 +41,19 @@ WsLayout workspace_layout(const sdq_plan_s* pl, int M) {
     const DecodeConfig& dc = pl->dcfg[M];
     off = align_up(off + sizeof(float) * (size_t)M * g.k_eff_pad, 256);
     L.pmax = off;
-    off = align_up(off + sizeof(float) * (size_t)M * dc.P, 256);
-    L.frag = off;
-    off = align_up(off + (size_t)(g.k_eff_pad / 32) * dc.NT * 32 * 16, 256);
-    L.scale = off;
-    off = align_up(off + sizeof(float) * kMaxDecodeM, 256);
+    off = align_up(off + sizeof(float) * (size_t)M * dc.pp, 256);
+    L.bimg = off;                                  // e4m3 B operand image, K/128 x NP x 128 bytes
+    off = align_up(off + (size_t)(g.k_eff_pad / 128) * dc.NP * 128, 256);
+    L.sexp = off;                                  // per-batch-row scale exponents
+    off = align_up(off + sizeof(int32_t) * kMaxDecodeM, 256);
     L.part = off;
-    off = align_up(off + (dc.S > 1 ? sizeof(float) * (size_t)dc.S * M * g.ng * 16 : 0), 256);
-    L.cnt = off;                                   // R counters, then the error word
-    L.err = off + sizeof(uint32_t) * (size_t)dc.R;
-    off = align_up(off + sizeof(uint32_t) * ((size_t)dc.R + 1), 256);
+    off = align_up(off + (dc.S > 1 ? sizeof(float) * (size_t)dc.S * M * g.ntiles * kTileRows : 0), 256);
+    L.cnt = off;                                   // one ticket per row tile, then the error word
+    L.err = off + sizeof(uint32_t) * (size_t)g.ntiles;
+    off = align_up(off + sizeof(uint32_t) * ((size_t)g.ntiles + 1), 256);
   } else {
     off = align_up(off + sizeof(uint16_t) * (size_t)M * g.k_eff_pad, 256);
-    L.pmax = L.frag = L.scale = L.part = L.cnt = L.err = off;   // error word only
+    L.pmax = L.bimg = L.sexp = L.part = L.cnt = L.err = off;   // error word only
     off = align_up(off + sizeof(uint32_t), 256);
   }
   L.total = off;
@@ -159,28 +159,36 @@ extern "C" int sdq_prep_activations(sdq_plan p, const uint16_t* x, int32_t M, vo
   if (st != SDQ_OK) return st;
   if (!x || !aligned16(x)) return SDQ_ERR_INVALID_ARG;
   cudaError_t e = launch_prep(p, x, M, ws, (cudaStream_t)stream);
-  if (e == cudaSuccess && M <= kMaxDecodeM) e = launch_frag(p, M, ws, (cudaStream_t)stream);
+  if (e == cudaSuccess && M <= kMaxDecodeM) e = launch_terms(p, M, ws, (cudaStream_t)stream);
+  return cuda_status(e);
+}
+
+static int contract(sdq_plan p, const uint32_t* codes_tiled, const float* alpha, int32_t M, float* y,
+                    void* ws, size_t ws_bytes, void* stream, int early) {
+  int st = check_ws(p, M, ws, ws_bytes);
+  if (st != SDQ_OK) return st;
+  if (!codes_tiled || !alpha || !y || !aligned16(codes_tiled) || !aligned16(y)) return SDQ_ERR_INVALID_ARG;
+  cudaError_t e = M <= kMaxDecodeM
+                      ? launch_decode(p, codes_tiled, alpha, M, y, ws, (cudaStream_t)stream, early)
+                      : launch_prefill(p, codes_tiled, alpha, M, y, ws, (cudaStream_t)stream);
+  if (e == cudaErrorNotSupported) return SDQ_ERR_UNSUPPORTED;
   return cuda_status(e);
 }
 
 extern "C" int sdq_contract(sdq_plan p, const uint32_t* codes_tiled, const float* alpha, int32_t M,
                             float* y, void* ws, size_t ws_bytes, void* stream) {
-  int st = check_ws(p, M, ws, ws_bytes);
-  if (st != SDQ_OK) return st;
-  if (!codes_tiled || !alpha || !y || !aligned16(codes_tiled) || !aligned16(y)) return SDQ_ERR_INVALID_ARG;
-  if (M <= kMaxDecodeM)
-    return cuda_status(launch_decode(p, codes_tiled, alpha, M, y, ws, (cudaStream_t)stream));
-  cudaError_t e = launch_prefill(p, codes_tiled, alpha, M, y, ws, (cudaStream_t)stream);
-  if (e == cudaErrorNotSupported) return SDQ_ERR_UNSUPPORTED;
-  return cuda_status(e);
+  return contract(p, codes_tiled, alpha, M, y, ws, ws_bytes, stream, 0);
 }
 
+// Behind its own prepare kernels the decode kernel may start reading the
+// codes before the preceding grid finishes: that grid waited for everything
+// before it in the stream, and it does not write the codes.
 extern "C" int sdq_linear_forward(sdq_plan p, const uint32_t* codes_tiled, const float* alpha,
                                   const uint16_t* x, int32_t M, float* y, void* ws, size_t ws_bytes,
                                   void* stream) {
   int st = sdq_prep_activations(p, x, M, ws, ws_bytes, stream);
   if (st != SDQ_OK) return st;
-  return sdq_contract(p, codes_tiled, alpha, M, y, ws, ws_bytes, stream);
+  return contract(p, codes_tiled, alpha, M, y, ws, ws_bytes, stream, 1);
 }
 
 extern "C" int sdq_workspace_status(sdq_plan p, int32_t M, const void* ws, void* stream) {

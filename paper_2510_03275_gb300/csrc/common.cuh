@@ -1,6 +1,7 @@
 // Device helpers shared by the libsdq kernels (sm_103a).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_fp8.h>
 #include <cstdint>
@@ -14,7 +15,7 @@ DecodeConfig decode_config_search(const sdq_plan_s* plan, int M);
 inline const DecodeConfig& decode_config(const sdq_plan_s* plan, int M) { return plan->dcfg[M]; }
 
 struct WsLayout {
-  size_t xt, pmax, frag, scale, part, cnt, err, total;
+  size_t xt, pmax, bimg, sexp, part, cnt, err, total;
 };
 WsLayout workspace_layout(const sdq_plan_s* plan, int M);
 
@@ -25,11 +26,13 @@ cudaError_t launch_pack(const sdq_plan_s* p, const uint32_t* plain, uint32_t* ti
 cudaError_t launch_unpack(const sdq_plan_s* p, const uint32_t* tiled, uint32_t* plain,
                           uint32_t* bad, cudaStream_t st);
 cudaError_t launch_prep(const sdq_plan_s* p, const uint16_t* x, int M, void* ws, cudaStream_t st);
+// early = 1: the decode kernel starts streaming codes before waiting for the
+// preceding grid (valid only behind this library's own prep kernels).
 cudaError_t launch_decode(const sdq_plan_s* p, const uint32_t* codes, const float* alpha, int M,
-                          float* y, void* ws, cudaStream_t st);
+                          float* y, void* ws, cudaStream_t st, int early);
+cudaError_t launch_terms(const sdq_plan_s* p, int M, void* ws, cudaStream_t st);
 cudaError_t launch_prefill(const sdq_plan_s* p, const uint32_t* codes, const float* alpha, int M,
                            float* y, void* ws, cudaStream_t st);
-cudaError_t launch_frag(const sdq_plan_s* p, int M, void* ws, cudaStream_t st);
 int prep_partials(const sdq_plan_s* p, int M);  // per-row max partials of the prep grid
 cudaError_t launch_read_prep(const sdq_plan_s* p, int M, const void* ws, float* out, cudaStream_t st);
 
@@ -147,14 +150,122 @@ cudaError_t launch_pdl(Kern k, dim3 grid, dim3 block, size_t smem, cudaStream_t 
   return cudaLaunchKernelEx(&cfg, k, args...);
 }
 
+// ------------------------------------------------------ tcgen05 / TMEM
+__device__ __forceinline__ void tmem_alloc(uint32_t* dst, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_u32(dst)),
+               "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
+}
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                          uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate) : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(
+                   smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int c0, int c1,
+                                            uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];\n" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(smem_u32(bar)) : "memory");
+}
+// 32 TMEM lanes x 16 columns of 32-bit values: register i of the thread of
+// lane l holds (lane base + l, column + i).
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15},"
+      " [%16];\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory"); }
+
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
+// 1024 bytes apart (SBO), start address in 16-byte units.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1 << 16;                 // leading byte offset (unused for swizzled K-major)
+  d |= (uint64_t)(1024 >> 4) << 32;       // stride byte offset
+  d |= (uint64_t)1 << 46;                 // descriptor version
+  d |= (uint64_t)2 << 61;                 // SWIZZLE_128B
+  return d;
+}
+
+// 32 TMEM lanes x 32 columns of 32-bit values from registers: register i of
+// the thread of lane l goes to (lane base + l, column + i).
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};\n" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]),
+      "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]),
+      "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;\n" ::: "memory"); }
+// D (TMEM, fp32) (+)= A (TMEM, e4m3) . B (smem descriptor, e4m3)^T.
+__device__ __forceinline__ void umma_f8_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                           uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate) : "memory");
+}
+__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
+  asm volatile("bar.sync %0, %1;\n" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// Natural k (within a 128-code decode block) at MMA K index kap: the order in
+// which the decode expander lays a row's codes into TMEM columns.
+//   ternary: column 4 wi + j (word wi, shift 2j) byte b = code 16 wi + 4b + 3 - j
+//   binary:  column 8 wi + j (word wi, shift j)  byte b = code 32 wi + 8b + 7 - j
+__host__ __device__ __forceinline__ int decode_stage_k(int kap, bool ternary) {
+  if (ternary) {
+    const int kp = kap & 15;
+    return (kap & ~15) + 4 * (kp & 3) + 3 - (kp >> 2);
+  }
+  const int kp = kap & 31;
+  return (kap & ~31) + 8 * (kp & 3) + 7 - (kp >> 2);
+}
+
 // Position of natural index kl (0..63) inside a 64-code stage of the prefill
-// operand order: the order in which the prefill expander writes codes (and
-// the prep kernel writes x_tilde) so that each 16-byte chunk of a bf16 tile
-// row is one shift-and-mask expansion of a tiled word.
-__host__ __device__ __forceinline__ int prefill_perm64(int kl) {
-  const int qq = kl >> 5, r = kl & 31, h = r >> 4, t = (r & 15) >> 2, i = r & 3;
-  const int inv = (i & 1) ? ((i >> 1) + 2 * h) : (4 + (i >> 1) + 2 * h);
-  return 8 * (4 * qq + t) + inv;
+// operand order: the order in which the prefill expander writes a row's codes
+// (and the prep kernel writes x_tilde) when word i of the row is expanded by
+// shift-and-mask into bf16 pairs.
+//   ternary: pair j of word i (i < 4, j < 8) holds codes 16i + 7 - j (low
+//            half) and 16i + 15 - j (high half) at positions 16i + 2j, +1
+//   binary:  pair j of word i (i < 2, j < 16) holds codes 32i + 15 - j and
+//            32i + 31 - j at positions 32i + 2j, +1
+__host__ __device__ __forceinline__ int prefill_pos64(int kl, bool ternary) {
+  if (ternary) {
+    const int i = kl >> 4, f = kl & 15;
+    return f < 8 ? 16 * i + 2 * (7 - f) : 16 * i + 2 * (15 - f) + 1;
+  }
+  const int i = kl >> 5, f = kl & 31;
+  return f < 16 ? 32 * i + 2 * (15 - f) : 32 * i + 2 * (31 - f) + 1;
 }
 
 }  // namespace sdq

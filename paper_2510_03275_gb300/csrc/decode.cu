@@ -1,350 +1,480 @@
-// K4 (+K6): decode contraction for batch M <= 64.
+// K4: decode contraction (M <= 64) on the 5th-generation tensor cores, with
+// the code operand expanded into tensor memory.
 //
-//   y[m, r] = alpha_r * sum_j c[r, j] * x_tilde[m, j]
+//   y[m, r] = alpha_r * sum_j c[r, j] * x_tilde[m, j]        (section 3.5, eq. 12)
 //
-// (SDQ-LLM section 3.5 with eq. (12): the codes multiply the upsampled,
-// Hadamard-rotated activations; every product is a signed copy of x_tilde,
-// i.e. an add or a subtract.)
+// A skinny contraction whose cost is streaming the packed codes (2 or 1 bits
+// per weight sample) from HBM.  Expanding codes into multiply-accumulate
+// operands on the CUDA cores costs more integer issue slots than the HBM rate
+// leaves, so the products run on tcgen05.mma kind::f8f6f4 (M = 128, N = NP,
+// K = 32 per instruction) and the CUDA cores only expand:
+//   A (TMEM)  the codes of a 128-row tile as e4m3 +-2.0 / 0: thread = TMEM
+//             lane = weight row, 4 codes per 32-bit column, written with
+//             tcgen05.st straight from the shift-and-mask expansion of the
+//             row's packed words (no shared-memory round trip)
+//   B (smem)  the activations as T e4m3 terms per batch row m:
+//             x_tilde[m] * 2^-e_m = sum_t 16^-t q_t[m] (e_m from max |x_tilde|),
+//             N = M*T rows rounded up to 16, K-major, 128-byte swizzle,
+//             written for all of K by the prep stage's terms kernel; each CTA
+//             copies the part of its k chunk once
+//   D (TMEM)  fp32, 128 lanes x NP columns
+// so that y[m, r] = alpha_r / 2 * 2^e_m * sum_t 16^-t D[r, m T + t].
 //
-// The tiled code layout is built so that one shift and one mask of a packed
-// word is a bf16 A-operand register pair of a 16x8x16 warp MMA: each half
-// +-2.0 or 0, exact.  (The layout also yields fp8 registers with a wider
-// mask, but sm_103 runs warp-level fp8 MMAs through conversions; bf16 is
-// the native warp MMA.)  The activations enter as the B operand, written by
-// the fragment kernel as bf16 hi + lo terms (hi only for M > 16); each
-// (batch, term) pair is one of the 8 MMA columns.  The fp32 accumulators
-// therefore hold the add/subtract sums of the codes against each term; the
-// epilogue adds the terms and applies alpha / 2.
+// A stage is up to sb blocks of 128 codes (4 sb MMAs): every mbarrier wait
+// of an MMA-issuing thread costs about as much as several MMAs, and one
+// thread issues at most one MMA every ~45 cycles, so the CTA runs two
+// independent pipelines e = 0, 1 on alternate stages (i = e mod 2), each with
+// its own producer thread, expander warps, MMA issuer, two TMEM slots and
+// accumulator; the epilogue adds the two accumulators.  Every mbarrier thus
+// has one producer and one consumer that both walk its phases in order.
 //
-// Memory path: every warp streams its own sequence of 512-byte code tiles
-// (16 rows x 128 / 256 codes) through a private ring of shared-memory
-// slots filled with cp.async (16 bytes per lane, one commit group per tile),
-// so each SM keeps ~64 KB of loads in flight without holding them in
-// registers.  The CTA's slice of B-fragments arrives by one 1-D TMA bulk
-// copy.  The first code tiles are requested before the grid waits on the
-// fragment kernel (programmatic dependent launch), overlapping the
-// activation preparation.
-//
-// Work split: grid (R row ranges) x (S k-slices); each warp owns whole row
-// groups of its CTA's range (no CTA barrier in the stream).  With S > 1,
-// per-slice partials go to the workspace and the last CTA of each row range
-// (atomic ticket) sums them in slice order, so the result does not depend on
-// CTA scheduling.
+// CTA (k chunk s, row set p) of one SM, 16 warps:
+//   warps 0, 1    lane 0 of warp e streams pipeline e's stages (one 128-row
+//                 tile x up to sb * 128 codes = contiguous slabs of the tiled
+//                 layout) into its shared-memory ring slots with bulk copies;
+//                 warp 0 also owns the TMEM allocation and copies the chunk's
+//                 B operand
+//   warps 2, 3    lane 0 of warp 2 + e issues pipeline e's MMAs, commits to
+//                 the stage's TMEM slot and, after its last stage of a row
+//                 tile, to its accumulator
+//   warps 4..11   expanders: warps 4 + 4e .. 7 + 4e (one per TMEM lane
+//                 quadrant) expand pipeline e's stages into its TMEM slots
+//   warps 12..15  epilogue: read and add the accumulators, combine the
+//                 terms, scale and store y, or store a split-K partial; after
+//                 the CTA's last tile, one fence and one ticket per tile, and
+//                 the last CTA of each tile sums its S partials in a fixed
+//                 order (deterministic)
+// With `early` set the producers start the code stream before waiting for
+// the preceding grid (codes are never written by the prep kernels).
+// Every mbarrier wait is bounded (about 2 s); a timeout sets the workspace
+// error word and the CTA drains its copies and MMAs before freeing TMEM.
+#include <algorithm>
+#include <cmath>
+
 #include "common.cuh"
 
 namespace sdq {
 
 namespace {
 
-// Occupancy and cp.async ring depth (512-byte tiles per warp) by column tiles.
-__host__ __device__ constexpr int ctas_per_sm(int NT) { return NT == 1 ? 3 : (NT <= 4 ? 2 : 1); }
-__host__ __device__ constexpr int ring_depth(int NT) { return NT == 1 ? 6 : (NT <= 4 ? 8 : 4); }
+constexpr int kBlk = 128;                        // codes per block (4 MMAs of K = 32)
+constexpr int kProducers = 2;                    // warps 0, 1
+constexpr int kIssuerWarp0 = 2;                  // warps 2, 3
+constexpr int kExpWarp0 = 4;                     // warps 4..11
+constexpr int kEpiWarp0 = kExpWarp0 + 8;         // warps 12..15
+constexpr int kThreads = 32 * (kEpiWarp0 + 4);   // 512
+constexpr int kMaxRing = 16;
+constexpr int kSmemMax = 224 * 1024;
+constexpr int kSmemMin = 120 * 1024;             // > half an SM: one CTA per SM
 
 struct DecodeParams {
   const uint32_t* codes;
   const float* alpha;
-  const uint4* frag;
-  const float* scale;
-  float* y;
-  float* part;
-  uint32_t* cnt;
+  const uint8_t* bimg;   // B operand image: KB x NP x 128 bytes
+  const int* sexp;       // per-batch-row scale exponents e_m
+  float* y;              // M x n_out
+  float* part;           // S x M x (ntiles * 128) split-K partials
+  uint32_t* cnt;         // ntiles tickets (zeroed by the prep kernel)
   uint32_t* err;
-  int M, T, n_out, ng, n_chunks;
-  int S, cps, rgc, WK, WR;
+  int M, T, NP, S, P, CB, KB, ring, sb, nbuf, dbase;
+  int n_out, ntiles, ngroups, ternary, early;
+  uint32_t blk_bytes, slot_bytes, b_bytes;
 };
 
-// One tile (4 words per lane) against the bf16 B-fragments of its chunk.
-// Ternary word w: (w << 2j) & 0xC000C000 is a bf16 pair, each half +-2.0 or 0
-// (sign = field bit 1, exponent MSB = field bit 0).  Registers j = 0..3 form
-// the A operand of one 16x8x16 MMA, j = 4..7 of a second one; the k order
-// they imply is matched by the B-fragment order the fragment kernel writes.
-// Binary word: ((~w << j) & 0x80008000) | 0x40004000, j = 0..15, four MMAs.
-template <int QT, int NT, int QA>
-__device__ __forceinline__ void mma_tile(float (&acc)[QA][NT][4], const uint32_t (&wq)[4],
-                                         const uint4* bf, int lanes, bool active) {
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const uint32_t w = wq[q];
-    if (QT == 2) {
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        uint32_t a[4];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) a[j] = (w << (2 * (4 * h + j))) & 0xC000C000u;
-#pragma unroll
-        for (int n = 0; n < NT; ++n) {
-          const uint4 b = active ? bf[(q * NT + n) * lanes] : make_uint4(0, 0, 0, 0);
-          mma_bf16_16816(acc[(2 * q + h) % QA][n], a, h ? b.z : b.x, h ? b.w : b.y);
-        }
-      }
-    } else {
-      const uint32_t nw = ~w;
-#pragma unroll
-      for (int h = 0; h < 4; ++h) {
-        uint32_t a[4];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) a[j] = ((nw << (4 * h + j)) & 0x80008000u) | 0x40004000u;
-#pragma unroll
-        for (int n = 0; n < NT; ++n) {
-          // h = 0, 1: odd fields (k-steps 2q, 2q + 1); h = 2, 3: even fields
-          const uint4 b = active ? bf[((2 * q + (h & 1)) * NT + n) * lanes] : make_uint4(0, 0, 0, 0);
-          mma_bf16_16816(acc[(4 * q + h) % QA][n], a, (h >> 1) ? b.z : b.x, (h >> 1) ? b.w : b.y);
-        }
-      }
-    }
-  }
+// Bounded wait whose outcome is the same for all lanes of the warp (the
+// tcgen05 loads and stores that follow are warp-collective).
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity) {
+  return __all_sync(0xffffffffu, mbar_wait(bar, parity));
+}
+// Barrier over `nthreads` threads that also ANDs a predicate across them.
+__device__ __forceinline__ bool group_and(int id, int nthreads, bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.and.pred q, %2, %3, p;\n"
+      " selp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(r) : "r"((uint32_t)v), "r"(id), "r"(nthreads) : "memory");
+  return r != 0;
 }
 
-__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(smem_u32(dst)), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+// Stage j of a row tile (spu stages over the chunk's ncb blocks) covers
+// blocks [first, last).
+__device__ __forceinline__ int stage_block(int j, int ncb, int spu) { return j * ncb / spu; }
 
-template <int QT, int NT>
-__global__ void __launch_bounds__(256, ctas_per_sm(NT)) decode_kernel(DecodeParams p) {
-  constexpr int KS = QT == 2 ? 4 : 8;                  // 32-code k-steps per chunk
-  constexpr int QA = NT == 1 ? 4 : (NT == 2 ? 2 : 1);  // independent accumulator sets
-  constexpr int D = ring_depth(NT);                    // ring slots per warp
-  extern __shared__ __align__(128) uint8_t smem[];
-  __shared__ __align__(8) uint64_t frag_bar;
-  __shared__ float scale_s[kMaxDecodeM];
-  __shared__ int last_flag;
+__global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t c_full[kMaxRing], c_empty[kMaxRing];
+  __shared__ __align__(8) uint64_t a_full[4], a_empty[4];
+  __shared__ __align__(8) uint64_t acc_full[2][2], acc_empty[2][2], b_full, mma_done[2];
+  __shared__ uint32_t tmem_base;
+  __shared__ int last[128];
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int s = blockIdx.y, r = blockIdx.x;
-  const int c0 = s * p.cps, c1 = min(p.n_chunks, c0 + p.cps);
-  const int rg0 = r * p.rgc, rg1 = min(p.ng, rg0 + p.rgc);
-  const int nc = c1 - c0;                                  // tiles per row group
-  uint8_t* ring = smem + (size_t)warp * D * 512;          // [8 warps][D][512 B]
-  uint4* bfrag = reinterpret_cast<uint4*>(smem + 8 * D * 512);
-  // With one column tile only the lanes of the used columns carry fragments.
-  const int flanes = NT == 1 ? 4 * p.M * p.T : 32;
-  float* wb = reinterpret_cast<float*>(smem + 8 * D * 512 + (size_t)p.cps * KS * NT * flanes * 16) +
-              (size_t)warp * 16 * 8 * NT;
+  const int sidx = blockIdx.x % p.S, prow = blockIdx.x / p.S;
+  const int kb0 = sidx * p.CB;
+  const int ncb = min(p.CB, p.KB - kb0);                        // blocks of this chunk
+  const int spu = max((ncb + p.sb - 1) / p.sb, min(2, ncb));   // stages per tile
+  const int nunits = (p.ntiles - prow + p.P - 1) / p.P;         // row tiles of this CTA
+  const int nstages = nunits * spu;
+  const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
+  uint8_t* base = smem_raw + (sbase - smem_u32(smem_raw));
+  uint8_t* bop = base;                                          // ncb x NP x 128 bytes
+  uint8_t* ring = base + p.b_bytes;                             // ring x slot_bytes
 
   if (tid == 0) {
-    mbar_init(&frag_bar, 1);
+    for (int i = 0; i < p.ring; ++i) {
+      mbar_init(&c_full[i], 1);
+      mbar_init(&c_empty[i], 128);
+    }
+    for (int i = 0; i < 4; ++i) {
+      mbar_init(&a_full[i], 128);
+      mbar_init(&a_empty[i], 1);
+    }
+    for (int e = 0; e < 2; ++e)
+      for (int b = 0; b < 2; ++b) {
+        mbar_init(&acc_full[e][b], 1);
+        mbar_init(&acc_empty[e][b], 128);
+      }
+    mbar_init(&b_full, 1);
+    mbar_init(&mma_done[0], 1);
+    mbar_init(&mma_done[1], 1);
     fence_mbar_init();
   }
+  if (warp == 0) {
+    __syncwarp();
+    tmem_alloc(&tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
   __syncthreads();
+  tc_fence_after();
   pdl_launch_dependents();
+  if (warp >= kProducers || !p.early) pdl_wait();
+  const uint32_t tmem = tmem_base;
+  bool ok = true;
 
-  // The warp's tiles: row groups rg0 + warp, rg0 + warp + 8, ...; all nc
-  // chunks of the slice for each.  Each lane copies 16 of a tile's 512 bytes
-  // (cp.async, one commit group per tile).  Codes do not depend on the
-  // preceding kernels, so the first D - 1 tiles are requested before the
-  // grid waits.
-  const int n_rg_w = rg1 - rg0 - warp > 0 ? (rg1 - rg0 - warp + 7) / 8 : 0;
-  const int total = n_rg_w * nc;
-  const uint8_t* src = reinterpret_cast<const uint8_t*>(
-      p.codes + ((size_t)(rg0 + warp) * p.n_chunks + c0) * 128) + 16 * lane;
-  const size_t rg_jump = (size_t)8 * p.n_chunks * 512 - (size_t)nc * 512;
-  uint8_t* dst = ring + 16 * lane;
-  uint8_t* const ring_end = ring + D * 512;
-  int ld_ci = 0, ld_t = 0;                                 // next tile to request
-  auto request = [&]() {
-    if (ld_t < total) {
-      cp_async16(dst, src);
-      src += 512;
-      if (++ld_ci == nc) { ld_ci = 0; src += rg_jump; }
-    }
-    ++ld_t;
-    dst += 512;
-    if (dst == ring_end + 16 * lane) dst = ring + 16 * lane;
-    cp_async_commit();
-  };
-#pragma unroll 1
-  for (int d = 0; d < D - 1; ++d) request();
-
-  // bf16 B-fragments (written by the fragment kernel) by one bulk copy.
-  pdl_wait();
-  const uint32_t frag_bytes = (uint32_t)(nc * KS * NT * flanes * 16);
-  if (tid == 0) {
-    mbar_expect_tx(&frag_bar, frag_bytes);
-    bulk_g2s(bfrag, p.frag + (size_t)c0 * KS * NT * flanes, frag_bytes, &frag_bar);
-  }
-  if (tid < p.M) scale_s[tid] = p.scale[tid];
-  const bool ok = mbar_wait(&frag_bar, 0);
-  __syncthreads();
-  if (!ok && tid == 0) atomicExch(p.err, 1u);
-
-  const int g = lane >> 2, t4 = lane & 3;
-  const int stride_part = p.ng * 16;
-  float acc[QA][NT][4];
-#pragma unroll
-  for (int a = 0; a < QA; ++a)
-#pragma unroll
-    for (int n = 0; n < NT; ++n)
-#pragma unroll
-      for (int e = 0; e < 4; ++e) acc[a][n][e] = 0.f;
-  int ci = 0, it = 0;
-  const bool active = lane < flanes;
-  const uint32_t* rd = reinterpret_cast<const uint32_t*>(ring) + lane;
-  const uint32_t* const rd_end = reinterpret_cast<const uint32_t*>(ring_end) + lane;
-  const uint4* bfl = bfrag + (active ? lane : 0);
-#pragma unroll 1
-  for (int t = 0; t < total; ++t) {
-    __syncwarp();        // every lane has consumed the slot refilled next
-    request();           // tile t + D - 1 into slot (t - 1) % D
-    cp_async_wait<D - 1>();
-    __syncwarp();        // the other lanes' copies of tile t are visible
-    const uint32_t wq[4] = {rd[0], rd[32], rd[64], rd[96]};
-    rd += 128;
-    if (rd == rd_end) rd = reinterpret_cast<const uint32_t*>(ring) + lane;
-    mma_tile<QT, NT, QA>(acc, wq, bfl + (size_t)ci * KS * NT * flanes, flanes, active);
-    if (++ci == nc) {
-      // Row group done: fold, stage in the warp's smem slot, combine the
-      // terms of every batch row, write y (or the slice partial).
-#pragma unroll
-      for (int n = 0; n < NT; ++n) {
-        float v[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          v[e] = acc[0][n][e];
-#pragma unroll
-          for (int a = 1; a < QA; ++a) v[e] += acc[a][n][e];
-#pragma unroll
-          for (int a = 0; a < QA; ++a) acc[a][n][e] = 0.f;
+  if (warp < kProducers) {
+    if (lane == 0) {
+      // Producer of pipeline `warp`: stages i = warp (mod 2), ring slots
+      // i mod ring (ring is even).  Stage (unit u, j) is the
+      // slabs (tile, 2 b) .. (tile, 2 b' - 1) of its blocks [b, b'),
+      // adjacent in the tiled layout.  Producer 0 also copies the chunk's B
+      // operand: after the first ring of stages when the codes may be read
+      // before the preceding grid is done, before everything otherwise.
+      int last_i = -1;
+      bool b_loaded = warp != 0;
+      const int pre = p.early ? min(p.ring, nstages) : 0;
+      for (int i = warp; i < nstages && ok; i += kProducers) {
+        if (!b_loaded && i >= pre) {
+          if (p.early) pdl_wait();
+          mbar_expect_tx(&b_full, p.b_bytes);
+          bulk_g2s(bop, p.bimg + (size_t)kb0 * p.NP * 128, p.b_bytes, &b_full);
+          b_loaded = true;
         }
-        const int col = n * 8 + 2 * t4;
-        wb[g * 8 * NT + col] = v[0];
-        wb[g * 8 * NT + col + 1] = v[1];
-        wb[(g + 8) * 8 * NT + col] = v[2];
-        wb[(g + 8) * 8 * NT + col + 1] = v[3];
+        const int slot = i % p.ring, r = i / p.ring;
+        if (r > 0) ok = mbar_wait(&c_empty[slot], (r - 1) & 1);
+        if (!ok) break;
+        const int u = i / spu, j = i - u * spu;
+        const int b0 = stage_block(j, ncb, spu), b1 = stage_block(j + 1, ncb, spu);
+        const int tile = prow + u * p.P;
+        const uint8_t* src = reinterpret_cast<const uint8_t*>(p.codes) +
+                             ((size_t)tile * p.KB + kb0 + b0) * p.blk_bytes;
+        const uint32_t bytes = (uint32_t)(b1 - b0) * p.blk_bytes;
+        mbar_expect_tx(&c_full[slot], bytes);
+        bulk_g2s(ring + (size_t)slot * p.slot_bytes, src, bytes, &c_full[slot]);
+        last_i = i;
       }
-      __syncwarp();
-      const int rg = rg0 + warp + 8 * it;
-      for (int idx = lane; idx < 16 * p.M; idx += 32) {
-        const int m = idx % p.M, row16 = idx / p.M;
-        const int row = rg * 16 + row16;
-        if (row < p.n_out) {
-          float tot = 0.f;
-          for (int term = 0; term < p.T; ++term) tot += wb[row16 * 8 * NT + m * p.T + term];
-          const float val = tot / (2.f * scale_s[m]);
-          if (p.S == 1)
-            p.y[(size_t)m * p.n_out + row] = val * __ldg(p.alpha + row);
-          else
-            p.part[((size_t)s * p.M + m) * stride_part + row] = val;
+      if (!b_loaded) {   // producer 0 had no stage at or past `pre`, or failed
+        if (p.early) pdl_wait();
+        if (ok) {
+          mbar_expect_tx(&b_full, p.b_bytes);
+          bulk_g2s(bop, p.bimg + (size_t)kb0 * p.NP * 128, p.b_bytes, &b_full);
+        }
+        b_loaded = ok;
+      }
+      // Every copy this thread issued has landed before the CTA may exit.
+      if (warp == 0 && b_loaded && !mbar_wait(&b_full, 0)) ok = false;
+      for (int i = last_i; i >= 0 && i > last_i - p.ring; i -= kProducers)
+        if (!mbar_wait(&c_full[i % p.ring], (i / p.ring) & 1)) ok = false;
+    }
+  } else if (warp < kExpWarp0) {
+    if (lane == 0) {
+      // MMA issuer of pipeline e: stages i = e (mod 2), the pipeline's j-th
+      // stage (j = i / 2) in TMEM slot e + 2 (j mod 2), into its own
+      // accumulator.
+      const int e = warp - kIssuerWarp0;
+      ok = mbar_wait(&b_full, 0);
+      tc_fence_after();
+      // kind::f8f6f4: D fp32, A and B e4m3, both K-major, N = NP, M = 128.
+      const uint32_t idesc = (1u << 4) | ((uint32_t)(p.NP >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+      int k = 0, prev_u = -1, buf = 0;
+      for (int i = e; i < nstages && ok; i += 2) {
+        const int u = i / spu, j = i - u * spu, jj = i >> 1, a = e + 2 * (jj & 1);
+        const bool first = u != prev_u;
+        if (first) {
+          prev_u = u;
+          buf = k % p.nbuf;
+          if (k >= p.nbuf) {
+            ok = mbar_wait(&acc_empty[e][buf], ((k / p.nbuf) - 1) & 1);
+            if (!ok) break;
+          }
+        }
+        ok = mbar_wait(&a_full[a], (jj >> 1) & 1);
+        if (!ok) break;
+        tc_fence_after();
+        const int b0 = stage_block(j, ncb, spu), nb = stage_block(j + 1, ncb, spu) - b0;
+        const uint32_t dt = tmem + (uint32_t)(p.dbase + (e * p.nbuf + buf) * p.NP);
+        const uint32_t at = tmem + (uint32_t)(a * 32 * p.sb);
+        for (int bb = 0; bb < nb; ++bb) {
+          const uint64_t bd = sw128_desc(sbase + (uint32_t)(b0 + bb) * p.NP * 128);
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            umma_f8_ts(dt, at + 32 * bb + 8 * kk, bd + 2 * kk, idesc, (first && bb == 0 && kk == 0) ? 0u : 1u);
+        }
+        umma_commit(&a_empty[a]);
+        if (i + 2 >= (u + 1) * spu) {   // this pipeline's last stage of the tile
+          umma_commit(&acc_full[e][buf]);
+          ++k;
         }
       }
-      __syncwarp();
-      ci = 0;
-      ++it;
+      umma_commit(&mma_done[e]);   // every MMA issued has finished before TMEM is freed
+      if (!mbar_wait(&mma_done[e], 0)) ok = false;
+      // ... and the last commit to each of this pipeline's TMEM slots has
+      // arrived (those phases have no other waiter).
+      const int njs = (nstages - e + 1) / 2;   // stages of this pipeline
+      for (int jj = max(0, njs - 2); jj < njs; ++jj)
+        if (!mbar_wait(&a_empty[e + 2 * (jj & 1)], (jj >> 1) & 1)) ok = false;
     }
-  }
-  cp_async_wait<0>();
-
-  if (p.S > 1) {
-    __threadfence();
-    __syncthreads();
-    if (tid == 0) {
-      const uint32_t prev = atomicAdd(p.cnt + r, 1u);
-      last_flag = prev == (uint32_t)(p.S - 1);
+  } else if (warp < kEpiWarp0) {
+    // ------------------------------------------------------------ expanders
+    // Warps 4 + 4e .. 7 + 4e expand pipeline e's stages, in order.
+    const int e = (warp - kExpWarp0) >> 2, q = warp & 3, r = 32 * q + lane;
+    const uint32_t lane_addr = tmem + ((uint32_t)(32 * q) << 16);
+    const uint32_t slab = p.blk_bytes / 2;
+    for (int i = e; i < nstages && ok; i += 2) {
+      const int slot = i % p.ring, jj = i >> 1, a = e + 2 * (jj & 1);
+      ok = warp_wait(&c_full[slot], (i / p.ring) & 1);
+      if (!ok) break;
+      if (jj >= 2) {
+        ok = warp_wait(&a_empty[a], ((jj >> 1) - 1) & 1);
+        if (!ok) break;
+        tc_fence_after();
+      }
+      const int u = i / spu, j = i - u * spu;
+      const int nb = stage_block(j + 1, ncb, spu) - stage_block(j, ncb, spu);
+      const uint8_t* cs = ring + (size_t)slot * p.slot_bytes;
+      for (int bb = 0; bb < nb; ++bb) {
+        uint32_t v[32];
+        const uint8_t* cb = cs + bb * p.blk_bytes;
+        if (p.ternary) {
+          const uint4 g0 = *reinterpret_cast<const uint4*>(cb + r * 16);
+          const uint4 g1 = *reinterpret_cast<const uint4*>(cb + slab + r * 16);
+          const uint32_t w[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+#pragma unroll
+          for (int wi = 0; wi < 8; ++wi)
+#pragma unroll
+            for (int jb = 0; jb < 4; ++jb) v[4 * wi + jb] = (w[wi] << (2 * jb)) & 0xC0C0C0C0u;
+        } else {
+          const uint2 g0 = *reinterpret_cast<const uint2*>(cb + r * 8);
+          const uint2 g1 = *reinterpret_cast<const uint2*>(cb + slab + r * 8);
+          const uint32_t w[4] = {~g0.x, ~g0.y, ~g1.x, ~g1.y};
+#pragma unroll
+          for (int wi = 0; wi < 4; ++wi)
+#pragma unroll
+            for (int jb = 0; jb < 8; ++jb) v[8 * wi + jb] = ((w[wi] << jb) & 0x80808080u) | 0x40404040u;
+        }
+        tmem_st32(lane_addr + (uint32_t)(a * 32 * p.sb + 32 * bb), v);
+      }
+      mbar_arrive(&c_empty[slot]);
+      tmem_st_wait();
+      tc_fence_before();
+      mbar_arrive(&a_full[a]);
     }
-    __syncthreads();
-    if (last_flag) {
+  } else {
+    // ------------------------------------------------------------- epilogue
+    const int q = warp & 3, r = 32 * q + lane, et = tid - 32 * kEpiWarp0;
+    const int NR = p.ntiles * kTileRows;
+    const int MT = p.M * p.T;
+    int kc[2] = {0, 0};
+    for (int u = 0; u < nunits && ok; ++u) {
+      // issuers with stages in this tile: both, unless the tile is one stage
+      const bool in0 = spu >= 2 || ((u * spu) & 1) == 0;
+      const bool in1 = spu >= 2 || ((u * spu) & 1) == 1;
+      const int bf0 = kc[0] % p.nbuf, bf1 = kc[1] % p.nbuf;
+      bool w = true;
+      if (in0) w = mbar_wait(&acc_full[0][bf0], (kc[0] / p.nbuf) & 1);
+      if (in1 && w) w = mbar_wait(&acc_full[1][bf1], (kc[1] / p.nbuf) & 1);
+      ok = group_and(2, 128, w);
+      if (!ok) break;
+      tc_fence_after();
+      const int row = (prow + u * p.P) * kTileRows + r;
+      const bool live = row < p.n_out;
+      const float sa = live ? 0.5f * __ldg(p.alpha + row) : 0.f;
+      const uint32_t lq = tmem + ((uint32_t)(32 * q) << 16);
+      const uint32_t d0 = lq + (uint32_t)(p.dbase + bf0 * p.NP);
+      const uint32_t d1 = lq + (uint32_t)(p.dbase + (p.nbuf + bf1) * p.NP);
+      int m = 0, t = 0;
+      float acc = 0.f, wt = 1.f;
+      for (int c0 = 0; c0 < MT; c0 += 16) {
+        uint32_t r0[16], r1[16];
+        if (in0) tmem_ld16(d0 + (uint32_t)c0, r0);
+        if (in1) tmem_ld16(d1 + (uint32_t)c0, r1);
+        tmem_ld_wait();
+        if (c0 + 16 >= MT) {
+          tc_fence_before();
+          if (in0) mbar_arrive(&acc_empty[0][bf0]);
+          if (in1) mbar_arrive(&acc_empty[1][bf1]);
+        }
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          if (c0 + i < MT) {
+            const float dv = (in0 ? __uint_as_float(r0[i]) : 0.f) + (in1 ? __uint_as_float(r1[i]) : 0.f);
+            acc += wt * dv;
+            wt *= 0.0625f;
+            if (++t == p.T) {
+              const float ym = ldexpf(acc, p.sexp[m]);
+              if (p.S == 1) {
+                if (live) p.y[(size_t)m * p.n_out + row] = sa * ym;
+              } else {
+                p.part[((size_t)sidx * p.M + m) * NR + row] = ym;
+              }
+              acc = 0.f; wt = 1.f; t = 0; ++m;
+            }
+          }
+        }
+      }
+      kc[0] += in0;
+      kc[1] += in1;
+    }
+    if (p.S > 1 && ok) {
+      // Split-K: one fence for all of this CTA's partials, then one ticket
+      // per tile; the CTA that takes the last ticket of a tile sums its S
+      // partials in k-chunk order.
       __threadfence();
-      const int row_lo = rg0 * 16, row_hi = min(p.n_out, rg1 * 16);
-      for (int idx = tid; idx < (row_hi - row_lo) * p.M; idx += 256) {
-        const int m = idx / (row_hi - row_lo), row = row_lo + idx % (row_hi - row_lo);
-        float v = 0.f;
-        for (int ss = 0; ss < p.S; ++ss) v += __ldcg(p.part + ((size_t)ss * p.M + m) * stride_part + row);
-        p.y[(size_t)m * p.n_out + row] = v * __ldg(p.alpha + row);
+      named_bar_sync(2, 128);
+      for (int u0 = 0; u0 < nunits; u0 += 128) {
+        const int u = u0 + et;
+        last[et] = u < nunits && atomicAdd(p.cnt + prow + u * p.P, 1u) == (uint32_t)(p.S - 1);
+        named_bar_sync(2, 128);
+        __threadfence();
+        for (int uu = 0; uu < min(128, nunits - u0); ++uu) {
+          if (!last[uu]) continue;
+          const int row = (prow + (u0 + uu) * p.P) * kTileRows + r;
+          if (row >= p.n_out) continue;
+          const float sa = 0.5f * __ldg(p.alpha + row);
+          const size_t sstride = (size_t)p.M * NR;
+          for (int mm = 0; mm < p.M; ++mm) {
+            const float* pr = p.part + (size_t)mm * NR + row;
+            float s0 = 0.f;
+            int kk = 0;
+            for (; kk + 4 <= p.S; kk += 4) {
+              const float a0 = __ldcg(pr + (size_t)kk * sstride), a1 = __ldcg(pr + (size_t)(kk + 1) * sstride);
+              const float a2 = __ldcg(pr + (size_t)(kk + 2) * sstride), a3 = __ldcg(pr + (size_t)(kk + 3) * sstride);
+              s0 = (((s0 + a0) + a1) + a2) + a3;
+            }
+            for (; kk < p.S; ++kk) s0 += __ldcg(pr + (size_t)kk * sstride);
+            p.y[(size_t)mm * p.n_out + row] = sa * s0;
+          }
+        }
+        named_bar_sync(2, 128);
       }
-      if (tid == 0) p.cnt[r] = 0u;
     }
+  }
+  if (!ok) atomicExch(p.err, 1u);
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    __syncwarp();   // warp-collective: lane 0 ran the producer loop alone
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
   }
 }
 
-template <int QT, int NT>
-cudaError_t launch_t(const DecodeConfig& dc, const DecodeParams& p, cudaStream_t st) {
-  auto k = decode_kernel<QT, NT>;
-  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dc.smem);
-  if (e != cudaSuccess) return e;
-  return launch_pdl(k, dim3(dc.R, dc.S), dim3(256), dc.smem, st, p);
+// TMEM split for N = NP: accumulators (2 pipelines x nbuf buffers x NP
+// columns) at the top, four A slots of sb blocks (32 sb columns) below.
+void tmem_split(int NP, int* sb, int* nbuf, int* dbase) {
+  *nbuf = NP <= 32 ? 2 : 1;
+  const int dcols = 2 * *nbuf * NP;
+  *sb = std::min(4, (512 - dcols) / (4 * 32));
+  *dbase = 512 - dcols;
 }
-
-int round_nt(int nt) { return nt <= 1 ? 1 : nt <= 2 ? 2 : nt <= 4 ? 4 : nt <= 8 ? 8 : 16; }
 
 }  // namespace
 
+// Launch shape for batch M: the (S, P) grid of at most one CTA per SM that
+// minimises a simple time model: the larger of the MMA time of the busiest
+// CTA and the HBM time of codes plus split-K partials (the bytes in flight
+// capped by the CTAs' code rings), plus the split-K tail (one fence, one
+// ticket, the final sums).
 DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
   const Geometry& g = pl->geo;
-  DecodeConfig dc{};
-  dc.M = M;
-  dc.T = decode_terms(M);
-  dc.NT = round_nt(decode_ntiles(M));
-  dc.P = prep_partials(pl, M);
-  dc.WK = 1;
-  dc.WR = 8;
-  const int KS = g.kc / 32;
-  const int flanes = dc.NT == 1 ? 4 * M * dc.T : 32;
-  const size_t frag_per_chunk = (size_t)KS * dc.NT * flanes * 16;
-  const int cpsm = ctas_per_sm(dc.NT);
-  const size_t fixed = (size_t)8 * ring_depth(dc.NT) * 512 + (size_t)8 * 16 * 8 * dc.NT * 4 + 1024;
-  const size_t budget = (size_t)(cpsm == 3 ? 72 : cpsm == 2 ? 110 : 220) * 1024;
-  int max_cps = (int)((budget - fixed) / frag_per_chunk);
-  if (max_cps < 1) max_cps = 1;
-  const int slots = pl->sm_count * cpsm;
-  double best = 1e30;
-  for (int S = 1; S <= g.n_chunks && S <= 64; ++S) {
-    const int cps = (g.n_chunks + S - 1) / S;
-    if (cps > max_cps) continue;
-    if ((g.n_chunks + cps - 1) / cps != S) continue;
-    // Row ranges near whole waves of CTAs, and one range per 8 groups.
-    int cand[32], nc = 0;
-    for (int w = 1; w <= 4; ++w) {
-      const int base = (w * slots) / S;
-      for (int dR = -2; dR <= 2; ++dR) cand[nc++] = base + dR;
-    }
-    cand[nc++] = (g.ng + 7) / 8;
-    for (int ci = 0; ci < nc; ++ci) {
-      const int Rr = cand[ci];
-      if (Rr < 1 || Rr > g.ng) continue;
-      const int rgc = (g.ng + Rr - 1) / Rr;
-      const int R = (g.ng + rgc - 1) / rgc;
-      const int waves = (S * R + slots - 1) / slots;
-      // per-warp cost in tiles (+ an epilogue term per row group, + prologue)
-      const double rg_w = (double)((rgc + 7) / 8);
-      const double per = rg_w * (cps + 1.0) + (double)cps * KS * dc.NT / 512.0 + 2.0;
-      const double tcost = waves * per + (S > 1 ? 0.01 * S * M : 0.0);
-      if (tcost < best - 1e-9) {
-        best = tcost;
-        dc.S = S; dc.R = R; dc.cps = cps; dc.rgc = rgc;
+  DecodeConfig best{};
+  best.M = M;
+  best.T = decode_terms(M);
+  best.NP = (M * best.T + 15) / 16 * 16;
+  best.pp = prep_partials(pl, M);
+  const int KB = (int)(g.k_eff_pad / kBlk);
+  const int sms = std::max(1, pl->sm_count);
+  const int blk_bytes = kTileRows * kBlk * g.bits / 8;
+  int sb = 0, nbuf = 0, dbase = 0;
+  tmem_split(best.NP, &sb, &nbuf, &dbase);
+  const int slot_bytes = sb * blk_bytes;
+  const double clk = 1.9e9, bw = 6.5e12, latency = 1.5e-6;
+  const double t_mma = std::max(38.0, best.NP * 0.4) / clk;     // per MMA, two issuers
+  const double code_bytes = (double)g.ntiles * kTileRows * g.k_eff_pad * g.bits / 8;
+  double best_t = 1e30;
+  for (int S = 1; S <= std::min(KB, sms); ++S) {
+    const int CB = (KB + S - 1) / S;
+    if ((S - 1) * CB >= KB) continue;                      // no empty chunk
+    const int b_bytes = CB * best.NP * 128;
+    int ring = std::min(kMaxRing, (kSmemMax - 2048 - b_bytes) / slot_bytes);
+    ring -= ring % kProducers;
+    if (ring < 4) continue;
+    const int spu = std::max((CB + sb - 1) / sb, std::min(2, CB));
+    for (int P = 1; P <= std::min(g.ntiles, sms / S); ++P) {
+      const int grid = S * P;
+      const int units = (g.ntiles + P - 1) / P;
+      const double inflight = (double)grid * ring * slot_bytes;
+      const double bw_eff = std::min(bw, inflight / latency);
+      const double part_bytes = S > 1 ? 8.0 * S * M * g.ntiles * kTileRows : 0.0;
+      const double tail = S > 1 ? 2.5e-6 + (double)M * S * kTileRows * 4 / 40e9 : 0.0;
+      const double t_cta = units * (4.0 * CB * t_mma + spu * 90.0 / clk + 300.0 / clk);
+      const double t = std::max(t_cta, (code_bytes + part_bytes) / bw_eff) + tail;
+      if (t < best_t * 0.999) {
+        best_t = t;
+        best.S = S; best.P = P; best.CB = CB; best.ring = ring;
+        best.smem = std::max<size_t>(kSmemMin, 1024 + (size_t)b_bytes + (size_t)ring * slot_bytes);
       }
     }
   }
-  dc.smem = (size_t)8 * ring_depth(dc.NT) * 512 + (size_t)dc.cps * frag_per_chunk +
-            (size_t)8 * 16 * 8 * dc.NT * 4;
-  return dc;
+  return best;
 }
 
 cudaError_t launch_decode(const sdq_plan_s* pl, const uint32_t* codes, const float* alpha, int M,
-                          float* y, void* ws, cudaStream_t st) {
+                          float* y, void* ws, cudaStream_t st, int early) {
   const Geometry& g = pl->geo;
   const DecodeConfig& dc = decode_config(pl, M);
+  if (dc.S < 1) return cudaErrorNotSupported;   // the B operand of a k chunk does not fit
   const WsLayout L = workspace_layout(pl, M);
   uint8_t* base = static_cast<uint8_t*>(ws);
   DecodeParams p;
-  p.codes = codes; p.alpha = alpha;
-  p.frag = reinterpret_cast<const uint4*>(base + L.frag);
-  p.scale = reinterpret_cast<const float*>(base + L.scale);
+  p.codes = codes; p.alpha = alpha; p.y = y;
+  p.bimg = base + L.bimg;
+  p.sexp = reinterpret_cast<const int*>(base + L.sexp);
   p.part = reinterpret_cast<float*>(base + L.part);
   p.cnt = reinterpret_cast<uint32_t*>(base + L.cnt);
   p.err = reinterpret_cast<uint32_t*>(base + L.err);
-  p.y = y;
-  p.M = M; p.T = dc.T; p.n_out = g.n_out; p.ng = g.ng; p.n_chunks = g.n_chunks;
-  p.S = dc.S; p.cps = dc.cps; p.rgc = dc.rgc; p.WK = dc.WK; p.WR = dc.WR;
-  const bool tern = pl->desc.quantizer == SDQ_TERNARY;
-  switch (dc.NT) {
-    case 1: return tern ? launch_t<2, 1>(dc, p, st) : launch_t<1, 1>(dc, p, st);
-    case 2: return tern ? launch_t<2, 2>(dc, p, st) : launch_t<1, 2>(dc, p, st);
-    case 4: return tern ? launch_t<2, 4>(dc, p, st) : launch_t<1, 4>(dc, p, st);
-    case 8: return tern ? launch_t<2, 8>(dc, p, st) : launch_t<1, 8>(dc, p, st);
-    default: return tern ? launch_t<2, 16>(dc, p, st) : launch_t<1, 16>(dc, p, st);
-  }
+  p.M = M; p.T = dc.T; p.NP = dc.NP; p.S = dc.S; p.P = dc.P; p.CB = dc.CB;
+  p.KB = (int)(g.k_eff_pad / kBlk); p.ring = dc.ring;
+  tmem_split(dc.NP, &p.sb, &p.nbuf, &p.dbase);
+  p.n_out = g.n_out; p.ntiles = g.ntiles; p.ngroups = g.ngroups; p.ternary = g.bits == 2;
+  p.early = early;
+  p.blk_bytes = (uint32_t)(kTileRows * kBlk * g.bits / 8);
+  p.slot_bytes = p.sb * p.blk_bytes;
+  p.b_bytes = (uint32_t)(dc.CB * dc.NP * 128);
+  cudaError_t e = cudaFuncSetAttribute(decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)dc.smem);
+  if (e != cudaSuccess) return e;
+  return launch_pdl(decode_kernel, dim3(dc.S * dc.P), dim3(kThreads), dc.smem, st, p);
 }
 
 }  // namespace sdq

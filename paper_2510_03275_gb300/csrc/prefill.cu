@@ -10,14 +10,16 @@
 // 128-byte-swizzled operand layout of tcgen05.mma.
 //
 // CTA tile 128 (M) x 256 (N), 64 codes per pipeline stage, kStages stages:
-//   warp 0      TMEM allocation; lane 0 issues the TMA loads of the A tile
-//               and of the packed code words of every stage
+//   warp 0      TMEM allocation; lane 0 issues the TMA load of the A tile
+//               and the bulk copies of the stage's two code slabs (tiled
+//               layout: 128 rows x 64 codes each, contiguous)
 //   warp 1      lane 0 issues tcgen05.mma (4 x K=16 per stage), commits to
 //               the stage's "empty" barrier, finally to the accumulator one
-//   warps 2..9  expand the B tile of every stage (one 16-byte smem chunk per
-//               8 codes of one row; the shift-and-mask expansion of a tiled
-//               word yields its codes in the permuted order the prep kernel
-//               also uses for A), then read the fp32 accumulator out of TMEM
+//   warps 2..9  expand the B tile of every stage, one thread per code row:
+//               the row's 64 codes (4 ternary / 2 binary words) become the
+//               row's 128-byte line of bf16 (the shift-and-mask expansion
+//               yields the codes in the permuted order the prep kernel also
+//               uses for A), then read the fp32 accumulator out of TMEM
 //               (tcgen05.ld), scale by alpha / 2 and store y.
 // Every wait on an mbarrier is bounded (about 2 s); a timeout sets the
 // workspace error word and the CTA finishes without further waits.
@@ -35,7 +37,7 @@ namespace {
 constexpr int kBM = 128, kBN = 256, kBK = 64, kStages = 4;
 constexpr int kATile = kBM * kBK * 2;     // 16 KB
 constexpr int kBTile = kBN * kBK * 2;     // 32 KB
-constexpr int kCTile = 16 * 64 * 4;       // packed codes of a stage: 16 row groups x 256 bytes
+constexpr int kCTile = kBN * 16;          // packed codes of a stage: 2 slabs of up to 2 KB
 constexpr int kSmem = kStages * (kATile + kBTile + kCTile) + 1024;
 constexpr int kThreads = 320;   // 2 control warps + 8 expander / epilogue warps
 constexpr int kExp = 256;       // expander threads
@@ -45,71 +47,8 @@ struct PrefillParams {
   const float* alpha;
   float* y;
   uint32_t* err;
-  int M, N, ng, n_chunks, nks, quantizer;
+  int M, N, ntiles, ngroups, wpg, nks, quantizer;
 };
-
-// ----------------------------------------------------------- PTX wrappers
-__device__ __forceinline__ void tmem_alloc(uint32_t* dst, uint32_t ncols) {
-  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_u32(dst)),
-               "r"(ncols) : "memory");
-}
-__device__ __forceinline__ void tmem_relinquish() {
-  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
-}
-__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
-  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(taddr), "r"(ncols) : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
-}
-__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                          uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
-      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate) : "memory");
-}
-__device__ __forceinline__ void umma_commit(uint64_t* bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(
-                   smem_u32(bar)) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(smem_u32(bar)) : "memory");
-}
-__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int c0, int c1,
-                                            uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3}], [%4];\n" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(smem_u32(bar)) : "memory");
-}
-// 32 TMEM lanes x 16 columns of 32-bit values: register i of the thread of
-// lane l holds (lane base + l, column + i).
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15},"
-      " [%16];\n"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-        "=r"(r[14]), "=r"(r[15])
-      : "r"(taddr));
-}
-__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory"); }
-
-// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
-// 1024 bytes apart (SBO), start address in 16-byte units.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
-  uint64_t d = 0;
-  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
-  d |= (uint64_t)1 << 16;                 // leading byte offset (unused for swizzled K-major)
-  d |= (uint64_t)(1024 >> 4) << 32;       // stride byte offset
-  d |= (uint64_t)1 << 46;                 // descriptor version
-  d |= (uint64_t)2 << 61;                 // SWIZZLE_128B
-  return d;
-}
 
 // Instruction descriptor, kind::f16: D fp32, A and B bf16, both K-major.
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) |
@@ -122,12 +61,10 @@ __device__ __forceinline__ void st_chunk(uint8_t* btile, int n, int c8, uint32_t
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-    prefill_kernel(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap cmap,
-                   PrefillParams p) {
+    prefill_kernel(const __grid_constant__ CUtensorMap amap, PrefillParams p) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_a[kStages], full_b[kStages], empty[kStages], acc_bar;
   __shared__ uint32_t tmem_base;
-  __shared__ int fail;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int n0 = blockIdx.x * kBN, m0 = blockIdx.y * kBM;
@@ -135,8 +72,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* base = smem_raw + (sbase - smem_u32(smem_raw));
   uint8_t* a_tiles = base;
   uint8_t* b_tiles = base + kStages * kATile;
-  const uint32_t* c_tiles = reinterpret_cast<const uint32_t*>(base + kStages * (kATile + kBTile));
-  const int cwords = p.quantizer == SDQ_TERNARY ? 64 : 32;      // words per row group per stage
+  uint8_t* c_tiles = base + kStages * (kATile + kBTile);
+  const uint32_t slab_bytes = (uint32_t)(kTileRows * p.wpg * 4);
+  const int tile0 = blockIdx.x * (kBN / kTileRows);
+  const int nslabs = min(kBN / kTileRows, p.ntiles - tile0);   // code slabs present per stage
 
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -145,7 +84,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&empty[s], 1);
     }
     mbar_init(&acc_bar, 1);
-    fail = 0;
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -163,17 +101,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       // Producer: TMA of the x_tilde tile [m0, m0+128) x [64 ks, 64 ks + 64)
-      // and of the packed code words of the same 64 codes for the CTA's 16
-      // row groups (one 2-D box of the tiled layout; rows past N read 0).
+      // and bulk copies of the code slabs (tile, group ks) of the CTA's
+      // tiles (k group = stage: 64 codes).  A tile past the last one is not
+      // copied; its rows are never stored.
       for (int ks = 0; ks < p.nks && ok; ++ks) {
         const int s = ks % kStages, r = ks / kStages;
         if (r > 0) ok = mbar_wait(&empty[s], (r - 1) & 1);
         if (!ok) break;
-        const int cx = p.quantizer == SDQ_TERNARY ? (ks >> 1) * 128 + 64 * (ks & 1)
-                                                   : (ks >> 2) * 128 + 32 * (ks & 3);
-        mbar_expect_tx(&full_a[s], kATile + 16 * cwords * 4);
+        mbar_expect_tx(&full_a[s], kATile + nslabs * slab_bytes);
         tma_load_2d(a_tiles + s * kATile, &amap, ks * kBK, m0, &full_a[s]);
-        tma_load_2d(base + kStages * (kATile + kBTile) + s * kCTile, &cmap, cx, n0 >> 4, &full_a[s]);
+        for (int t = 0; t < nslabs; ++t) {
+          const uint32_t* src = p.codes + (size_t)((int64_t)(tile0 + t) * p.ngroups + ks) * (slab_bytes / 4);
+          bulk_g2s(c_tiles + s * kCTile + t * slab_bytes, src, slab_bytes, &full_a[s]);
+        }
       }
     }
   } else if (warp == 1) {
@@ -193,43 +133,39 @@ __global__ void __launch_bounds__(kThreads, 1)
       umma_commit(&acc_bar);
     }
   } else {
-    // B expanders: kExp threads.  Lane -> (g = lane % 8, t = lane / 8) so
-    // the 8 lanes of each 128-bit store phase hit 8 distinct 16-byte banks.
-    const int et = tid - 64;
-    const int g = lane & 7, t = lane >> 3, L = 4 * g + t;
+    // B expanders: thread et = code row n of the CTA tile (slab n / 128,
+    // row n % 128).  Each thread writes its row's 128-byte line; the 8 lanes
+    // of a 128-bit store phase hold 8 consecutive rows, whose swizzled chunk
+    // positions differ, so the stores are free of bank conflicts.
+    const int n = tid - 64;
     for (int ks = 0; ks < p.nks && ok; ++ks) {
       const int s = ks % kStages, r = ks / kStages;
       if (r > 0) ok = mbar_wait(&empty[s], (r - 1) & 1);
       if (ok) ok = mbar_wait(&full_a[s], r & 1);             // packed codes have landed
       if (!ok) break;
       uint8_t* bt = b_tiles + s * kBTile;
-      const uint32_t* ct = c_tiles + s * (kCTile / 4);
+      const uint8_t* cs = c_tiles + s * kCTile + (n >> 7) * slab_bytes;
       if (p.quantizer == SDQ_TERNARY) {
+        const uint4 w4 = *reinterpret_cast<const uint4*>(cs + (n & 127) * 16);
+        const uint32_t w[4] = {w4.x, w4.y, w4.z, w4.w};
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int idx = (et >> 5) + 8 * u;            // (row group, word half) pair
-          const int rgl = idx >> 1, qh = idx & 1;
-          const uint32_t w = ct[rgl * 64 + 32 * qh + L];
+        for (int i = 0; i < 4; ++i) {
           uint32_t v[8];
 #pragma unroll
-          for (int j = 0; j < 8; ++j) v[j] = (w << (2 * j)) & 0xC000C000u;
-          const int n = 16 * rgl + g, c8 = 4 * qh + t;
-          st_chunk(bt, n, c8, v[0], v[2], v[4], v[6]);
-          st_chunk(bt, n + 8, c8, v[1], v[3], v[5], v[7]);
+          for (int j = 0; j < 8; ++j) v[j] = (w[i] << (2 * j)) & 0xC000C000u;
+          st_chunk(bt, n, 2 * i, v[0], v[1], v[2], v[3]);
+          st_chunk(bt, n, 2 * i + 1, v[4], v[5], v[6], v[7]);
         }
       } else {
+        const uint2 w2 = *reinterpret_cast<const uint2*>(cs + (n & 127) * 8);
+        const uint32_t w[2] = {~w2.x, ~w2.y};
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          const int rgl = (et >> 5) + 8 * u;
-          const uint32_t nw = ~ct[rgl * 32 + L];
+        for (int i = 0; i < 2; ++i) {
           uint32_t v[16];
 #pragma unroll
-          for (int j = 0; j < 16; ++j) v[j] = ((nw << j) & 0x80008000u) | 0x40004000u;
-          const int n = 16 * rgl + g;
-          st_chunk(bt, n, t, v[0], v[2], v[8], v[10]);
-          st_chunk(bt, n, 4 + t, v[4], v[6], v[12], v[14]);
-          st_chunk(bt, n + 8, t, v[1], v[3], v[9], v[11]);
-          st_chunk(bt, n + 8, 4 + t, v[5], v[7], v[13], v[15]);
+          for (int j = 0; j < 16; ++j) v[j] = ((w[i] << j) & 0x80008000u) | 0x40004000u;
+#pragma unroll
+          for (int c = 0; c < 4; ++c) st_chunk(bt, n, 4 * i + c, v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
         }
       }
       fence_proxy_async_smem();
@@ -267,13 +203,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   }
-  if (!ok) {
-    fail = 1;
-    atomicExch(p.err, 1u);
-  }
+  if (!ok) atomicExch(p.err, 1u);
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {
+    __syncwarp();   // warp-collective: lane 0 ran the producer loop alone
     tc_fence_after();
     tmem_dealloc(tmem, kBN);
   }
@@ -311,25 +245,16 @@ cudaError_t launch_prefill(const sdq_plan_s* pl, const uint32_t* codes, const fl
                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
-  // Tiled codes as a 2-D array: one row per row group, n_chunks * 128 words.
-  CUtensorMap cmap;
-  const cuuint64_t cdims[2] = {(cuuint64_t)g.n_chunks * 128, (cuuint64_t)g.ng};
-  const cuuint64_t cstrides[1] = {(cuuint64_t)g.n_chunks * 512};
-  const cuuint32_t cbox[2] = {(cuuint32_t)(pl->desc.quantizer == SDQ_TERNARY ? 64 : 32), 16};
-  cr = enc(&cmap, CU_TENSOR_MAP_DATA_TYPE_UINT32, 2, const_cast<uint32_t*>(codes), cdims, cstrides, cbox,
-           estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
   PrefillParams p;
   p.codes = codes; p.alpha = alpha; p.y = y;
   p.err = reinterpret_cast<uint32_t*>(wbase + L.err);
-  p.M = M; p.N = g.n_out; p.ng = g.ng; p.n_chunks = g.n_chunks;
+  p.M = M; p.N = g.n_out; p.ntiles = g.ntiles; p.ngroups = g.ngroups; p.wpg = g.wpg;
   p.nks = (int)(g.k_eff_pad / kBK);
   p.quantizer = pl->desc.quantizer;
   cudaError_t e = cudaFuncSetAttribute(prefill_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
   if (e != cudaSuccess) return e;
   dim3 grid((g.n_out + kBN - 1) / kBN, (M + kBM - 1) / kBM);
-  return launch_pdl(prefill_kernel, grid, dim3(kThreads), (size_t)kSmem, st, amap, cmap, p);
+  return launch_pdl(prefill_kernel, grid, dim3(kThreads), (size_t)kSmem, st, amap, p);
 }
 
 }  // namespace sdq

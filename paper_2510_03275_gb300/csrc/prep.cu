@@ -9,9 +9,8 @@
 // the pair ~2^-16), accumulation in fp32.
 //
 // Decode path (M <= 64): fp32 x_tilde (M x K_eff_pad) plus max |x_tilde|
-// per CTA and batch row; then the fragment kernel below turns x_tilde into
-// the bf16 B-operand fragments of the decode MMAs (hi and lo bf16 terms for
-// M <= 16, hi only above).  Prefill path: bf16 x_tilde in the permuted
+// per CTA and batch row; then the terms kernel below writes the decode
+// kernel's e4m3 B operand.  Prefill path: bf16 x_tilde in the permuted
 // 64-code stage order of the prefill kernel's operand tiles.
 #include "common.cuh"
 
@@ -33,7 +32,7 @@ struct PrepParams {
   int ncnt;
   int M, K, B, n_b, nblk, P, JT;
   int64_t k_eff, kpad;
-  int prefill, vec;
+  int prefill, vec, ternary;
 };
 
 // CTA tile: TB blocks (rows) x 64 samples j, 4 warps.  TB = 64: each warp
@@ -124,7 +123,7 @@ __global__ void __launch_bounds__(128) prep_kernel(PrepParams p) {
         const int64_t kk = (int64_t)b * p.n_b + j;
         const float v = acc[n][e];
         if (p.prefill) {
-          const int64_t phys = (kk & ~int64_t(63)) | prefill_perm64((int)(kk & 63));
+          const int64_t phys = (kk & ~int64_t(63)) | prefill_pos64((int)(kk & 63), p.ternary);
           p.xtb[(size_t)m * p.kpad + phys] = float_to_bf16_bits(v);
         } else {
           p.xt[(size_t)m * p.kpad + kk] = v;
@@ -144,7 +143,7 @@ __global__ void __launch_bounds__(128) prep_kernel(PrepParams p) {
   if (jt == 0 && bt == 0) {
     for (int64_t k = p.k_eff + tid; k < p.kpad; k += 128) {
       if (p.prefill) {
-        const int64_t phys = (k & ~int64_t(63)) | prefill_perm64((int)(k & 63));
+        const int64_t phys = (k & ~int64_t(63)) | prefill_pos64((int)(k & 63), p.ternary);
         p.xtb[(size_t)m * p.kpad + phys] = 0;
       } else {
         p.xt[(size_t)m * p.kpad + k] = 0.f;
@@ -155,53 +154,76 @@ __global__ void __launch_bounds__(128) prep_kernel(PrepParams p) {
   }
 }
 
-// ------------------------------------------------------- bf16 fragments
-// B operand of the decode MMAs, in the order one lane reads it: entry
-// (k-step ks, column tile nt, lane (g, t)) is a uint4 of bf16 pairs (with a
-// single column tile only the lanes of used columns, g < M * T, are stored)
-//   .x = (xt[4t+1], xt[4t+3])        .y = (xt[16+4t+1], xt[16+4t+3])
-//   .z = (xt[4t],   xt[4t+2])        .w = (xt[16+4t],   xt[16+4t+2])
-// (offsets from 32 ks) of column n = 8 nt + g = (batch m, term): term 0 is
-// bf16(xt), term 1 is bf16(xt - term 0).  This is the k order implied by the
-// shift-and-mask expansion of the tiled code words.
-struct FragParams {
+// ------------------------------------------------------------ e4m3 terms
+// B operand of the decode MMAs for the whole K range: block kb (128 codes)
+// is NP rows x 128 bytes in the 128-byte-swizzled K-major layout, row
+// n = m T + t holding term t of batch row m at MMA K index kap (natural code
+// decode_stage_k(kap)).  With e_m chosen so that max |x_tilde[m]| 2^-e_m <
+// 448, v = x_tilde 2^-e_m splits into sum_t 16^-t q_t: q_t = e4m3(v_t),
+// v_{t+1} = 16 (v_t - q_t) (exact: e4m3 rounding is relative, the residual
+// has few bits).  Rows past M T are not written: they only feed
+// accumulator columns that are never read.  One thread per (kb, m, 16-byte
+// chunk); e_m also goes to sexp for the decode epilogue.
+struct TermsParams {
   const float* xt;
-  uint4* frag;
-  float* scale;
-  int M, T, NT, lanes;   // lanes per (k-step, tile): 32, or 4 * M * T with one tile
-  int64_t kpad, total;
+  const float* pmax;
+  uint8_t* bimg;
+  int* sexp;
+  int M, T, NP, pp, KB, ternary;
+  int64_t kpad;
 };
 
-__device__ __forceinline__ uint32_t bf16_term(float v, int term) {
-  const uint32_t hi = float_to_bf16_bits(v);
-  if (term == 0) return hi;
-  return float_to_bf16_bits(v - bf16_bits_to_float((uint16_t)hi));
-}
-
-__device__ __forceinline__ uint32_t bf16_pair(const float* xr, int i0, int i1, int term) {
-  return bf16_term(xr[i0], term) | (bf16_term(xr[i1], term) << 16);
-}
-
-__global__ void __launch_bounds__(256) frag_kernel(FragParams p) {
+__global__ void __launch_bounds__(256) terms_kernel(TermsParams p) {
+  __shared__ int se[kMaxDecodeM];
   pdl_wait();
   pdl_launch_dependents();
-  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx < p.M && blockIdx.x == 0) p.scale[idx] = 1.f;
-  if (idx >= p.total) return;
-  const int ln = (int)(idx % p.lanes);
-  const int nt = (int)((idx / p.lanes) % p.NT);
-  const int64_t ks = idx / ((int64_t)p.lanes * p.NT);
-  const int g = ln >> 2, t = ln & 3, n = nt * 8 + g;
-  uint4 v = make_uint4(0, 0, 0, 0);
-  if (n < p.M * p.T) {
-    const int m = n / p.T, term = n - m * p.T;
-    const float* xr = p.xt + (size_t)m * p.kpad + ks * 32 + 4 * t;
-    v.x = bf16_pair(xr, 1, 3, term);
-    v.y = bf16_pair(xr, 17, 19, term);
-    v.z = bf16_pair(xr, 0, 2, term);
-    v.w = bf16_pair(xr, 16, 18, term);
+  const int tid = threadIdx.x;
+  if (tid < p.M) {
+    float mx = 0.f;
+    for (int i = 0; i < p.pp; ++i) mx = fmaxf(mx, p.pmax[(size_t)tid * p.pp + i]);
+    int e = 0;
+    if (mx > 0.f) frexpf(mx / 448.f, &e);   // max |x_tilde| * 2^-e < 448
+    e = max(e, -120);
+    se[tid] = e;
+    if (blockIdx.x == 0) p.sexp[tid] = e;
   }
-  p.frag[idx] = v;
+  __syncthreads();
+  const int64_t it = (int64_t)blockIdx.x * blockDim.x + tid;
+  if (it >= (int64_t)p.KB * p.M * 8) return;
+  const int ch = (int)(it & 7);
+  const int64_t mk = it >> 3;
+  const int m = (int)(mk % p.M);
+  const int64_t kb = mk / p.M;
+  const float* xr = p.xt + (size_t)m * p.kpad + (size_t)kb * 128;
+  const float inv = ldexpf(1.f, -se[m]);
+  float v[16];
+  if (p.ternary) {
+    // K indices 16 ch .. 16 ch + 15 hold codes 16 ch .. 16 ch + 15, permuted
+    const float4* x4 = reinterpret_cast<const float4*>(xr + 16 * ch);
+    float xv[16];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float4 f = x4[q];
+      xv[4 * q] = f.x; xv[4 * q + 1] = f.y; xv[4 * q + 2] = f.z; xv[4 * q + 3] = f.w;
+    }
+#pragma unroll
+    for (int u = 0; u < 16; ++u) v[u] = xv[decode_stage_k(u, true)] * inv;
+  } else {
+#pragma unroll
+    for (int u = 0; u < 16; ++u) v[u] = xr[decode_stage_k(16 * ch + u, false)] * inv;
+  }
+  uint8_t* dst = p.bimg + (size_t)kb * p.NP * 128;
+  for (int t = 0; t < p.T; ++t) {
+    uint32_t w[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+    for (int u = 0; u < 16; ++u) {
+      const uint32_t q = f32_to_e4m3(v[u]);
+      w[u >> 2] |= q << (8 * (u & 3));
+      v[u] = (v[u] - e4m3_to_f32(q)) * 16.f;
+    }
+    const int n = m * p.T + t;
+    *reinterpret_cast<uint4*>(dst + n * 128 + ((ch ^ (n & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+  }
 }
 
 }  // namespace
@@ -217,6 +239,7 @@ cudaError_t launch_prep(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws
   p.xtb = p.prefill ? reinterpret_cast<uint16_t*>(base + L.xt) : nullptr;
   p.M = M; p.K = g.k_in; p.B = g.block; p.n_b = g.n_b; p.nblk = g.nblk;
   p.k_eff = g.k_eff; p.kpad = g.k_eff_pad;
+  p.ternary = pl->desc.quantizer == SDQ_TERNARY;
   p.vec = (g.block % 32 == 0) && ((reinterpret_cast<uintptr_t>(x) & 15u) == 0);
   const bool small = (int64_t)M * g.nblk < 4 * (int64_t)pl->sm_count;
   const int TB = small ? 16 : 64;
@@ -228,10 +251,9 @@ cudaError_t launch_prep(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws
     p.cnt = reinterpret_cast<uint32_t*>(base + L.err);   // the error word
     p.ncnt = 1;
   } else {
-    const DecodeConfig& dc = decode_config(pl, M);
     p.pmax = reinterpret_cast<float*>(base + L.pmax);
     p.cnt = reinterpret_cast<uint32_t*>(base + L.cnt);
-    p.ncnt = dc.R + 1;   // the counters and the error word that follows them
+    p.ncnt = g.ntiles + 1;   // the tile tickets and the error word that follows them
   }
   dim3 grid(p.JT, BT, M);
   return small ? launch_pdl(prep_kernel<16>, grid, dim3(128), 0, st, p)
@@ -245,21 +267,22 @@ int prep_partials(const sdq_plan_s* pl, int M) {
   return ((g.n_b + 63) / 64) * ((g.nblk + TB - 1) / TB);
 }
 
-cudaError_t launch_frag(const sdq_plan_s* pl, int M, void* ws, cudaStream_t st) {
+cudaError_t launch_terms(const sdq_plan_s* pl, int M, void* ws, cudaStream_t st) {
   const Geometry& g = pl->geo;
   const WsLayout L = workspace_layout(pl, M);
   const DecodeConfig& dc = decode_config(pl, M);
   uint8_t* base = static_cast<uint8_t*>(ws);
-  FragParams p;
+  TermsParams p;
   p.xt = reinterpret_cast<const float*>(base + L.xt);
-  p.frag = reinterpret_cast<uint4*>(base + L.frag);
-  p.scale = reinterpret_cast<float*>(base + L.scale);
-  p.M = M; p.T = dc.T; p.NT = dc.NT;
-  p.lanes = dc.NT == 1 ? 4 * M * dc.T : 32;
+  p.pmax = reinterpret_cast<const float*>(base + L.pmax);
+  p.bimg = base + L.bimg;
+  p.sexp = reinterpret_cast<int*>(base + L.sexp);
+  p.M = M; p.T = dc.T; p.NP = dc.NP; p.pp = dc.pp;
+  p.KB = (int)(g.k_eff_pad / 128);
+  p.ternary = g.bits == 2;
   p.kpad = g.k_eff_pad;
-  p.total = (g.k_eff_pad / 32) * dc.NT * p.lanes;
-  const int64_t blocks = (p.total + 255) / 256;
-  return launch_pdl(frag_kernel, dim3((unsigned)blocks), dim3(256), 0, st, p);
+  const int64_t items = (int64_t)p.KB * M * 8;
+  return launch_pdl(terms_kernel, dim3((unsigned)((items + 255) / 256)), dim3(256), 0, st, p);
 }
 
 }  // namespace sdq

@@ -9,16 +9,19 @@
 
 namespace sdq {
 
+constexpr int kTileRows = 128;    // rows per tile of the tiled code layout
+constexpr int kGroupCodes = 64;   // codes per k group of the tiled code layout
+
 // Geometry derived from a validated descriptor.
 struct Geometry {
   int32_t n_out, k_in, block, n_b, nblk;  // n_b = B * OSR, nblk = K / B
   int64_t k_eff;                          // nblk * n_b
   int32_t bits;                           // 2 ternary, 1 binary
   int32_t words_per_row;                  // plain layout
-  int32_t ng;                             // row groups of 16
-  int32_t kc;                             // codes per tile chunk (128 / 256)
-  int32_t n_chunks;                       // chunks per row group
-  int64_t k_eff_pad;                      // n_chunks * kc
+  int32_t ntiles;                         // tiles of kTileRows rows (tiled layout)
+  int32_t ngroups;                        // k groups of kGroupCodes codes per tile
+  int32_t wpg;                            // words per row per k group (4 ternary, 2 binary)
+  int64_t k_eff_pad;                      // K_eff rounded up to 128 codes
 };
 
 // Returns SDQ_OK and fills `g`, or SDQ_ERR_INVALID_ARG.
@@ -29,21 +32,20 @@ int validate(const sdq_layer_desc* d, Geometry* g);
 //   g:     n_b x B row-major, G[j][k]     = fp32(sum_k' Dt[j][k'] Had[k][k'])
 int build_tables(const sdq_layer_desc* d, const int8_t* signs, float* a_enc, float* g);
 
-// Decode-path terms per activation (bf16 hi + lo below 17 rows, hi only
-// above) and 8-column MMA tiles for batch M.
-inline int decode_terms(int M) { return M <= 16 ? 2 : 1; }
-inline int decode_ntiles(int M) { return (M * decode_terms(M) + 7) / 8; }
-
 constexpr int kMaxDecodeM = 64;
 
+// e4m3 terms per activation on the decode path: the MMA cost does not grow
+// with N up to 64 columns (M * T), so small batches take more terms.
+inline int decode_terms(int M) { return M <= 16 ? 4 : (M <= 21 ? 3 : 2); }
+
 // Launch shape of the decode kernel for one batch size (chosen at plan time).
+// Grid = S * P CTAs, one per SM: CTA (s, p) contracts k chunk s (CB blocks
+// of 128 codes) against row tiles p, p + P, p + 2P, ...
 struct DecodeConfig {
-  int M, T, NT;           // batch, fp8 terms per activation, 8-column MMA tiles
-  int S, R;               // k-slices and row ranges (grid = R x S)
-  int WK, WR;             // warps along k and along rows (WK * WR = 8)
-  int cps;                // chunks per k-slice
-  int rgc;                // row groups per row range
-  int P;                  // per-row partial maxima written by the prep kernel
+  int M, T, NP;           // batch, e4m3 terms per activation, MMA N (M*T rounded up to 16)
+  int S, P, CB;           // k chunks, CTAs per k chunk, 128-code blocks per chunk
+  int ring;               // code stages in the shared-memory ring
+  int pp;                 // per-row partial maxima written by the prep kernel
   size_t smem;            // dynamic shared memory of the decode kernel
 };
 

@@ -47,10 +47,10 @@ int validate(const sdq_layer_desc* d, Geometry* g) {
     g->k_eff = k_eff;
     g->bits = d->quantizer;
     g->words_per_row = (int32_t)(4 * ((k_eff * g->bits + 127) / 128));
-    g->ng = (d->n_out + 15) / 16;
-    g->kc = d->quantizer == SDQ_TERNARY ? 128 : 256;
-    g->n_chunks = (int32_t)((k_eff + g->kc - 1) / g->kc);
-    g->k_eff_pad = (int64_t)g->n_chunks * g->kc;
+    g->ntiles = (d->n_out + kTileRows - 1) / kTileRows;
+    g->k_eff_pad = (k_eff + 127) / 128 * 128;
+    g->ngroups = (int32_t)(g->k_eff_pad / kGroupCodes);
+    g->wpg = kGroupCodes * g->bits / 32;
   }
   return SDQ_OK;
 }
@@ -160,7 +160,7 @@ extern "C" size_t sdq_plain_bytes(const sdq_layer_desc* desc) {
 extern "C" size_t sdq_tiled_bytes(const sdq_layer_desc* desc) {
   sdq::Geometry g;
   if (sdq::validate(desc, &g) != SDQ_OK) return 0;
-  return (size_t)g.ng * g.n_chunks * 512;
+  return (size_t)g.ntiles * g.ngroups * sdq::kTileRows * g.wpg * 4;
 }
 
 extern "C" const char* sdq_status_string(int s) {

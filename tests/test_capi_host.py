@@ -35,9 +35,9 @@ def test_status_strings(sdq):
 
 
 @pytest.mark.parametrize("n,k,b,osr,q,keff,plain,tiled", [
-    (256, 512, 512, Fraction(2), 2, 1024, 256 * 64 * 4, 16 * 8 * 512),
-    (768, 768, 128, Fraction(5, 2), 1, 1920, 768 * 60 * 4, 48 * 8 * 512),
-    (17, 20, 4, Fraction(5, 2), 2, 50, 17 * 4 * 4, 2 * 1 * 512),
+    (256, 512, 512, Fraction(2), 2, 1024, 256 * 64 * 4, 2 * 16 * 128 * 16),
+    (768, 768, 128, Fraction(5, 2), 1, 1920, 768 * 60 * 4, 6 * 30 * 128 * 8),
+    (17, 20, 4, Fraction(5, 2), 2, 50, 17 * 4 * 4, 1 * 2 * 128 * 16),
 ])
 def test_geometry(sdq, n, k, b, osr, q, keff, plain, tiled):
     d = sdq.LayerDesc(n, k, b, osr, q)
@@ -45,6 +45,8 @@ def test_geometry(sdq, n, k, b, osr, q, keff, plain, tiled):
     assert sdq.sdq_plain_bytes(d) == plain
     assert sdq.sdq_tiled_bytes(d) == tiled
     assert O.plain_words_per_row(keff, q) * 4 * n == plain
+    nt, ng, wpg = O.tiled_geometry(n, keff, q)
+    assert nt * ng * 128 * wpg * 4 == tiled
 
 
 @pytest.mark.parametrize("bad", [

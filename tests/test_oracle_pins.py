@@ -358,21 +358,50 @@ def test_pack_plain_literal():
 
 def test_pack_tiled_hand_positions():
     """Single codes land where the layout's definition puts them."""
-    # ternary: row 9 (g=1, upper half), k = 53 = 32*1 + 16*1 + 4*1 + 1
-    # -> q=1, j = 2*1+1 = 3, t=1, b=1, f = 4*1 + (3-3) = 4, lane L = 4*1+1 = 5
-    c = np.zeros((16, 128), dtype=np.int8)
-    c[9, 53] = -1
+    # ternary, 130 x 200 codes: 2 tiles, K padded to 256 -> 4 groups of 64,
+    # 4 words per row per group.  Row 129 = (tile 1, r 1), k 83 = (group 1,
+    # word 1, field 3); word = 4 * (128 * (1 * 4 + 1) + 1) + 1 = 2565, and
+    # -1 is field value 3 at bit 6.
+    c = np.zeros((130, 200), dtype=np.int8)
+    c[129, 83] = -1
     w = O.pack_tiled(c, O.TERNARY)
+    assert w.size == 2 * 4 * 128 * 4
     nz = np.nonzero(w)[0]
-    assert list(nz) == [32 * 1 + 5] and int(w[nz[0]]) == 3 << 8
-    # binary: row 2 (g=2, lower half), k = 200 = 64*3 + 0 + 0 + 4*2 + 0
-    # -> q=3, u=0, h=0, t=2, b=0, j=0, f = 7, lane L = 10; code +1 -> bit set
-    cb = -np.ones((16, 256), dtype=np.int8)
-    cb[2, 200] = 1
+    assert list(nz) == [2565] and int(w[2565]) == 3 << 6
+    # binary, 5 x 100 codes: 1 tile, K padded to 128 -> 2 groups, 2 words per
+    # row per group.  Row 3, k 70 = (group 1, word 0, bit 6); word =
+    # 2 * (128 * 1 + 3) = 262.  +1 sets the bit, -1 leaves it clear.
+    cb = -np.ones((5, 100), dtype=np.int8)
+    cb[3, 70] = 1
     wb = O.pack_tiled(cb, O.BINARY)
+    assert wb.size == 1 * 2 * 128 * 2
     nz = np.nonzero(wb)[0]
-    assert list(nz) == [32 * 3 + 10] and int(wb[nz[0]]) == 1 << 7
+    assert list(nz) == [262] and int(wb[262]) == 1 << 6
     rng = np.random.default_rng(16)
     cc = np.where(rng.random((20, 300)) < 0.5, 1, -1).astype(np.int8)
     cc[rng.random((20, 300)) < 0.3] = 0
     assert np.array_equal(O.unpack_tiled(O.pack_tiled(cc, O.TERNARY), O.TERNARY, 20, 300), cc)
+    cb = np.where(rng.random((7, 333)) < 0.5, 1, -1).astype(np.int8)
+    assert np.array_equal(O.unpack_tiled(O.pack_tiled(cb, O.BINARY), O.BINARY, 7, 333), cb)
+
+
+@pytest.mark.parametrize("q,n,k", [(O.TERNARY, 200, 300), (O.BINARY, 131, 520)])
+def test_tiled_is_a_regrouping_of_plain_chunks(q, n, k):
+    """Both layouts keep a row's codes in natural order inside 64-code groups,
+    so every (tile, group, row) run of the tiled words equals the plain words
+    of that row and group (zero past the last row)."""
+    rng = np.random.default_rng(17 + q)
+    c = np.where(rng.random((n, k)) < 0.5, 1, -1).astype(np.int8)
+    if q == O.TERNARY:
+        c[rng.random((n, k)) < 0.4] = 0
+    plain = O.pack_plain(c, q)
+    tiled = O.pack_tiled(c, q)
+    nt, ng, wpr = O.tiled_geometry(n, k, q)
+    slabs = tiled.reshape(nt, ng, 128, wpr)
+    for T in range(nt):
+        for G in range(ng):
+            for r in range(128):
+                row = 128 * T + r
+                want = plain[row, wpr * G: wpr * G + wpr] if row < n and wpr * G < plain.shape[1] \
+                    else np.zeros(wpr, np.uint32)
+                assert np.array_equal(slabs[T, G, r], want), (T, G, r)

@@ -146,7 +146,7 @@ def test_pack_unpack_bit_exact(sdq, torch_cuda, q, n, keff):
     assert int(bad.item()) == 0
     if q == O.TERNARY:
         tw = _np_u32(tiled).copy()
-        # one invalid field "10" at field 3 of word 0: row 0, k = 0 (never padding)
+        # one invalid field "10" at field 3 of word 0: row 0, k = 3 (never padding)
         tw[0] = (tw[0] & ~np.uint32(0xC0)) | np.uint32(0x80)
         bad.zero_()
         sdq.sdq_unpack(plan.handle, _u32(torch, tw), back, bad)
@@ -156,7 +156,8 @@ def test_pack_unpack_bit_exact(sdq, torch_cuda, q, n, keff):
 
 def test_pack_full_size_sampled_tiles(sdq, torch_cuda):
     """cfg4 gate (28672 x 16384 codes): round trip, and a seeded sample of
-    row groups compared tile-for-tile with the oracle's tiled layout."""
+    (tile, k group) slabs compared with the oracle's tiled layout of the same
+    128 rows."""
     torch = torch_cuda
     n, keff = 28672, 16384
     d = _desc(sdq, n, 8192, 128, 2, O.TERNARY)
@@ -173,12 +174,14 @@ def test_pack_full_size_sampled_tiles(sdq, torch_cuda):
     sdq.sdq_unpack(plan.handle, tiled, back)
     assert torch.equal(back, plain)
     pw = plain.cpu().numpy().view(np.uint32).reshape(n, -1)
-    tw = _np_u32(tiled)
-    per_group = (keff // 128) * 128
-    for rg in np.random.default_rng(1).choice(n // 16, 3, replace=False):
-        c = O.unpack_plain(pw[16 * rg:16 * rg + 16], O.TERNARY, keff)
-        want = O.pack_tiled(c[:, :1024], O.TERNARY)           # first 8 chunks
-        assert np.array_equal(tw[rg * per_group: rg * per_group + want.size], want)
+    nt, ng, wpg = O.tiled_geometry(n, keff, O.TERNARY)
+    slabs = _np_u32(tiled).reshape(nt, ng, 128 * wpg)
+    rng = np.random.default_rng(1)
+    for T in rng.choice(nt, 3, replace=False):
+        c = O.unpack_plain(pw[128 * T:128 * T + 128], O.TERNARY, keff)
+        for G in rng.choice(ng, 2, replace=False):
+            want = O.pack_tiled(c[:, 64 * G:64 * G + 64], O.TERNARY)[:128 * wpg]
+            assert np.array_equal(slabs[T, G], want), (T, G)
 
 
 # ---------------------------------------------------------------- forward
