@@ -1,4 +1,6 @@
 // C ABI of libsdq (declarations and contracts in include/sdq.h).
+#include <algorithm>
+#include <cmath>
 #include <cstdlib>
 #include <cstring>
 #include <new>
@@ -40,8 +42,7 @@ WsLayout workspace_layout(const sdq_plan_s* pl, int M) {
   if (M <= kMaxDecodeM) {
     const DecodeConfig& dc = pl->dcfg[M];
     off = align_up(off + sizeof(float) * (size_t)M * g.k_eff_pad, 256);
-    L.pmax = off;
-    off = align_up(off + sizeof(float) * (size_t)M * dc.pp, 256);
+    L.pmax = off;                                  // (unused on the decode path)
     L.bimg = off;                                  // e4m3 B operand image, K/128 x NP x 128 bytes
     off = align_up(off + (size_t)(g.k_eff_pad / 128) * dc.NP * 128, 256);
     L.sexp = off;                                  // per-batch-row scale exponents
@@ -84,6 +85,13 @@ extern "C" int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_sig
   if (st != SDQ_OK) return st;
   for (int j = 0; j < g.n_b; ++j)
     for (int k = 0; k < g.block; ++k) at[(size_t)k * g.n_b + j] = a_enc[(size_t)j * g.block + k];
+  // max_j sum_k |G[j][k]|, with a margin for the bf16 hi + lo split of G
+  double gnorm = 0.0;
+  for (int j = 0; j < g.n_b; ++j) {
+    double sr = 0.0;
+    for (int k = 0; k < g.block; ++k) sr += std::fabs((double)gm[(size_t)j * g.block + k]);
+    gnorm = std::max(gnorm, sr);
+  }
   std::vector<uint16_t> ghi(tab), glo(tab);
   for (size_t i = 0; i < tab; ++i) {
     ghi[i] = host_bf16(gm[i]);
@@ -96,6 +104,7 @@ extern "C" int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_sig
   p->geo = g;
   p->device = dev;
   p->sm_count = sms;
+  p->gnorm = (float)(gnorm * (1.0 + 1.0 / 1024));
   if (cudaMalloc(&p->d_at, sizeof(float) * tab) != cudaSuccess ||
       cudaMalloc(&p->d_g_hi, sizeof(uint16_t) * tab) != cudaSuccess ||
       cudaMalloc(&p->d_g_lo, sizeof(uint16_t) * tab) != cudaSuccess) {
@@ -158,9 +167,7 @@ extern "C" int sdq_prep_activations(sdq_plan p, const uint16_t* x, int32_t M, vo
   int st = check_ws(p, M, ws, ws_bytes);
   if (st != SDQ_OK) return st;
   if (!x || !aligned16(x)) return SDQ_ERR_INVALID_ARG;
-  cudaError_t e = launch_prep(p, x, M, ws, (cudaStream_t)stream);
-  if (e == cudaSuccess && M <= kMaxDecodeM) e = launch_terms(p, M, ws, (cudaStream_t)stream);
-  return cuda_status(e);
+  return cuda_status(launch_prep(p, x, M, ws, (cudaStream_t)stream));
 }
 
 static int contract(sdq_plan p, const uint32_t* codes_tiled, const float* alpha, int32_t M, float* y,

@@ -30,7 +30,6 @@ cudaError_t launch_prep(const sdq_plan_s* p, const uint16_t* x, int M, void* ws,
 // preceding grid (valid only behind this library's own prep kernels).
 cudaError_t launch_decode(const sdq_plan_s* p, const uint32_t* codes, const float* alpha, int M,
                           float* y, void* ws, cudaStream_t st, int early);
-cudaError_t launch_terms(const sdq_plan_s* p, int M, void* ws, cudaStream_t st);
 cudaError_t launch_prefill(const sdq_plan_s* p, const uint32_t* codes, const float* alpha, int M,
                            float* y, void* ws, cudaStream_t st);
 int prep_partials(const sdq_plan_s* p, int M);  // per-row max partials of the prep grid
@@ -104,24 +103,24 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
   asm volatile("mov.u64 %0, %globaltimer;\n" : "=l"(t));
   return t;
 }
-// Bounded wait for phase `parity` of `bar`: gives up after ~2 s of wall time
-// and returns false (callers record an error and skip the dependent work).
+// Bounded wait for phase `parity` of `bar`: gives up after ~4e9 SM cycles
+// (about 2 s) and returns false (callers record an error and skip the
+// dependent work).  The clock is read only once the first test has failed.
+__device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok) : "r"(a), "r"(parity) : "memory");
+  return ok != 0;
+}
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
   const uint32_t a = smem_u32(bar);
-  uint64_t t0 = 0;
-  for (uint32_t i = 0;; ++i) {
-    uint32_t ok;
-    asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-        " selp.u32 %0, 1, 0, p;\n}\n"
-        : "=r"(ok) : "r"(a), "r"(parity) : "memory");
-    if (ok) return true;
-    if ((i & 1023u) == 0u) {
-      const uint64_t now = globaltimer_ns();
-      if (i == 0) t0 = now;
-      else if (now - t0 > 2000000000ull) return false;
-    }
-  }
+  if (mbar_try(a, parity)) return true;
+  const long long t0 = clock64();
+  while (!mbar_try(a, parity))
+    if (clock64() - t0 > 4000000000ll) return false;
+  return true;
 }
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");

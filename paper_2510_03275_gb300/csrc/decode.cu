@@ -24,11 +24,13 @@
 // of an MMA-issuing thread costs about as much as several MMAs, and one
 // thread issues at most one MMA every ~45 cycles, so the CTA runs two
 // independent pipelines e = 0, 1 on alternate stages (i = e mod 2), each with
-// its own producer thread, expander warps, MMA issuer, two TMEM slots and
-// accumulator; the epilogue adds the two accumulators.  Every mbarrier thus
-// has one producer and one consumer that both walk its phases in order.
+// its own producer thread, two expander sets, MMA issuer, two TMEM slots
+// and accumulator; the epilogue adds the two accumulators.  Set t of
+// pipeline e owns TMEM slot 2e + t and expands the pipeline's stages
+// j = t (mod 2): every mbarrier has one producer and one consumer that both
+// walk its phases in order.
 //
-// CTA (k chunk s, row set p) of one SM, 16 warps:
+// CTA (k chunk s, row set p) of one SM, 24 warps:
 //   warps 0, 1    lane 0 of warp e streams pipeline e's stages (one 128-row
 //                 tile x up to sb * 128 codes = contiguous slabs of the tiled
 //                 layout) into its shared-memory ring slots with bulk copies;
@@ -37,9 +39,10 @@
 //   warps 2, 3    lane 0 of warp 2 + e issues pipeline e's MMAs, commits to
 //                 the stage's TMEM slot and, after its last stage of a row
 //                 tile, to its accumulator
-//   warps 4..11   expanders: warps 4 + 4e .. 7 + 4e (one per TMEM lane
-//                 quadrant) expand pipeline e's stages into its TMEM slots
-//   warps 12..15  epilogue: read and add the accumulators, combine the
+//   warps 4..19   expanders: set x = 2e + t (warps 4 + 4x .. 7 + 4x, one per
+//                 TMEM lane quadrant) expands stages i = e + 2t (mod 4) into
+//                 TMEM slot x
+//   warps 20..23  epilogue: read and add the accumulators, combine the
 //                 terms, scale and store y, or store a split-K partial; after
 //                 the CTA's last tile, one fence and one ticket per tile, and
 //                 the last CTA of each tile sums its S partials in a fixed
@@ -60,10 +63,14 @@ namespace {
 constexpr int kBlk = 128;                        // codes per block (4 MMAs of K = 32)
 constexpr int kProducers = 2;                    // warps 0, 1
 constexpr int kIssuerWarp0 = 2;                  // warps 2, 3
-constexpr int kExpWarp0 = 4;                     // warps 4..11
-constexpr int kEpiWarp0 = kExpWarp0 + 8;         // warps 12..15
-constexpr int kThreads = 32 * (kEpiWarp0 + 4);   // 512
-constexpr int kMaxRing = 16;
+constexpr int kSlots = 2;                        // TMEM A slots (and expander sets) per pipeline
+constexpr int kMaxSb = 3;                        // at most 3 blocks per stage
+constexpr int kExpWarp0 = 4;                     // warps 4..19
+constexpr int kExpSets = 2 * kSlots;
+constexpr int kEpiWarp0 = kExpWarp0 + 4 * kExpSets;   // warps 20..23
+constexpr int kThreads = 32 * (kEpiWarp0 + 4);   // 768
+constexpr int kMaxRing = 24;
+constexpr int kMaxSpu = 128;                     // stages per row tile (config search bound)
 constexpr int kSmemMax = 224 * 1024;
 constexpr int kSmemMin = 120 * 1024;             // > half an SM: one CTA per SM
 
@@ -103,10 +110,12 @@ __device__ __forceinline__ int stage_block(int j, int ncb, int spu) { return j *
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t c_full[kMaxRing], c_empty[kMaxRing];
-  __shared__ __align__(8) uint64_t a_full[4], a_empty[4];
+  __shared__ __align__(8) uint64_t a_full[2 * kSlots], a_empty[2 * kSlots];
   __shared__ __align__(8) uint64_t acc_full[2][2], acc_empty[2][2], b_full, mma_done[2];
   __shared__ uint32_t tmem_base;
   __shared__ int last[128];
+  __shared__ float scale_s[kMaxDecodeM];   // 2^e_m
+  __shared__ int sblk[kMaxSpu + 1];         // first block of stage j of a tile
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int sidx = blockIdx.x % p.S, prow = blockIdx.x / p.S;
@@ -123,10 +132,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   if (tid == 0) {
     for (int i = 0; i < p.ring; ++i) {
       mbar_init(&c_full[i], 1);
-      mbar_init(&c_empty[i], 128);
+      mbar_init(&c_empty[i], 4);     // one arrival per expander warp
     }
-    for (int i = 0; i < 4; ++i) {
-      mbar_init(&a_full[i], 128);
+    for (int i = 0; i < 2 * kSlots; ++i) {
+      mbar_init(&a_full[i], 4);
       mbar_init(&a_empty[i], 1);
     }
     for (int e = 0; e < 2; ++e)
@@ -134,6 +143,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         mbar_init(&acc_full[e][b], 1);
         mbar_init(&acc_empty[e][b], 128);
       }
+    for (int j = 0; j <= spu; ++j) sblk[j] = stage_block(j, ncb, spu);
     mbar_init(&b_full, 1);
     mbar_init(&mma_done[0], 1);
     mbar_init(&mma_done[1], 1);
@@ -158,11 +168,13 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       // i mod ring (ring is even).  Stage (unit u, j) is the
       // slabs (tile, 2 b) .. (tile, 2 b' - 1) of its blocks [b, b'),
       // adjacent in the tiled layout.  Producer 0 also copies the chunk's B
-      // operand: after the first ring of stages when the codes may be read
-      // before the preceding grid is done, before everything otherwise.
+      // operand: after its first two stages when the codes may be read before
+      // the preceding grid is done, before everything otherwise.
       int last_i = -1;
       bool b_loaded = warp != 0;
-      const int pre = p.early ? min(p.ring, nstages) : 0;
+      const int pre = p.early ? min(2 * kProducers, nstages) : 0;
+      int u = 0, j = warp;
+      while (j >= spu) { j -= spu; ++u; }
       for (int i = warp; i < nstages && ok; i += kProducers) {
         if (!b_loaded && i >= pre) {
           if (p.early) pdl_wait();
@@ -173,8 +185,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         const int slot = i % p.ring, r = i / p.ring;
         if (r > 0) ok = mbar_wait(&c_empty[slot], (r - 1) & 1);
         if (!ok) break;
-        const int u = i / spu, j = i - u * spu;
-        const int b0 = stage_block(j, ncb, spu), b1 = stage_block(j + 1, ncb, spu);
+        const int b0 = sblk[j], b1 = sblk[j + 1];
         const int tile = prow + u * p.P;
         const uint8_t* src = reinterpret_cast<const uint8_t*>(p.codes) +
                              ((size_t)tile * p.KB + kb0 + b0) * p.blk_bytes;
@@ -182,6 +193,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         mbar_expect_tx(&c_full[slot], bytes);
         bulk_g2s(ring + (size_t)slot * p.slot_bytes, src, bytes, &c_full[slot]);
         last_i = i;
+        j += kProducers;
+        while (j >= spu) { j -= spu; ++u; }
       }
       if (!b_loaded) {   // producer 0 had no stage at or past `pre`, or failed
         if (p.early) pdl_wait();
@@ -198,40 +211,52 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
     }
   } else if (warp < kExpWarp0) {
     if (lane == 0) {
-      // MMA issuer of pipeline e: stages i = e (mod 2), the pipeline's j-th
-      // stage (j = i / 2) in TMEM slot e + 2 (j mod 2), into its own
+      // MMA issuer of pipeline e: stages i = e (mod 2), the pipeline's jj-th
+      // stage (jj = i / 2) in TMEM slot 2e + (jj mod 2), into its own
       // accumulator.
       const int e = warp - kIssuerWarp0;
       ok = mbar_wait(&b_full, 0);
       tc_fence_after();
       // kind::f8f6f4: D fp32, A and B e4m3, both K-major, N = NP, M = 128.
       const uint32_t idesc = (1u << 4) | ((uint32_t)(p.NP >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
-      int k = 0, prev_u = -1, buf = 0;
-      for (int i = e; i < nstages && ok; i += 2) {
-        const int u = i / spu, j = i - u * spu, jj = i >> 1, a = e + 2 * (jj & 1);
-        const bool first = u != prev_u;
+      // Per stage: one wait, 4 nb MMAs, one commit; stage bookkeeping is
+      // kept incremental (a single thread's scalar latency is on the path).
+      const uint64_t bd0 = sw128_desc(sbase);
+      const uint64_t bstep = (uint64_t)((p.NP * 128) >> 4);   // descriptor units per block
+      const uint32_t abase = tmem + (uint32_t)(kSlots * e * 32 * p.sb);
+      const uint32_t aslot = (uint32_t)(32 * p.sb);
+      int k = 0, buf = 0, u = 0, j = e;
+      while (j >= spu) { j -= spu; ++u; }
+      bool first = true;
+      uint32_t dt = 0;
+      for (int i = e, jj = 0; i < nstages && ok; i += 2, ++jj) {
         if (first) {
-          prev_u = u;
-          buf = k % p.nbuf;
+          buf = p.nbuf == 2 ? (k & 1) : 0;
           if (k >= p.nbuf) {
             ok = mbar_wait(&acc_empty[e][buf], ((k / p.nbuf) - 1) & 1);
             if (!ok) break;
           }
+          dt = tmem + (uint32_t)(p.dbase + (e * p.nbuf + buf) * p.NP);
         }
+        const int a = kSlots * e + (jj & 1);
         ok = mbar_wait(&a_full[a], (jj >> 1) & 1);
         if (!ok) break;
         tc_fence_after();
-        const int b0 = stage_block(j, ncb, spu), nb = stage_block(j + 1, ncb, spu) - b0;
-        const uint32_t dt = tmem + (uint32_t)(p.dbase + (e * p.nbuf + buf) * p.NP);
-        const uint32_t at = tmem + (uint32_t)(a * 32 * p.sb);
-        for (int bb = 0; bb < nb; ++bb) {
-          const uint64_t bd = sw128_desc(sbase + (uint32_t)(b0 + bb) * p.NP * 128);
-#pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            umma_f8_ts(dt, at + 32 * bb + 8 * kk, bd + 2 * kk, idesc, (first && bb == 0 && kk == 0) ? 0u : 1u);
+        const int b0 = sblk[j], nb = sblk[j + 1] - b0;
+        uint64_t bd = bd0 + (uint64_t)b0 * bstep;
+        uint32_t at = abase + (uint32_t)(jj & 1) * aslot;
+        for (int bb = 0; bb < nb; ++bb, at += 32, bd += bstep) {
+          umma_f8_ts(dt, at, bd, idesc, (first && bb == 0) ? 0u : 1u);
+          umma_f8_ts(dt, at + 8, bd + 2, idesc, 1u);
+          umma_f8_ts(dt, at + 16, bd + 4, idesc, 1u);
+          umma_f8_ts(dt, at + 24, bd + 6, idesc, 1u);
         }
         umma_commit(&a_empty[a]);
-        if (i + 2 >= (u + 1) * spu) {   // this pipeline's last stage of the tile
+        const int u0 = u;
+        j += 2;
+        while (j >= spu) { j -= spu; ++u; }
+        first = u != u0;
+        if (first) {   // this pipeline's last stage of the tile
           umma_commit(&acc_full[e][buf]);
           ++k;
         }
@@ -241,59 +266,83 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       // ... and the last commit to each of this pipeline's TMEM slots has
       // arrived (those phases have no other waiter).
       const int njs = (nstages - e + 1) / 2;   // stages of this pipeline
-      for (int jj = max(0, njs - 2); jj < njs; ++jj)
-        if (!mbar_wait(&a_empty[e + 2 * (jj & 1)], (jj >> 1) & 1)) ok = false;
+      for (int jj = max(0, njs - kSlots); jj < njs; ++jj)
+        if (!mbar_wait(&a_empty[kSlots * e + jj % kSlots], (jj / kSlots) & 1)) ok = false;
     }
   } else if (warp < kEpiWarp0) {
     // ------------------------------------------------------------ expanders
-    // Warps 4 + 4e .. 7 + 4e expand pipeline e's stages, in order.
-    const int e = (warp - kExpWarp0) >> 2, q = warp & 3, r = 32 * q + lane;
+    // Set x = 2e + t expands stages i = e + 2t (mod 4) in order: TMEM slot
+    // x, ring slots i mod ring (ring is a multiple of 4).
+    const int x = (warp - kExpWarp0) >> 2, q = warp & 3, r = 32 * q + lane;
+    const int ex = x / kSlots, tx = x - ex * kSlots;
     const uint32_t lane_addr = tmem + ((uint32_t)(32 * q) << 16);
     const uint32_t slab = p.blk_bytes / 2;
-    for (int i = e; i < nstages && ok; i += 2) {
-      const int slot = i % p.ring, jj = i >> 1, a = e + 2 * (jj & 1);
+    int u = 0, j = ex + 2 * tx;
+    while (j >= spu) { j -= spu; ++u; }
+    for (int i = ex + 2 * tx; i < nstages && ok; i += 2 * kSlots) {
+      const int slot = i % p.ring, jj = i >> 1, a = x;
       ok = warp_wait(&c_full[slot], (i / p.ring) & 1);
       if (!ok) break;
-      if (jj >= 2) {
-        ok = warp_wait(&a_empty[a], ((jj >> 1) - 1) & 1);
+      // Codes into registers first, so that the ring slot goes back to the
+      // producer before this set waits for its TMEM slot.
+      const int nb = sblk[j + 1] - sblk[j];
+      j += 2 * kSlots;
+      while (j >= spu) { j -= spu; ++u; }
+      const uint8_t* cs = ring + (size_t)slot * p.slot_bytes;
+      uint32_t w[kMaxSb][8];
+#pragma unroll
+      for (int bb = 0; bb < kMaxSb; ++bb) {
+        if (bb < nb) {
+          const uint8_t* cb = cs + bb * p.blk_bytes;
+          if (p.ternary) {
+            const uint4 g0 = *reinterpret_cast<const uint4*>(cb + r * 16);
+            const uint4 g1 = *reinterpret_cast<const uint4*>(cb + slab + r * 16);
+            w[bb][0] = g0.x; w[bb][1] = g0.y; w[bb][2] = g0.z; w[bb][3] = g0.w;
+            w[bb][4] = g1.x; w[bb][5] = g1.y; w[bb][6] = g1.z; w[bb][7] = g1.w;
+          } else {
+            const uint2 g0 = *reinterpret_cast<const uint2*>(cb + r * 8);
+            const uint2 g1 = *reinterpret_cast<const uint2*>(cb + slab + r * 8);
+            w[bb][0] = ~g0.x; w[bb][1] = ~g0.y; w[bb][2] = ~g1.x; w[bb][3] = ~g1.y;
+          }
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&c_empty[slot]);
+      if (jj >= kSlots) {
+        ok = warp_wait(&a_empty[a], ((jj / kSlots) - 1) & 1);
         if (!ok) break;
         tc_fence_after();
       }
-      const int u = i / spu, j = i - u * spu;
-      const int nb = stage_block(j + 1, ncb, spu) - stage_block(j, ncb, spu);
-      const uint8_t* cs = ring + (size_t)slot * p.slot_bytes;
-      for (int bb = 0; bb < nb; ++bb) {
-        uint32_t v[32];
-        const uint8_t* cb = cs + bb * p.blk_bytes;
-        if (p.ternary) {
-          const uint4 g0 = *reinterpret_cast<const uint4*>(cb + r * 16);
-          const uint4 g1 = *reinterpret_cast<const uint4*>(cb + slab + r * 16);
-          const uint32_t w[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
 #pragma unroll
-          for (int wi = 0; wi < 8; ++wi)
+      for (int bb = 0; bb < kMaxSb; ++bb) {
+        if (bb < nb) {
+          uint32_t v[32];
+          if (p.ternary) {
 #pragma unroll
-            for (int jb = 0; jb < 4; ++jb) v[4 * wi + jb] = (w[wi] << (2 * jb)) & 0xC0C0C0C0u;
-        } else {
-          const uint2 g0 = *reinterpret_cast<const uint2*>(cb + r * 8);
-          const uint2 g1 = *reinterpret_cast<const uint2*>(cb + slab + r * 8);
-          const uint32_t w[4] = {~g0.x, ~g0.y, ~g1.x, ~g1.y};
+            for (int wi = 0; wi < 8; ++wi)
 #pragma unroll
-          for (int wi = 0; wi < 4; ++wi)
+              for (int jb = 0; jb < 4; ++jb) v[4 * wi + jb] = (w[bb][wi] << (2 * jb)) & 0xC0C0C0C0u;
+          } else {
 #pragma unroll
-            for (int jb = 0; jb < 8; ++jb) v[8 * wi + jb] = ((w[wi] << jb) & 0x80808080u) | 0x40404040u;
+            for (int wi = 0; wi < 4; ++wi)
+#pragma unroll
+              for (int jb = 0; jb < 8; ++jb) v[8 * wi + jb] = ((w[bb][wi] << jb) & 0x80808080u) | 0x40404040u;
+          }
+          tmem_st32(lane_addr + (uint32_t)(a * 32 * p.sb + 32 * bb), v);
         }
-        tmem_st32(lane_addr + (uint32_t)(a * 32 * p.sb + 32 * bb), v);
       }
-      mbar_arrive(&c_empty[slot]);
       tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(&a_full[a]);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&a_full[a]);
     }
   } else {
     // ------------------------------------------------------------- epilogue
     const int q = warp & 3, r = 32 * q + lane, et = tid - 32 * kEpiWarp0;
     const int NR = p.ntiles * kTileRows;
     const int MT = p.M * p.T;
+    if (et < p.M) scale_s[et] = ldexpf(1.f, p.sexp[et]);
+    named_bar_sync(2, 128);
     int kc[2] = {0, 0};
     for (int u = 0; u < nunits && ok; ++u) {
       // issuers with stages in this tile: both, unless the tile is one stage
@@ -331,7 +380,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
             acc += wt * dv;
             wt *= 0.0625f;
             if (++t == p.T) {
-              const float ym = ldexpf(acc, p.sexp[m]);
+              const float ym = acc * scale_s[m];
               if (p.S == 1) {
                 if (live) p.y[(size_t)m * p.n_out + row] = sa * ym;
               } else {
@@ -394,7 +443,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
 void tmem_split(int NP, int* sb, int* nbuf, int* dbase) {
   *nbuf = NP <= 32 ? 2 : 1;
   const int dcols = 2 * *nbuf * NP;
-  *sb = std::min(4, (512 - dcols) / (4 * 32));
+  *sb = std::max(1, std::min(kMaxSb, (512 - dcols) / (2 * kSlots * 32)));
   *dbase = 512 - dcols;
 }
 
@@ -418,7 +467,7 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
   int sb = 0, nbuf = 0, dbase = 0;
   tmem_split(best.NP, &sb, &nbuf, &dbase);
   const int slot_bytes = sb * blk_bytes;
-  const double clk = 1.9e9, bw = 6.5e12, latency = 1.5e-6;
+  const double clk = 1.9e9, bw = 6.5e12, latency = 2.2e-6;   // loaded HBM latency
   const double t_mma = std::max(38.0, best.NP * 0.4) / clk;     // per MMA, two issuers
   const double code_bytes = (double)g.ntiles * kTileRows * g.k_eff_pad * g.bits / 8;
   double best_t = 1e30;
@@ -427,9 +476,10 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
     if ((S - 1) * CB >= KB) continue;                      // no empty chunk
     const int b_bytes = CB * best.NP * 128;
     int ring = std::min(kMaxRing, (kSmemMax - 2048 - b_bytes) / slot_bytes);
-    ring -= ring % kProducers;
-    if (ring < 4) continue;
+    ring -= ring % kExpSets;          // each ring slot belongs to one expander set
+    if (ring < kExpSets) continue;
     const int spu = std::max((CB + sb - 1) / sb, std::min(2, CB));
+    if (spu > kMaxSpu) continue;
     for (int P = 1; P <= std::min(g.ntiles, sms / S); ++P) {
       const int grid = S * P;
       const int units = (g.ntiles + P - 1) / P;

@@ -8,10 +8,11 @@
 // x is bf16 (exact), G is split into bf16 hi + lo parts (relative error of
 // the pair ~2^-16), accumulation in fp32.
 //
-// Decode path (M <= 64): fp32 x_tilde (M x K_eff_pad) plus max |x_tilde|
-// per CTA and batch row; then the terms kernel below writes the decode
-// kernel's e4m3 B operand.  Prefill path: bf16 x_tilde in the permuted
-// 64-code stage order of the prefill kernel's operand tiles.
+// Decode path (M <= 64): the decode prepare kernel below (x_tilde and the
+// decode kernel's e4m3 B operand in one pass).  Prefill path: bf16 x_tilde
+// in the permuted 64-code stage order of the prefill kernel's operand tiles.
+#include <algorithm>
+
 #include "common.cuh"
 
 namespace sdq {
@@ -154,75 +155,186 @@ __global__ void __launch_bounds__(128) prep_kernel(PrepParams p) {
   }
 }
 
-// ------------------------------------------------------------ e4m3 terms
-// B operand of the decode MMAs for the whole K range: block kb (128 codes)
-// is NP rows x 128 bytes in the 128-byte-swizzled K-major layout, row
-// n = m T + t holding term t of batch row m at MMA K index kap (natural code
-// decode_stage_k(kap)).  With e_m chosen so that max |x_tilde[m]| 2^-e_m <
-// 448, v = x_tilde 2^-e_m splits into sum_t 16^-t q_t: q_t = e4m3(v_t),
-// v_{t+1} = 16 (v_t - q_t) (exact: e4m3 rounding is relative, the residual
-// has few bits).  Rows past M T are not written: they only feed
-// accumulator columns that are never read.  One thread per (kb, m, 16-byte
-// chunk); e_m also goes to sexp for the decode epilogue.
-struct TermsParams {
-  const float* xt;
-  const float* pmax;
-  uint8_t* bimg;
-  int* sexp;
-  int M, T, NP, pp, KB, ternary;
-  int64_t kpad;
+// ------------------------------------------------- decode prepare (M <= 64)
+// One kernel per call: x_tilde = G x_b as above (fp32, kept for checking),
+// and directly the decode kernel's e4m3 B operand.  That operand covers all
+// of K: block kb (128 codes) is NP rows x 128 bytes in the 128-byte-swizzled
+// K-major layout, row n = m T + t holding term t of batch row m at the MMA K
+// position of each code (decode_pos).  With x_tilde[m] 2^-e_m < 448,
+// v = x_tilde 2^-e_m splits into sum_t 16^-t q_t: q_t = e4m3(v_t),
+// v_{t+1} = 16 (v_t - q_t) (exact: e4m3 rounding is relative).  e_m comes
+// from a bound rather than from the maximum of x_tilde, so that no CTA waits
+// for another: |x_tilde[m, j]| <= sum_k |G[j, k]| |x[m, k]| <= gnorm max|x[m]|,
+// gnorm = max_j sum_k |G[j, k]| (with a margin for the bf16 split of G).
+// e4m3 is floating point, so the looser scale costs no relative precision.
+// Rows past M T are not written: they only feed accumulator columns that
+// are never read.  The CTA's x tile and G rows arrive in one round of loads
+// (k chunks of up to 256), overlapped with its reading of the x row for
+// max |x[m]|.
+struct DecPrepParams {
+  const uint16_t* x;
+  const uint16_t* g_hi;
+  const uint16_t* g_lo;
+  float* xt;          // M x kpad fp32
+  uint8_t* bimg;      // e4m3 B operand image
+  int* sexp;          // e_m per batch row
+  uint32_t* cnt;      // decode tickets and error word to zero
+  int ncnt;
+  float gnorm;
+  int M, K, B, n_b, nblk, T, NP, kc, ternary, vec;
+  int64_t k_eff, kpad;
 };
 
-__global__ void __launch_bounds__(256) terms_kernel(TermsParams p) {
-  __shared__ int se[kMaxDecodeM];
+// MMA K position (within a 128-code block) of natural code kl: the inverse of
+// decode_stage_k.
+__device__ __forceinline__ int decode_pos(int kl, bool ternary) {
+  if (ternary) {
+    const int f = kl & 15;
+    return (kl & ~15) + 4 * (3 - (f & 3)) + (f >> 2);
+  }
+  const int f = kl & 31;
+  return (kl & ~31) + 4 * (7 - (f & 7)) + (f >> 3);
+}
+
+__device__ __forceinline__ float bf16_abs(uint32_t h) { return __uint_as_float((h & 0x7FFFu) << 16); }
+
+__global__ void __launch_bounds__(128) prep_decode_kernel(DecPrepParams p) {
+  constexpr int TB = 16, NTW = 2;   // 16 blocks x 64 j per CTA; warp w owns j 16w .. 16w + 15
+  extern __shared__ __align__(16) uint8_t dsm[];
+  const int ld = p.kc + 8;
+  uint16_t* xs = reinterpret_cast<uint16_t*>(dsm);   // TB x ld
+  uint16_t* ghs = xs + TB * ld;                        // 64 x ld
+  uint16_t* gls = ghs + 64 * ld;                       // 64 x ld
+  __shared__ float red[4];
+  __shared__ int e_s;
   pdl_wait();
   pdl_launch_dependents();
-  const int tid = threadIdx.x;
-  if (tid < p.M) {
-    float mx = 0.f;
-    for (int i = 0; i < p.pp; ++i) mx = fmaxf(mx, p.pmax[(size_t)tid * p.pp + i]);
+  const int jt = blockIdx.x, bt = blockIdx.y, m = blockIdx.z;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t = lane & 3;
+  const int b0 = bt * TB, j0 = jt * 64, wcol = warp * 16;
+  const uint16_t* xr = p.x + (size_t)m * p.K;
+
+  // max |x[m, :]| (loads issued before the tile loads)
+  float xmax = 0.f;
+  if (p.vec) {
+    for (int i = tid; i < p.K / 8; i += 128) {
+      const uint4 v = *reinterpret_cast<const uint4*>(xr + 8 * i);
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) xmax = fmaxf(xmax, fmaxf(bf16_abs(w[q]), bf16_abs(w[q] >> 16)));
+    }
+  } else {
+    for (int i = tid; i < p.K; i += 128) xmax = fmaxf(xmax, bf16_abs(xr[i]));
+  }
+
+  float acc[NTW][4];
+#pragma unroll
+  for (int n = 0; n < NTW; ++n)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) acc[n][e] = 0.f;
+  for (int kc0 = 0; kc0 < p.B; kc0 += p.kc) {
+    if (p.vec) {   // B % 32 == 0, rows 16-byte aligned
+      const int q8 = p.kc / 8;
+      for (int i = tid; i < TB * q8; i += 128) {
+        const int rr = i / q8, q = i - rr * q8, b = b0 + rr;
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (b < p.nblk) v = *reinterpret_cast<const uint4*>(xr + (size_t)b * p.B + kc0 + 8 * q);
+        *reinterpret_cast<uint4*>(xs + rr * ld + 8 * q) = v;
+      }
+      for (int i = tid; i < 64 * q8; i += 128) {
+        const int rr = i / q8, q = i - rr * q8, j = j0 + rr;
+        uint4 vh = make_uint4(0, 0, 0, 0), vl = vh;
+        if (j < p.n_b) {
+          vh = *reinterpret_cast<const uint4*>(p.g_hi + (size_t)j * p.B + kc0 + 8 * q);
+          vl = *reinterpret_cast<const uint4*>(p.g_lo + (size_t)j * p.B + kc0 + 8 * q);
+        }
+        *reinterpret_cast<uint4*>(ghs + rr * ld + 8 * q) = vh;
+        *reinterpret_cast<uint4*>(gls + rr * ld + 8 * q) = vl;
+      }
+    } else {
+      for (int i = tid; i < TB * p.kc; i += 128) {
+        const int rr = i / p.kc, kk = i - rr * p.kc, k = kc0 + kk, b = b0 + rr;
+        xs[rr * ld + kk] = (b < p.nblk && k < p.B) ? xr[(size_t)b * p.B + k] : 0;
+      }
+      for (int i = tid; i < 64 * p.kc; i += 128) {
+        const int rr = i / p.kc, kk = i - rr * p.kc, k = kc0 + kk, j = j0 + rr;
+        const bool gv = j < p.n_b && k < p.B;
+        ghs[rr * ld + kk] = gv ? p.g_hi[(size_t)j * p.B + k] : 0;
+        gls[rr * ld + kk] = gv ? p.g_lo[(size_t)j * p.B + k] : 0;
+      }
+    }
+    __syncthreads();
+    for (int ks = 0; ks < p.kc; ks += 16) {
+      uint32_t a[4];
+      const uint16_t* ar = xs + g * ld + ks + 2 * t;
+      a[0] = *reinterpret_cast<const uint32_t*>(ar);
+      a[1] = *reinterpret_cast<const uint32_t*>(ar + 8 * ld);
+      a[2] = *reinterpret_cast<const uint32_t*>(ar + 8);
+      a[3] = *reinterpret_cast<const uint32_t*>(ar + 8 * ld + 8);
+#pragma unroll
+      for (int n = 0; n < NTW; ++n) {
+        const int off = (wcol + n * 8 + g) * ld + ks + 2 * t;
+        const uint32_t h0 = *reinterpret_cast<const uint32_t*>(ghs + off);
+        const uint32_t h1 = *reinterpret_cast<const uint32_t*>(ghs + off + 8);
+        const uint32_t l0 = *reinterpret_cast<const uint32_t*>(gls + off);
+        const uint32_t l1 = *reinterpret_cast<const uint32_t*>(gls + off + 8);
+        mma_bf16_16816(acc[n], a, h0, h1);
+        mma_bf16_16816(acc[n], a, l0, l1);
+      }
+    }
+    __syncthreads();
+  }
+
+  // term scale exponent e_m from the bound
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) xmax = fmaxf(xmax, __shfl_xor_sync(0xffffffffu, xmax, o));
+  if (lane == 0) red[warp] = xmax;
+  __syncthreads();
+  if (tid == 0) {
+    const float mx = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
     int e = 0;
-    if (mx > 0.f) frexpf(mx / 448.f, &e);   // max |x_tilde| * 2^-e < 448
+    if (mx > 0.f) frexpf(mx * p.gnorm / 448.f, &e);   // bound * 2^-e < 448
     e = max(e, -120);
-    se[tid] = e;
-    if (blockIdx.x == 0) p.sexp[tid] = e;
+    e_s = e;
+    if (jt == 0 && bt == 0) p.sexp[m] = e;
   }
   __syncthreads();
-  const int64_t it = (int64_t)blockIdx.x * blockDim.x + tid;
-  if (it >= (int64_t)p.KB * p.M * 8) return;
-  const int ch = (int)(it & 7);
-  const int64_t mk = it >> 3;
-  const int m = (int)(mk % p.M);
-  const int64_t kb = mk / p.M;
-  const float* xr = p.xt + (size_t)m * p.kpad + (size_t)kb * 128;
-  const float inv = ldexpf(1.f, -se[m]);
-  float v[16];
-  if (p.ternary) {
-    // K indices 16 ch .. 16 ch + 15 hold codes 16 ch .. 16 ch + 15, permuted
-    const float4* x4 = reinterpret_cast<const float4*>(xr + 16 * ch);
-    float xv[16];
+  const float inv = ldexpf(1.f, -e_s);
+  const bool ter = p.ternary != 0;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const float4 f = x4[q];
-      xv[4 * q] = f.x; xv[4 * q + 1] = f.y; xv[4 * q + 2] = f.z; xv[4 * q + 3] = f.w;
+  for (int n = 0; n < NTW; ++n)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int b = b0 + g + (e >> 1) * 8;
+      const int j = j0 + wcol + n * 8 + 2 * t + (e & 1);
+      if (b < p.nblk && j < p.n_b) {
+        const int64_t kk = (int64_t)b * p.n_b + j;
+        p.xt[(size_t)m * p.kpad + kk] = acc[n][e];
+        uint8_t* blk = p.bimg + (size_t)(kk >> 7) * p.NP * 128;
+        const int kap = decode_pos((int)(kk & 127), ter);
+        float v = acc[n][e] * inv;
+        for (int tt = 0; tt < p.T; ++tt) {
+          const uint32_t q = f32_to_e4m3(v);
+          const int row = m * p.T + tt;
+          blk[row * 128 + (((kap >> 4) ^ (row & 7)) << 4) + (kap & 15)] = (uint8_t)q;
+          v = (v - e4m3_to_f32(q)) * 16.f;
+        }
+      }
     }
-#pragma unroll
-    for (int u = 0; u < 16; ++u) v[u] = xv[decode_stage_k(u, true)] * inv;
-  } else {
-#pragma unroll
-    for (int u = 0; u < 16; ++u) v[u] = xr[decode_stage_k(16 * ch + u, false)] * inv;
-  }
-  uint8_t* dst = p.bimg + (size_t)kb * p.NP * 128;
-  for (int t = 0; t < p.T; ++t) {
-    uint32_t w[4] = {0u, 0u, 0u, 0u};
-#pragma unroll
-    for (int u = 0; u < 16; ++u) {
-      const uint32_t q = f32_to_e4m3(v[u]);
-      w[u >> 2] |= q << (8 * (u & 3));
-      v[u] = (v[u] - e4m3_to_f32(q)) * 16.f;
+  // K padding of this batch row (x_tilde and its terms are 0 there), and the
+  // decode tickets and error word.
+  if (jt == 0 && bt == 0) {
+    for (int64_t k = p.k_eff + tid; k < p.kpad; k += 128) {
+      p.xt[(size_t)m * p.kpad + k] = 0.f;
+      uint8_t* blk = p.bimg + (size_t)(k >> 7) * p.NP * 128;
+      const int kap = decode_pos((int)(k & 127), ter);
+      for (int tt = 0; tt < p.T; ++tt) {
+        const int row = m * p.T + tt;
+        blk[row * 128 + (((kap >> 4) ^ (row & 7)) << 4) + (kap & 15)] = 0;
+      }
     }
-    const int n = m * p.T + t;
-    *reinterpret_cast<uint4*>(dst + n * 128 + ((ch ^ (n & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+    if (m == 0 && p.cnt)
+      for (int i = tid; i < p.ncnt; i += 128) p.cnt[i] = 0u;
   }
 }
 
@@ -231,30 +343,47 @@ __global__ void __launch_bounds__(256) terms_kernel(TermsParams p) {
 cudaError_t launch_prep(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws, cudaStream_t st) {
   const Geometry& g = pl->geo;
   const WsLayout L = workspace_layout(pl, M);
+  uint8_t* base = static_cast<uint8_t*>(ws);
+  const int vec = (g.block % 32 == 0) && ((reinterpret_cast<uintptr_t>(x) & 15u) == 0);
+  if (M <= kMaxDecodeM) {
+    const DecodeConfig& dc = decode_config(pl, M);
+    DecPrepParams p;
+    p.x = x; p.g_hi = pl->d_g_hi; p.g_lo = pl->d_g_lo;
+    p.xt = reinterpret_cast<float*>(base + L.xt);
+    p.bimg = base + L.bimg;
+    p.sexp = reinterpret_cast<int*>(base + L.sexp);
+    p.cnt = reinterpret_cast<uint32_t*>(base + L.cnt);
+    p.ncnt = g.ntiles + 1;   // the tile tickets and the error word that follows them
+    p.gnorm = pl->gnorm;
+    p.M = M; p.K = g.k_in; p.B = g.block; p.n_b = g.n_b; p.nblk = g.nblk;
+    p.T = dc.T; p.NP = dc.NP;
+    p.kc = std::max(16, std::min(g.block, 256));
+    p.ternary = g.bits == 2;
+    p.vec = vec;
+    p.k_eff = g.k_eff; p.kpad = g.k_eff_pad;
+    const size_t smem = (size_t)(16 + 128) * (p.kc + 8) * sizeof(uint16_t);
+    cudaError_t e = cudaFuncSetAttribute(prep_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    dim3 grid((g.n_b + 63) / 64, (g.nblk + 15) / 16, M);
+    return launch_pdl(prep_decode_kernel, grid, dim3(128), smem, st, p);
+  }
   PrepParams p;
   p.x = x; p.g_hi = pl->d_g_hi; p.g_lo = pl->d_g_lo;
-  uint8_t* base = static_cast<uint8_t*>(ws);
-  p.prefill = M > kMaxDecodeM;
-  p.xt = p.prefill ? nullptr : reinterpret_cast<float*>(base + L.xt);
-  p.xtb = p.prefill ? reinterpret_cast<uint16_t*>(base + L.xt) : nullptr;
+  p.prefill = 1;
+  p.xt = nullptr;
+  p.xtb = reinterpret_cast<uint16_t*>(base + L.xt);
   p.M = M; p.K = g.k_in; p.B = g.block; p.n_b = g.n_b; p.nblk = g.nblk;
   p.k_eff = g.k_eff; p.kpad = g.k_eff_pad;
   p.ternary = pl->desc.quantizer == SDQ_TERNARY;
-  p.vec = (g.block % 32 == 0) && ((reinterpret_cast<uintptr_t>(x) & 15u) == 0);
+  p.vec = vec;
   const bool small = (int64_t)M * g.nblk < 4 * (int64_t)pl->sm_count;
   const int TB = small ? 16 : 64;
   p.JT = (g.n_b + 63) / 64;
   const int BT = (g.nblk + TB - 1) / TB;
   p.P = p.JT * BT;
-  if (p.prefill) {
-    p.pmax = nullptr;
-    p.cnt = reinterpret_cast<uint32_t*>(base + L.err);   // the error word
-    p.ncnt = 1;
-  } else {
-    p.pmax = reinterpret_cast<float*>(base + L.pmax);
-    p.cnt = reinterpret_cast<uint32_t*>(base + L.cnt);
-    p.ncnt = g.ntiles + 1;   // the tile tickets and the error word that follows them
-  }
+  p.pmax = nullptr;
+  p.cnt = reinterpret_cast<uint32_t*>(base + L.err);   // the error word
+  p.ncnt = 1;
   dim3 grid(p.JT, BT, M);
   return small ? launch_pdl(prep_kernel<16>, grid, dim3(128), 0, st, p)
                : launch_pdl(prep_kernel<64>, grid, dim3(128), 0, st, p);
@@ -265,24 +394,6 @@ int prep_partials(const sdq_plan_s* pl, int M) {
   const bool small = (int64_t)M * g.nblk < 4 * (int64_t)pl->sm_count;
   const int TB = small ? 16 : 64;
   return ((g.n_b + 63) / 64) * ((g.nblk + TB - 1) / TB);
-}
-
-cudaError_t launch_terms(const sdq_plan_s* pl, int M, void* ws, cudaStream_t st) {
-  const Geometry& g = pl->geo;
-  const WsLayout L = workspace_layout(pl, M);
-  const DecodeConfig& dc = decode_config(pl, M);
-  uint8_t* base = static_cast<uint8_t*>(ws);
-  TermsParams p;
-  p.xt = reinterpret_cast<const float*>(base + L.xt);
-  p.pmax = reinterpret_cast<const float*>(base + L.pmax);
-  p.bimg = base + L.bimg;
-  p.sexp = reinterpret_cast<int*>(base + L.sexp);
-  p.M = M; p.T = dc.T; p.NP = dc.NP; p.pp = dc.pp;
-  p.KB = (int)(g.k_eff_pad / 128);
-  p.ternary = g.bits == 2;
-  p.kpad = g.k_eff_pad;
-  const int64_t items = (int64_t)p.KB * M * 8;
-  return launch_pdl(terms_kernel, dim3((unsigned)((items + 255) / 256)), dim3(256), 0, st, p);
 }
 
 }  // namespace sdq

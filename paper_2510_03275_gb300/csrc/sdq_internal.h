@@ -56,6 +56,7 @@ struct sdq_plan_s {
   sdq::Geometry geo;
   int device;
   int sm_count;
+  float gnorm;         // max_j sum_k |G[j][k]| (bound of |x_tilde| / max |x|)
   float* d_at;         // encode table, transposed: B x n_b (At[k][j] = A_enc[j][k])
   uint16_t* d_g_hi;    // G as bf16 hi part, n_b x B row-major
   uint16_t* d_g_lo;    // G - hi as bf16, n_b x B row-major
