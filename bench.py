@@ -43,6 +43,9 @@ def parse():
     ap.add_argument("--m", type=int, default=1, help="decode batch")
     ap.add_argument("--no-extras", action="store_true", help="skip encode/prefill/sweep/cpu legs")
     ap.add_argument("--linears", default="", help="comma list of cfg4 linears to run (default: all 7)")
+    ap.add_argument("--eager", action="store_true",
+                    help="launch every step eagerly instead of replaying a CUDA graph (same kernels; "
+                         "for profilers that cannot follow stream capture)")
     return ap.parse_args()
 
 
@@ -210,16 +213,21 @@ def run_sdq(args, rank, world, dist):
         for _ in range(3):
             step()
     torch.cuda.synchronize()
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph, stream=stream):
-        step()
-    torch.cuda.synchronize()
+    if args.eager:
+        replay = step
+    else:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            step()
+        torch.cuda.synchronize()
+        replay = graph.replay
 
     sampler = ClockSampler(dev)
     sampler.start()
     time.sleep(0.3)
-    for _ in range(max(3, args.warmup)):
-        graph.replay()
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, args.warmup)):
+            replay()
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
@@ -229,7 +237,7 @@ def run_sdq(args, rank, world, dist):
     ev0.record(stream)
     with torch.cuda.stream(stream):
         for _ in range(args.steps):
-            graph.replay()
+            replay()
     ev1.record(stream)
     torch.cuda.synchronize()
     t_wall1 = time.time()
@@ -309,7 +317,8 @@ def run_sdq(args, rank, world, dist):
                                + (f" [only {args.linears}]" if args.linears else ""),
                    "decode_batch": M, "code_bytes_per_step": code_bytes,
                    "l2": "7 code matrices (428 MB) streamed in turn > 129 MB L2",
-                   "timing": "CUDA graph of one step, replayed; events on the launch stream",
+                   "timing": ("eager launches" if args.eager else "CUDA graph of one step, replayed")
+                             + "; events on the launch stream",
                    "parallelism": f"replicas x{world}"},
         "clocks": clocks,
         "e2e": {"value": round(e2e_val, 1), "unit": "GB/s", "h2d_bytes_per_step": h2d,

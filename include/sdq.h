@@ -48,21 +48,20 @@
  * Ternary fields: 00 = 0, 01 = +1, 11 = -1 (10 is invalid).  Binary: 1 = +1,
  * 0 = -1.  Padding bits are 0.
  *
- * Tiled layout (input of sdq_contract; built by sdq_pack):  rows are grouped
- * by 16 (row group G) and codes by kc = 128 (ternary) or 256 (binary)
- * (chunk c).  Tile (G, c) holds rows [16G, 16G+16) x codes [kc c, kc c + kc)
- * in 128 consecutive uint32 words starting at word 128 * (G * C + c),
- * C = ceil(K_eff / kc).  Word 32 q + L (q = 0..3, L = 0..31, g = L / 4,
- * t = L % 4) holds these codes, field f at bits [b f, b f + b):
- *   ternary: j = 3 - f % 4, i = f / 4,
- *            row = 16G + g + 8 (j % 2),  k = 128c + 32q + 16 (j / 2) + 4t + i
- *   binary:  j = 7 - f % 8, i = f / 8,
- *            row = 16G + g + 8 (j % 2),
- *            k = 256c + 64q + 32 (j / 4) + 16 ((j / 2) % 2) + 4t + i
- * Codes past n_out or K_eff are padding with field value 0.  With this map,
- * (word << 2j) & 0xC0C0C0C0 (ternary) and ((~word << j) & 0x80808080) |
- * 0x40404040 (binary) are directly the fp8 (e4m3) A-operand registers of a
- * 16x8x32 warp MMA, each byte +-2.0 or 0.
+ * Tiled layout (input of sdq_contract; built by sdq_pack): the library's own
+ * format (the paper prescribes no storage order).  K_eff is padded to
+ * K_pad = 128 ceil(K_eff / 128) codes; rows are grouped by 128 (row tile T,
+ * n_tiles = ceil(n_out / 128)) and codes by 64 (code group G,
+ * n_groups = K_pad / 64).  Slab (T, G) holds rows [128T, 128T+128) x codes
+ * [64G, 64G+64) in 128 wpg consecutive uint32 words starting at word
+ * 128 wpg (T n_groups + G), wpg = 64 b / 32 (4 ternary, 2 binary): row
+ * 128T + r owns the wpg words from 128 wpg (T n_groups + G) + wpg r, in
+ * which its 64 codes sit in natural order with the plain layout's bit map
+ * (code 64G + kk at bit b (kk % (32/b)) of word kk / (32/b)).  So every row
+ * keeps a 16-byte (ternary) or 8-byte (binary) run of its plain words per
+ * group, and the tile's slabs of consecutive groups are contiguous in
+ * memory: one bulk copy streams a 128-row x (64 n)-code stage.  Codes past
+ * n_out or K_eff are padding with field value 0.
  */
 #ifndef SDQ_H_
 #define SDQ_H_
@@ -160,19 +159,22 @@ int sdq_unpack(sdq_plan plan, const uint32_t* codes_tiled, uint32_t* codes_plain
 
 /* x_tilde = G x_b for every block b of every row of x (device, bf16 bits,
  * M x k_in row-major), written into the workspace `ws` for sdq_contract.
- * For M <= 64 x_tilde is kept in fp32 and, by a second kernel, as the fp8
- * B-operand fragments of the decode MMAs (a three-term e4m3 expansion of
- * x_tilde * s for M <= 2, two-term above; s a power of two per batch row);
- * for M > 64 it is written in bf16 in the permuted K order the prefill kernel
- * reads.  Kernels are launched with programmatic dependent launch. */
+ * M <= 64: one kernel writes x_tilde in fp32 and, as the decode kernel's
+ * tensor-core B operand, T e4m3 terms per batch row m with
+ * x_tilde[m] 2^-e_m = sum_t 16^-t q_t[m] (T = 4 for M <= 16, 3 for M <= 21,
+ * else 2); e_m is set from the bound |x_tilde[m, j]| <= gnorm max_k |x[m, k]|,
+ * gnorm = max_j sum_k |G[j, k]|, so that no thread block waits for another.
+ * M > 64: x_tilde is written in bf16 in the permuted K order the prefill
+ * kernel reads.  Kernels are launched with programmatic dependent launch. */
 int sdq_prep_activations(sdq_plan plan, const uint16_t* x, int32_t M,
                          void* ws, size_t ws_bytes, void* stream);
 
 /* Contraction against the tiled codes: y (device, fp32, M x n_out row-major)
  * = alpha_r * sum_j c[r,j] x_tilde[m,j], reading the x_tilde that
  * sdq_prep_activations left in `ws` for the same M.  M <= 64: decode kernel
- * (fp8 warp MMAs on register-expanded codes, split-K over CTAs with a
- * deterministic last-CTA reduction).  M > 64: tcgen05 prefill kernel. */
+ * (tcgen05 fp8 MMAs with the codes expanded into tensor memory as the A
+ * operand, split-K over thread blocks with a deterministic last-block
+ * reduction).  M > 64: tcgen05 bf16 prefill kernel. */
 int sdq_contract(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha, int32_t M,
                  float* y, void* ws, size_t ws_bytes, void* stream);
 

@@ -42,7 +42,6 @@ WsLayout workspace_layout(const sdq_plan_s* pl, int M) {
   if (M <= kMaxDecodeM) {
     const DecodeConfig& dc = pl->dcfg[M];
     off = align_up(off + sizeof(float) * (size_t)M * g.k_eff_pad, 256);
-    L.pmax = off;                                  // (unused on the decode path)
     L.bimg = off;                                  // e4m3 B operand image, K/128 x NP x 128 bytes
     off = align_up(off + (size_t)(g.k_eff_pad / 128) * dc.NP * 128, 256);
     L.sexp = off;                                  // per-batch-row scale exponents
@@ -54,7 +53,7 @@ WsLayout workspace_layout(const sdq_plan_s* pl, int M) {
     off = align_up(off + sizeof(uint32_t) * ((size_t)g.ntiles + 1), 256);
   } else {
     off = align_up(off + sizeof(uint16_t) * (size_t)M * g.k_eff_pad, 256);
-    L.pmax = L.bimg = L.sexp = L.part = L.cnt = L.err = off;   // error word only
+    L.bimg = L.sexp = L.part = L.cnt = L.err = off;   // error word only
     off = align_up(off + sizeof(uint32_t), 256);
   }
   L.total = off;

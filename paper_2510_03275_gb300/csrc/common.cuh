@@ -15,7 +15,7 @@ DecodeConfig decode_config_search(const sdq_plan_s* plan, int M);
 inline const DecodeConfig& decode_config(const sdq_plan_s* plan, int M) { return plan->dcfg[M]; }
 
 struct WsLayout {
-  size_t xt, pmax, bimg, sexp, part, cnt, err, total;
+  size_t xt, bimg, sexp, part, cnt, err, total;
 };
 WsLayout workspace_layout(const sdq_plan_s* plan, int M);
 
@@ -32,7 +32,6 @@ cudaError_t launch_decode(const sdq_plan_s* p, const uint32_t* codes, const floa
                           float* y, void* ws, cudaStream_t st, int early);
 cudaError_t launch_prefill(const sdq_plan_s* p, const uint32_t* codes, const float* alpha, int M,
                            float* y, void* ws, cudaStream_t st);
-int prep_partials(const sdq_plan_s* p, int M);  // per-row max partials of the prep grid
 cudaError_t launch_read_prep(const sdq_plan_s* p, int M, const void* ws, float* out, cudaStream_t st);
 
 // ------------------------------------------------------------------ device

@@ -13,9 +13,9 @@
 //             tcgen05.st straight from the shift-and-mask expansion of the
 //             row's packed words (no shared-memory round trip)
 //   B (smem)  the activations as T e4m3 terms per batch row m:
-//             x_tilde[m] * 2^-e_m = sum_t 16^-t q_t[m] (e_m from max |x_tilde|),
+//             x_tilde[m] * 2^-e_m = sum_t 16^-t q_t[m] (e_m from a bound on |x_tilde[m]|),
 //             N = M*T rows rounded up to 16, K-major, 128-byte swizzle,
-//             written for all of K by the prep stage's terms kernel; each CTA
+//             written for all of K by the decode prepare kernel; each CTA
 //             copies the part of its k chunk once
 //   D (TMEM)  fp32, 128 lanes x NP columns
 // so that y[m, r] = alpha_r / 2 * 2^e_m * sum_t 16^-t D[r, m T + t].
@@ -460,7 +460,6 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
   best.M = M;
   best.T = decode_terms(M);
   best.NP = (M * best.T + 15) / 16 * 16;
-  best.pp = prep_partials(pl, M);
   const int KB = (int)(g.k_eff_pad / kBlk);
   const int sms = std::max(1, pl->sm_count);
   const int blk_bytes = kTileRows * kBlk * g.bits / 8;

@@ -22,18 +22,17 @@ namespace {
 constexpr int kKC = 32;       // k per smem stage
 constexpr int kLd = kKC + 8;  // padded bf16 row stride
 
+// Prefill prepare (M > 64): bf16 x_tilde, each 64-code stage of K in the
+// prefill kernel's operand order (prefill_pos64).
 struct PrepParams {
   const uint16_t* x;
   const uint16_t* g_hi;
   const uint16_t* g_lo;
-  float* xt;          // decode: fp32 M x kpad
-  uint16_t* xtb;      // prefill: bf16 M x kpad (permuted)
-  float* pmax;        // decode: M x P
-  uint32_t* cnt;      // decode counters and error word to zero
-  int ncnt;
-  int M, K, B, n_b, nblk, P, JT;
+  uint16_t* xtb;      // bf16 M x kpad (permuted)
+  uint32_t* err;      // the workspace error word, zeroed here
+  int M, K, B, n_b, nblk;
   int64_t k_eff, kpad;
-  int prefill, vec, ternary;
+  int vec, ternary;
 };
 
 // CTA tile: TB blocks (rows) x 64 samples j, 4 warps.  TB = 64: each warp
@@ -44,7 +43,6 @@ __global__ void __launch_bounds__(128) prep_kernel(PrepParams p) {
   __shared__ __align__(16) uint16_t xs[TB * kLd];
   __shared__ __align__(16) uint16_t ghs[64 * kLd];
   __shared__ __align__(16) uint16_t gls[64 * kLd];
-  __shared__ float red[4];
   pdl_wait();
   pdl_launch_dependents();
   const int jt = blockIdx.x, bt = blockIdx.y, m = blockIdx.z;
@@ -113,7 +111,6 @@ __global__ void __launch_bounds__(128) prep_kernel(PrepParams p) {
     __syncthreads();
   }
 
-  float vmax = 0.f;
 #pragma unroll
   for (int n = 0; n < NTW; ++n)
 #pragma unroll
@@ -122,36 +119,17 @@ __global__ void __launch_bounds__(128) prep_kernel(PrepParams p) {
       const int j = j0 + wcol + n * 8 + 2 * t + (e & 1);
       if (b < p.nblk && j < p.n_b) {
         const int64_t kk = (int64_t)b * p.n_b + j;
-        const float v = acc[n][e];
-        if (p.prefill) {
-          const int64_t phys = (kk & ~int64_t(63)) | prefill_pos64((int)(kk & 63), p.ternary);
-          p.xtb[(size_t)m * p.kpad + phys] = float_to_bf16_bits(v);
-        } else {
-          p.xt[(size_t)m * p.kpad + kk] = v;
-          vmax = fmaxf(vmax, fabsf(v));
-        }
+        const int64_t phys = (kk & ~int64_t(63)) | prefill_pos64((int)(kk & 63), p.ternary);
+        p.xtb[(size_t)m * p.kpad + phys] = float_to_bf16_bits(acc[n][e]);
       }
     }
-  if (!p.prefill) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) vmax = fmaxf(vmax, __shfl_xor_sync(0xffffffffu, vmax, o));
-    if (lane == 0) red[warp] = vmax;
-    __syncthreads();
-    if (tid == 0)
-      p.pmax[(size_t)m * p.P + bt * p.JT + jt] = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
-  }
-  // Zero the K padding of this batch row, and the decode counters.
+  // Zero the K padding of this batch row, and the error word.
   if (jt == 0 && bt == 0) {
     for (int64_t k = p.k_eff + tid; k < p.kpad; k += 128) {
-      if (p.prefill) {
-        const int64_t phys = (k & ~int64_t(63)) | prefill_pos64((int)(k & 63), p.ternary);
-        p.xtb[(size_t)m * p.kpad + phys] = 0;
-      } else {
-        p.xt[(size_t)m * p.kpad + k] = 0.f;
-      }
+      const int64_t phys = (k & ~int64_t(63)) | prefill_pos64((int)(k & 63), p.ternary);
+      p.xtb[(size_t)m * p.kpad + phys] = 0;
     }
-    if (m == 0 && p.cnt)
-      for (int i = tid; i < p.ncnt; i += 128) p.cnt[i] = 0u;
+    if (m == 0 && tid == 0) *p.err = 0u;
   }
 }
 
@@ -369,8 +347,6 @@ cudaError_t launch_prep(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws
   }
   PrepParams p;
   p.x = x; p.g_hi = pl->d_g_hi; p.g_lo = pl->d_g_lo;
-  p.prefill = 1;
-  p.xt = nullptr;
   p.xtb = reinterpret_cast<uint16_t*>(base + L.xt);
   p.M = M; p.K = g.k_in; p.B = g.block; p.n_b = g.n_b; p.nblk = g.nblk;
   p.k_eff = g.k_eff; p.kpad = g.k_eff_pad;
@@ -378,22 +354,10 @@ cudaError_t launch_prep(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws
   p.vec = vec;
   const bool small = (int64_t)M * g.nblk < 4 * (int64_t)pl->sm_count;
   const int TB = small ? 16 : 64;
-  p.JT = (g.n_b + 63) / 64;
-  const int BT = (g.nblk + TB - 1) / TB;
-  p.P = p.JT * BT;
-  p.pmax = nullptr;
-  p.cnt = reinterpret_cast<uint32_t*>(base + L.err);   // the error word
-  p.ncnt = 1;
-  dim3 grid(p.JT, BT, M);
+  p.err = reinterpret_cast<uint32_t*>(base + L.err);
+  dim3 grid((g.n_b + 63) / 64, (g.nblk + TB - 1) / TB, M);
   return small ? launch_pdl(prep_kernel<16>, grid, dim3(128), 0, st, p)
                : launch_pdl(prep_kernel<64>, grid, dim3(128), 0, st, p);
-}
-
-int prep_partials(const sdq_plan_s* pl, int M) {
-  const Geometry& g = pl->geo;
-  const bool small = (int64_t)M * g.nblk < 4 * (int64_t)pl->sm_count;
-  const int TB = small ? 16 : 64;
-  return ((g.n_b + 63) / 64) * ((g.nblk + TB - 1) / TB);
 }
 
 }  // namespace sdq
