@@ -178,16 +178,33 @@ int sdq_prep_activations(sdq_plan plan, const uint16_t* x, int32_t M,
 int sdq_contract(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha, int32_t M,
                  float* y, void* ws, size_t ws_bytes, void* stream);
 
-/* sdq_prep_activations followed by sdq_contract on the same stream. */
+/* y = the layer applied to x: same inputs, outputs and errors as
+ * sdq_prep_activations followed by sdq_contract.  For small decode batches
+ * (sdq_forward_kernels() == 1) it is ONE kernel: the decode kernel computes
+ * the part of x_tilde its k chunk needs and its fp8 terms itself, with its own
+ * power-of-two term scale, and writes no x_tilde to `ws` (sdq_read_prep then
+ * returns stale data).  Otherwise it runs the two kernels.  Results of the two
+ * routes agree to within the fp8 term rounding (about 2^-16 relative with
+ * four terms), not bit for bit. */
 int sdq_linear_forward(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha,
                        const uint16_t* x, int32_t M, float* y, void* ws, size_t ws_bytes,
                        void* stream);
 
+/* Kernels sdq_linear_forward launches for this plan, batch M and activation
+ * pointer x (its 16-byte alignment matters): 1 (the decode kernel builds its
+ * own B operand: M <= 4, block a multiple of 16, n_b a multiple of 8, x
+ * 16-byte aligned, and a per-CTA build of at most 64 16-deep MMA steps per
+ * warp) or 2.  0 on invalid input.  Host only. */
+int sdq_forward_kernels(sdq_plan plan, int32_t M, const uint16_t* x);
+
 /* Wait for `stream`, then report whether the last contraction that used
  * `ws` (same plan and M) completed its bounded device-side waits: SDQ_OK or
- * SDQ_ERR_TIMEOUT (a TMA copy did not arrive within about 2 s; the output of
- * that call is invalid).  Prepare calls reset the flag.  Covers both the
- * decode (M <= 64) and the prefill (M > 64) kernels. */
+ * SDQ_ERR_TIMEOUT (a copy or an MMA did not complete within about 2 s; the
+ * output of that call is invalid).  Covers the decode (M <= 64) and the
+ * prefill (M > 64) kernels.  Workspace contents never need resetting: the
+ * split-K tickets and this record carry a process-wide call number, so stale
+ * or random bytes (another call, plan or batch size) do not count, and one
+ * workspace may serve several plans in turn (never two calls at once). */
 int sdq_workspace_status(sdq_plan plan, int32_t M, const void* ws, void* stream);
 
 /* Copy x_tilde for M <= 64 out of the workspace as fp32 (M x K_eff,

@@ -24,7 +24,7 @@ __all__ = [
     "sdq_workspace_bytes", "sdq_build_tables", "sdq_encode_rows", "sdq_pack", "sdq_unpack",
     "sdq_prep_activations", "sdq_contract", "sdq_linear_forward", "sdq_read_prep",
     "sdq_workspace_status", "sdq_linear_forward_noalloc", "sdq_noalloc_scratch_bytes",
-    "sdq_status_string", "Plan",
+    "sdq_forward_kernels", "sdq_status_string", "Plan",
 ]
 
 SDQ_OK = 0
@@ -89,6 +89,7 @@ _SIGS = {
     "sdq_linear_forward": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _vp, _vp, _sz, _vp]),
     "sdq_read_prep": (ctypes.c_int, [_vp, _i32, _vp, _vp, _vp]),
     "sdq_workspace_status": (ctypes.c_int, [_vp, _i32, _vp, _vp]),
+    "sdq_forward_kernels": (ctypes.c_int, [_vp, _i32, _vp]),
     "sdq_linear_forward_noalloc": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _vp, _vp]),
     "sdq_noalloc_scratch_bytes": (_sz, []),
     "sdq_status_string": (ctypes.c_char_p, [ctypes.c_int]),
@@ -211,6 +212,11 @@ def sdq_read_prep(plan, M, ws, out, stream=None):
 def sdq_workspace_status(plan, M, ws, stream=None) -> int:
     """Synchronize and return the status of the last decode using ``ws``."""
     return lib().sdq_workspace_status(plan, M, _ptr(ws), _stream(stream))
+
+
+def sdq_forward_kernels(plan, M, x) -> int:
+    """1 if sdq_linear_forward runs as one kernel for this batch and x, else 2."""
+    return lib().sdq_forward_kernels(plan, M, _ptr(x))
 
 
 def sdq_linear_forward_noalloc(plan, codes_tiled, alpha, x, M, y, stream=None):

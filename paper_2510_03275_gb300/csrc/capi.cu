@@ -1,5 +1,6 @@
 // C ABI of libsdq (declarations and contracts in include/sdq.h).
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
@@ -34,6 +35,11 @@ int cuda_status(cudaError_t e) { return e == cudaSuccess ? SDQ_OK : SDQ_ERR_CUDA
 
 }  // namespace
 
+uint64_t next_call_number() {
+  static std::atomic<uint64_t> calls{0};
+  return ++calls;
+}
+
 WsLayout workspace_layout(const sdq_plan_s* pl, int M) {
   const Geometry& g = pl->geo;
   WsLayout L{};
@@ -48,13 +54,14 @@ WsLayout workspace_layout(const sdq_plan_s* pl, int M) {
     off = align_up(off + sizeof(int32_t) * kMaxDecodeM, 256);
     L.part = off;
     off = align_up(off + (dc.S > 1 ? sizeof(float) * (size_t)dc.S * M * g.ntiles * kTileRows : 0), 256);
-    L.cnt = off;                                   // one ticket per row tile, then the error word
-    L.err = off + sizeof(uint32_t) * (size_t)g.ntiles;
-    off = align_up(off + sizeof(uint32_t) * ((size_t)g.ntiles + 1), 256);
+    L.cnt = off;                                   // one 64-bit ticket per row tile
+    off = align_up(off + sizeof(uint64_t) * (size_t)g.ntiles, 256);
+    L.err = off;                                   // call record
+    off = align_up(off + 2 * sizeof(uint64_t), 256);
   } else {
     off = align_up(off + sizeof(uint16_t) * (size_t)M * g.k_eff_pad, 256);
-    L.bimg = L.sexp = L.part = L.cnt = L.err = off;   // error word only
-    off = align_up(off + sizeof(uint32_t), 256);
+    L.bimg = L.sexp = L.part = L.cnt = L.err = off;   // call record only
+    off = align_up(off + 2 * sizeof(uint64_t), 256);
   }
   L.total = off;
   return L;
@@ -97,6 +104,23 @@ extern "C" int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_sig
     glo[i] = host_bf16((double)gm[i] - host_bf16_value(ghi[i]));
   }
 
+  std::vector<uint16_t> gfrag;
+  if (g.block % 16 == 0 && g.n_b % 8 == 0) {
+    const int kbw = g_frag_batch(g.block), R = kbw / 4, nkb = g.block / kbw;
+    gfrag.resize(2 * tab);
+    for (int jt = 0; jt < g.n_b / 8; ++jt)
+      for (int kb = 0; kb < nkb; ++kb)
+        for (int lane = 0; lane < 32; ++lane) {
+          const int j = 8 * jt + (lane >> 2), t = lane & 3;
+          uint16_t* dst = gfrag.data() + (size_t)2 * R * (32 * ((size_t)jt * nkb + kb) + lane);
+          const size_t src = (size_t)j * g.block + (size_t)kb * kbw + (size_t)t * R;
+          for (int e = 0; e < R; ++e) {   // 32-bit words alternate hi, lo
+            dst[4 * (e >> 1) + (e & 1)] = ghi[src + e];
+            dst[4 * (e >> 1) + 2 + (e & 1)] = glo[src + e];
+          }
+        }
+  }
+
   sdq_plan_s* p = new (std::nothrow) sdq_plan_s();
   if (!p) return SDQ_ERR_ALLOC;
   p->desc = *desc;
@@ -106,13 +130,16 @@ extern "C" int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_sig
   p->gnorm = (float)(gnorm * (1.0 + 1.0 / 1024));
   if (cudaMalloc(&p->d_at, sizeof(float) * tab) != cudaSuccess ||
       cudaMalloc(&p->d_g_hi, sizeof(uint16_t) * tab) != cudaSuccess ||
-      cudaMalloc(&p->d_g_lo, sizeof(uint16_t) * tab) != cudaSuccess) {
+      cudaMalloc(&p->d_g_lo, sizeof(uint16_t) * tab) != cudaSuccess ||
+      (!gfrag.empty() && cudaMalloc(&p->d_g_frag, sizeof(uint16_t) * gfrag.size()) != cudaSuccess)) {
     sdq_plan_destroy(p);
     return SDQ_ERR_ALLOC;
   }
   if (cudaMemcpy(p->d_at, at.data(), sizeof(float) * tab, cudaMemcpyHostToDevice) != cudaSuccess ||
       cudaMemcpy(p->d_g_hi, ghi.data(), sizeof(uint16_t) * tab, cudaMemcpyHostToDevice) != cudaSuccess ||
-      cudaMemcpy(p->d_g_lo, glo.data(), sizeof(uint16_t) * tab, cudaMemcpyHostToDevice) != cudaSuccess) {
+      cudaMemcpy(p->d_g_lo, glo.data(), sizeof(uint16_t) * tab, cudaMemcpyHostToDevice) != cudaSuccess ||
+      (!gfrag.empty() && cudaMemcpy(p->d_g_frag, gfrag.data(), sizeof(uint16_t) * gfrag.size(),
+                                    cudaMemcpyHostToDevice) != cudaSuccess)) {
     sdq_plan_destroy(p);
     return SDQ_ERR_CUDA;
   }
@@ -127,6 +154,7 @@ extern "C" int sdq_plan_destroy(sdq_plan p) {
   if (p->d_at && (e2 = cudaFree(p->d_at)) != cudaSuccess) e = e2;
   if (p->d_g_hi && (e2 = cudaFree(p->d_g_hi)) != cudaSuccess) e = e2;
   if (p->d_g_lo && (e2 = cudaFree(p->d_g_lo)) != cudaSuccess) e = e2;
+  if (p->d_g_frag && (e2 = cudaFree(p->d_g_frag)) != cudaSuccess) e = e2;
   delete p;
   return cuda_status(e);
 }
@@ -170,12 +198,12 @@ extern "C" int sdq_prep_activations(sdq_plan p, const uint16_t* x, int32_t M, vo
 }
 
 static int contract(sdq_plan p, const uint32_t* codes_tiled, const float* alpha, int32_t M, float* y,
-                    void* ws, size_t ws_bytes, void* stream, int early) {
+                    void* ws, size_t ws_bytes, void* stream, int early, const uint16_t* x_fused) {
   int st = check_ws(p, M, ws, ws_bytes);
   if (st != SDQ_OK) return st;
   if (!codes_tiled || !alpha || !y || !aligned16(codes_tiled) || !aligned16(y)) return SDQ_ERR_INVALID_ARG;
   cudaError_t e = M <= kMaxDecodeM
-                      ? launch_decode(p, codes_tiled, alpha, M, y, ws, (cudaStream_t)stream, early)
+                      ? launch_decode(p, codes_tiled, alpha, M, y, ws, (cudaStream_t)stream, early, x_fused)
                       : launch_prefill(p, codes_tiled, alpha, M, y, ws, (cudaStream_t)stream);
   if (e == cudaErrorNotSupported) return SDQ_ERR_UNSUPPORTED;
   return cuda_status(e);
@@ -183,29 +211,38 @@ static int contract(sdq_plan p, const uint32_t* codes_tiled, const float* alpha,
 
 extern "C" int sdq_contract(sdq_plan p, const uint32_t* codes_tiled, const float* alpha, int32_t M,
                             float* y, void* ws, size_t ws_bytes, void* stream) {
-  return contract(p, codes_tiled, alpha, M, y, ws, ws_bytes, stream, 0);
+  return contract(p, codes_tiled, alpha, M, y, ws, ws_bytes, stream, 0, nullptr);
 }
 
-// Behind its own prepare kernels the decode kernel may start reading the
-// codes before the preceding grid finishes: that grid waited for everything
-// before it in the stream, and it does not write the codes.
+// Small decode batches: one kernel that builds its own B operand from x.
+// Otherwise the prepare kernel, then the contraction; behind its own prepare
+// kernel the decode kernel may start reading the codes before the preceding
+// grid finishes: that grid waited for everything before it in the stream, and
+// it does not write the codes.
 extern "C" int sdq_linear_forward(sdq_plan p, const uint32_t* codes_tiled, const float* alpha,
                                   const uint16_t* x, int32_t M, float* y, void* ws, size_t ws_bytes,
                                   void* stream) {
+  if (p && x && M >= 1 && M <= kMaxDecodeM && decode_fusable(p, M, x))
+    return contract(p, codes_tiled, alpha, M, y, ws, ws_bytes, stream, 0, x);
   int st = sdq_prep_activations(p, x, M, ws, ws_bytes, stream);
   if (st != SDQ_OK) return st;
-  return contract(p, codes_tiled, alpha, M, y, ws, ws_bytes, stream, 1);
+  return contract(p, codes_tiled, alpha, M, y, ws, ws_bytes, stream, 1, nullptr);
+}
+
+extern "C" int sdq_forward_kernels(sdq_plan p, int32_t M, const uint16_t* x) {
+  if (!p || !x || M < 1 || M > 65535) return 0;
+  return M <= kMaxDecodeM && decode_fusable(p, M, x) ? 1 : 2;
 }
 
 extern "C" int sdq_workspace_status(sdq_plan p, int32_t M, const void* ws, void* stream) {
   if (!p || M < 1 || M > 65535 || !ws) return SDQ_ERR_INVALID_ARG;
   const WsLayout L = workspace_layout(p, M);
-  uint32_t err = 0;
-  cudaError_t e = cudaMemcpyAsync(&err, static_cast<const uint8_t*>(ws) + L.err, sizeof(err),
+  uint64_t rec[2] = {0, 0};   // last failed call, last call
+  cudaError_t e = cudaMemcpyAsync(rec, static_cast<const uint8_t*>(ws) + L.err, sizeof(rec),
                                   cudaMemcpyDeviceToHost, (cudaStream_t)stream);
   if (e == cudaSuccess) e = cudaStreamSynchronize((cudaStream_t)stream);
   if (e != cudaSuccess) return SDQ_ERR_CUDA;
-  return err ? SDQ_ERR_TIMEOUT : SDQ_OK;
+  return rec[1] != 0 && rec[0] == rec[1] ? SDQ_ERR_TIMEOUT : SDQ_OK;
 }
 
 extern "C" int sdq_read_prep(sdq_plan p, int32_t M, const void* ws, float* xt_out, void* stream) {

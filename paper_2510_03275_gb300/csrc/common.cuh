@@ -14,10 +14,14 @@ namespace sdq {
 DecodeConfig decode_config_search(const sdq_plan_s* plan, int M);
 inline const DecodeConfig& decode_config(const sdq_plan_s* plan, int M) { return plan->dcfg[M]; }
 
+// Workspace regions (byte offsets).  cnt: one 64-bit split-K ticket per row
+// tile; err: the call record (two 64-bit words, see call_record_*).
 struct WsLayout {
   size_t xt, bimg, sexp, part, cnt, err, total;
 };
 WsLayout workspace_layout(const sdq_plan_s* plan, int M);
+// Number of a contraction call, from one process-wide counter (never 0).
+uint64_t next_call_number();
 
 // Kernel launchers (return cudaError_t of the launch).
 cudaError_t launch_encode(const sdq_plan_s* p, const float* W, uint32_t* codes, float* alpha,
@@ -28,8 +32,12 @@ cudaError_t launch_unpack(const sdq_plan_s* p, const uint32_t* tiled, uint32_t* 
 cudaError_t launch_prep(const sdq_plan_s* p, const uint16_t* x, int M, void* ws, cudaStream_t st);
 // early = 1: the decode kernel starts streaming codes before waiting for the
 // preceding grid (valid only behind this library's own prep kernels).
+// x != nullptr: the decode kernel builds its B operand from x itself (no prep
+// kernel; see decode_fusable).
 cudaError_t launch_decode(const sdq_plan_s* p, const uint32_t* codes, const float* alpha, int M,
-                          float* y, void* ws, cudaStream_t st, int early);
+                          float* y, void* ws, cudaStream_t st, int early, const uint16_t* x);
+// Whether the decode kernel can build its own B operand for batch M from x.
+bool decode_fusable(const sdq_plan_s* p, int M, const uint16_t* x);
 cudaError_t launch_prefill(const sdq_plan_s* p, const uint32_t* codes, const float* alpha, int M,
                            float* y, void* ws, cudaStream_t st);
 cudaError_t launch_read_prep(const sdq_plan_s* p, int M, const void* ws, float* out, cudaStream_t st);
@@ -234,6 +242,46 @@ __device__ __forceinline__ void umma_f8_ts(uint32_t d_tmem, uint32_t a_tmem, uin
 }
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;\n" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// Call record in the workspace: word 0 = number of the last call that gave up
+// a bounded wait, word 1 = number of the last call that ran.  Call numbers
+// are never 0 and never repeat, so a record written by another call, plan or
+// batch size (or random initial contents, barring a 2^-64 coincidence) does
+// not read as the current call's: nothing in the workspace needs resetting.
+__device__ __forceinline__ void call_record_start(uint64_t* rec, uint64_t call, bool leader) {
+  if (leader) rec[1] = call;
+}
+__device__ __forceinline__ void call_record_fail(uint64_t* rec, uint64_t call) {
+  atomicExch(reinterpret_cast<unsigned long long*>(rec), (unsigned long long)call);
+}
+
+// Split-K ticket of one row tile: bits 8..63 the call number, bits 0..7 the
+// arrivals of that call.  A ticket that carries another call number counts
+// as empty, so tickets need no reset between calls.  Returns this CTA's
+// arrival number (1..255), or 0 if the compare-and-swap did not settle within
+// its retry bound.
+__device__ __forceinline__ uint32_t ticket_take(uint64_t* tk, uint64_t call) {
+  unsigned long long* p = reinterpret_cast<unsigned long long*>(tk);
+  unsigned long long cur = *reinterpret_cast<volatile unsigned long long*>(p);
+  for (int it = 0; it < (1 << 20); ++it) {
+    const unsigned long long base = (cur >> 8) == call ? cur : ((unsigned long long)call << 8);
+    const unsigned long long prev = atomicCAS(p, cur, base + 1);
+    if (prev == cur) return (uint32_t)((base & 0xFFu) + 1);
+    cur = prev;
+  }
+  return 0;
+}
+
+// MMA K position (within a 128-code block) of natural code kl: the inverse of
+// decode_stage_k below.
+__host__ __device__ __forceinline__ int decode_pos(int kl, bool ternary) {
+  if (ternary) {
+    const int f = kl & 15;
+    return (kl & ~15) + 4 * (3 - (f & 3)) + (f >> 2);
+  }
+  const int f = kl & 31;
+  return (kl & ~31) + 4 * (7 - (f & 7)) + (f >> 3);
 }
 
 // Natural k (within a 128-code decode block) at MMA K index kap: the order in

@@ -73,16 +73,27 @@ constexpr int kMaxRing = 24;
 constexpr int kMaxSpu = 128;                     // stages per row tile (config search bound)
 constexpr int kSmemMax = 224 * 1024;
 constexpr int kSmemMin = 120 * 1024;             // > half an SM: one CTA per SM
+constexpr int kMaxFuseM = 4;                     // batch rows of the fused B operand
+constexpr int kBuildThreads = 32 * 4 * kExpSets; // the expander warps build it
+constexpr int kMaxBuildSteps = 64;               // 16-deep MMA steps per warp (fusion bound)
+constexpr int kFusePre = 4;                      // code stages requested before the B operand is built
 
 struct DecodeParams {
   const uint32_t* codes;
   const float* alpha;
-  const uint8_t* bimg;   // B operand image: KB x NP x 128 bytes
-  const int* sexp;       // per-batch-row scale exponents e_m
+  const uint8_t* bimg;   // B operand image: KB x NP x 128 bytes (prepared path)
+  const int* sexp;       // per-batch-row scale exponents e_m (prepared path)
   float* y;              // M x n_out
   float* part;           // S x M x (ntiles * 128) split-K partials
-  uint32_t* cnt;         // ntiles tickets (zeroed by the prep kernel)
-  uint32_t* err;
+  uint64_t* cnt;         // ntiles split-K tickets (ticket_take)
+  uint64_t* rec;         // call record
+  uint64_t call;
+  // Fused path (fused = 1): the B operand is built in the kernel from x.
+  const uint16_t* x;     // M x K bf16 bits
+  const uint16_t* g_frag; // G = D^T Had^T, bf16 hi + lo, warp-fragment order (g_frag_batch)
+  float gnorm;           // max_j sum_i |G[j, i]| (with margin)
+  int fused, K, B, n_b;
+  int64_t k_eff;
   int M, T, NP, S, P, CB, KB, ring, sb, nbuf, dbase;
   int n_out, ntiles, ngroups, ternary, early;
   uint32_t blk_bytes, slot_bytes, b_bytes;
@@ -107,6 +118,257 @@ __device__ __forceinline__ bool group_and(int id, int nthreads, bool v) {
 // blocks [first, last).
 __device__ __forceinline__ int stage_block(int j, int ncb, int spu) { return j * ncb / spu; }
 
+__device__ __forceinline__ float bf16_mag(uint32_t h) { return __uint_as_float((h & 0x7FFFu) << 16); }
+
+// Fused B operand (small decode batches): the expander warps compute x_tilde
+// for this CTA's k chunk only,
+//   x_tilde[m, b n_b + j] = sum_i G[j, i] x[m, b B + i]      (G = D^T Had^T)
+// on warp MMAs (bf16 x exact, G as bf16 hi + lo, fp32 accumulation), and
+// write its T e4m3 terms into the shared-memory B image, laid out as the
+// decode prepare kernel lays out the global one.  The term scale 2^e_m is
+// this CTA's own, from the bound |x_tilde[m, k]| <= gnorm max |x[m, i]| over
+// the input blocks the chunk reads; the epilogue applies it to this CTA's
+// products only, so no CTA waits for another.
+//
+// MMA tiles are 16 (m, b) rows x 8 codes j.  Per k batch of kbw inputs each
+// lane loads one contiguous run of x per row and one of G (the plan's
+// fragment-ordered copy), 16 bytes at a time: input t R + 4 s + r of the batch
+// is MMA K index 2t + (r & 1) + 8 (r >> 1) of step s, for x and G alike, which
+// leaves the dot products unchanged.
+struct BuildGeo {
+  int64_t k0, k1, kend;   // chunk codes [k0, kend), with a value below k1
+  int blo, nbi, rows;     // first input block, input blocks, (m, b) rows (m-major)
+  int kbw, R, nkb, S4;    // k batch, run length, batches, 16-deep steps per batch
+};
+
+// G fragments of code tile jt, batch kb.
+__device__ __forceinline__ void load_g_frags(const DecodeParams& p, const BuildGeo& q, int jt, int kb, int lane,
+                                             uint32_t (&gw)[16]) {
+  const uint4* gf = reinterpret_cast<const uint4*>(p.g_frag) +
+                    ((size_t)(jt * q.nkb + kb) * 32 + lane) * (q.kbw / 16);
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (c < q.kbw / 16) v = __ldg(gf + c);
+    gw[4 * c] = v.x; gw[4 * c + 1] = v.y; gw[4 * c + 2] = v.z; gw[4 * c + 3] = v.w;
+  }
+}
+
+// x runs of rows xa0 / xa1 (lane offset applied) for batch kb.
+__device__ __forceinline__ void load_x_frags(const BuildGeo& q, const uint16_t* xa0, const uint16_t* xa1, int kb,
+                                             uint32_t (&xw)[2][8]) {
+#pragma unroll
+  for (int c = 0; c < 2; ++c) {
+    const bool in = c < q.kbw / 32 || (c == 0 && q.kbw == 16);
+    uint4 v0 = make_uint4(0, 0, 0, 0), v1 = v0;
+    if (in && q.kbw >= 32) {
+      v0 = __ldg(reinterpret_cast<const uint4*>(xa0 + kb * q.kbw) + c);
+      v1 = __ldg(reinterpret_cast<const uint4*>(xa1 + kb * q.kbw) + c);
+    } else if (in) {   // kbw = 16: R = 4 inputs, 8 bytes per row
+      const uint2 h0 = __ldg(reinterpret_cast<const uint2*>(xa0 + kb * q.kbw));
+      const uint2 h1 = __ldg(reinterpret_cast<const uint2*>(xa1 + kb * q.kbw));
+      v0.x = h0.x; v0.y = h0.y; v1.x = h1.x; v1.y = h1.y;
+    }
+    xw[0][4 * c] = v0.x; xw[0][4 * c + 1] = v0.y; xw[0][4 * c + 2] = v0.z; xw[0][4 * c + 3] = v0.w;
+    xw[1][4 * c] = v1.x; xw[1][4 * c + 1] = v1.y; xw[1][4 * c + 2] = v1.z; xw[1][4 * c + 3] = v1.w;
+  }
+}
+
+// Separate accumulators for the hi and lo parts of G halve the MMA
+// dependency chains; they are summed once per tile.
+__device__ __forceinline__ void mma_batch(const BuildGeo& q, const uint32_t (&xw)[2][8], const uint32_t (&gw)[16],
+                                          float (&acc)[2][4]) {
+#pragma unroll
+  for (int s = 0; s < 4; ++s)
+    if (s < q.S4) {
+      const uint32_t a[4] = {xw[0][2 * s], xw[1][2 * s], xw[0][2 * s + 1], xw[1][2 * s + 1]};
+      mma_bf16_16816(acc[0], a, gw[4 * s], gw[4 * s + 2]);       // G words alternate hi and lo pairs
+      mma_bf16_16816(acc[1], a, gw[4 * s + 1], gw[4 * s + 3]);
+    }
+}
+__device__ __forceinline__ void acc_sum(const float (&a)[2][4], float (&out)[4]) {
+#pragma unroll
+  for (int e = 0; e < 4; ++e) out[e] = a[0][e] + a[1][e];
+}
+// max of |bf16| over the halves of a word, as an order-preserving integer
+// (the magnitude bits of a non-negative float)
+__device__ __forceinline__ uint32_t bf16x2_absmax_bits(uint32_t w, uint32_t cur) {
+  return max(cur, max(w & 0x7FFF0000u, (w << 16) & 0x7FFF0000u));
+}
+
+// T e4m3 terms of the lane's four x_tilde values of tile (rows r0, r1; codes 8 jt ..).
+template <int T>
+__device__ __forceinline__ void write_terms_t(const DecodeParams& p, const BuildGeo& q, uint8_t* bop, int jt, int t,
+                                              int r0, int r1, int m0, int m1, float inv0, float inv1,
+                                              const float (&acc)[4]) {
+  const bool ter = p.ternary != 0;
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const int rho = e < 2 ? r0 : r1;
+    if (rho >= q.rows) continue;
+    const int m = e < 2 ? m0 : m1;
+    const int64_t k = (int64_t)(q.blo + rho - m * q.nbi) * p.n_b + jt * 8 + 2 * t + (e & 1);
+    if (k < q.k0 || k >= q.k1) continue;
+    const int kl = (int)(k - q.k0);
+    uint8_t* blk = bop + (size_t)(kl >> 7) * p.NP * 128;
+    const int kap = decode_pos(kl & 127, ter);
+    float v = acc[e] * (e < 2 ? inv0 : inv1);
+#pragma unroll
+    for (int tt = 0; tt < T; ++tt) {
+      const uint32_t qb = f32_to_e4m3(v);
+      const int row = m * T + tt;
+      blk[row * 128 + (((kap >> 4) ^ (row & 7)) << 4) + (kap & 15)] = (uint8_t)qb;
+      if (tt + 1 < T) v = (v - e4m3_to_f32(qb)) * 16.f;
+    }
+  }
+}
+__device__ __forceinline__ void write_terms(const DecodeParams& p, const BuildGeo& q, uint8_t* bop, int jt, int t,
+                                            int r0, int r1, int m0, int m1, float inv0, float inv1,
+                                            const float (&acc)[4]) {
+  switch (p.T) {
+    case 4: write_terms_t<4>(p, q, bop, jt, t, r0, r1, m0, m1, inv0, inv1, acc); break;
+    case 3: write_terms_t<3>(p, q, bop, jt, t, r0, r1, m0, m1, inv0, inv1, acc); break;
+    default: write_terms_t<2>(p, q, bop, jt, t, r0, r1, m0, m1, inv0, inv1, acc); break;
+  }
+}
+
+__device__ __forceinline__ int term_exponent(float mx, float gnorm) {
+  int e = 0;
+  if (mx > 0.f) frexpf(mx * gnorm / 448.f, &e);   // bound * 2^-e < 448
+  return max(e, -120);
+}
+
+// Called by the kBuildThreads expander threads before their first stage; it
+// waits for the preceding grid itself (x may come from it; G does not).
+__device__ void build_b_operand(const DecodeParams& p, uint8_t* bop, int kb0, int ncb, int et,
+                                uint32_t* xmax_u, float* inv_s, float* scale_s) {
+  BuildGeo q;
+  q.k0 = (int64_t)kb0 * kBlk;
+  q.kend = q.k0 + (int64_t)ncb * kBlk;
+  q.k1 = min(q.kend, p.k_eff);
+  q.blo = (int)(q.k0 / p.n_b);
+  q.nbi = (int)((q.k1 - 1) / p.n_b) - q.blo + 1;   // k1 > k0: a block always holds a code
+  q.rows = p.M * q.nbi;
+  q.kbw = g_frag_batch(p.B);
+  q.R = q.kbw / 4;
+  q.nkb = p.B / q.kbw;
+  q.S4 = q.kbw / 16;
+  const int ew = et >> 5, lane = et & 31, g = lane >> 2, t = lane & 3;
+  constexpr int NW = kBuildThreads / 32;
+  const int JT = p.n_b / 8;
+
+  if (q.rows <= 16 && q.nkb <= 2) {
+    // One row tile, B <= 128: every warp holds all of x's chunk in its A
+    // fragments, so each takes max |x[m]| from them (no cross-warp step); the
+    // G fragments of the warp's first code tile are loaded before the wait.
+    pdl_wait();
+    const bool v0 = g < q.rows, v1 = g + 8 < q.rows;
+    const int m0 = v0 ? g / q.nbi : 0, m1 = v1 ? (g + 8) / q.nbi : 0;
+    const uint16_t* xa0 = p.x + t * q.R + (v0 ? (size_t)m0 * p.K + (size_t)(q.blo + g - m0 * q.nbi) * p.B : 0);
+    const uint16_t* xa1 = p.x + t * q.R + (v1 ? (size_t)m1 * p.K + (size_t)(q.blo + g + 8 - m1 * q.nbi) * p.B : 0);
+    uint32_t mx0 = 0u, mx1 = 0u;   // max |x| bits of rows g, g + 8
+    float inv0 = 1.f, inv1 = 1.f;
+    for (int jt = ew; jt < JT; jt += NW) {
+      const bool first = jt == ew;
+      float acc4[2][4] = {};
+#pragma unroll
+      for (int kb = 0; kb < 2; ++kb)
+        if (kb < q.nkb) {
+          uint32_t xw[2][8], gw[16];
+          load_g_frags(p, q, jt, kb, lane, gw);
+          load_x_frags(q, xa0, xa1, kb, xw);   // (again for later tiles: an L1 hit)
+          if (first)
+#pragma unroll
+            for (int w = 0; w < 8; ++w) {
+              mx0 = bf16x2_absmax_bits(xw[0][w], mx0);
+              mx1 = bf16x2_absmax_bits(xw[1][w], mx1);
+            }
+          mma_batch(q, xw, gw, acc4);
+        }
+      float acc[4];
+      acc_sum(acc4, acc);
+      if (first) {   // max |x[m]| over the warp's fragments = over the whole chunk
+#pragma unroll
+        for (int mm = 0; mm < kMaxFuseM; ++mm) {
+          if (mm >= p.M) break;
+          uint32_t v = max(v0 && m0 == mm ? mx0 : 0u, v1 && m1 == mm ? mx1 : 0u);
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) v = max(v, __shfl_xor_sync(0xffffffffu, v, o));
+          const int e = term_exponent(__uint_as_float(v), p.gnorm);
+          if (m0 == mm) inv0 = ldexpf(1.f, -e);
+          if (m1 == mm) inv1 = ldexpf(1.f, -e);
+          if (et == mm) scale_s[mm] = ldexpf(1.f, e);
+        }
+      }
+      write_terms(p, q, bop, jt, t, g, g + 8, m0, m1, inv0, inv1, acc);
+    }
+  } else {
+    pdl_wait();
+    // max |x[m, .]| over the chunk's input blocks: 16-byte loads, 4 in flight
+    const int bq = p.B / 8;
+    const int nq = q.rows * bq;
+    for (int i0 = et; i0 < nq; i0 += 4 * kBuildThreads) {
+      uint4 v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = i0 + u * kBuildThreads;
+        v[u] = make_uint4(0, 0, 0, 0);
+        if (i < nq) {
+          const int rho = i / bq, c = i - rho * bq, m = rho / q.nbi, b = q.blo + rho - m * q.nbi;
+          v[u] = __ldg(reinterpret_cast<const uint4*>(p.x + (size_t)m * p.K + (size_t)b * p.B) + c);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = i0 + u * kBuildThreads;
+        if (i < nq) {
+          const uint32_t w[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+          float mx = 0.f;
+#pragma unroll
+          for (int c = 0; c < 4; ++c) mx = fmaxf(mx, fmaxf(bf16_mag(w[c]), bf16_mag(w[c] >> 16)));
+          atomicMax(xmax_u + (i / bq) / q.nbi, __float_as_uint(mx));   // non-negative floats order as integers
+        }
+      }
+    }
+    named_bar_sync(3, kBuildThreads);
+    if (et < p.M) {
+      const int e = term_exponent(__uint_as_float(xmax_u[et]), p.gnorm);
+      scale_s[et] = ldexpf(1.f, e);
+      inv_s[et] = ldexpf(1.f, -e);
+    }
+    named_bar_sync(3, kBuildThreads);
+    const int RT = (q.rows + 15) / 16;
+    for (int it = ew; it < RT * JT; it += NW) {
+      const int rt = it / JT, jt = it - rt * JT;
+      const int r0 = rt * 16 + g, r1 = r0 + 8;
+      const int m0 = r0 < q.rows ? r0 / q.nbi : 0, m1 = r1 < q.rows ? r1 / q.nbi : 0;
+      const uint16_t* xa0 = p.x + t * q.R + (r0 < q.rows ? (size_t)m0 * p.K + (size_t)(q.blo + r0 - m0 * q.nbi) * p.B : 0);
+      const uint16_t* xa1 = p.x + t * q.R + (r1 < q.rows ? (size_t)m1 * p.K + (size_t)(q.blo + r1 - m1 * q.nbi) * p.B : 0);
+      float acc4[2][4] = {};
+      for (int kb = 0; kb < q.nkb; ++kb) {
+        uint32_t xw[2][8], gw[16];
+        load_x_frags(q, xa0, xa1, kb, xw);
+        load_g_frags(p, q, jt, kb, lane, gw);
+        mma_batch(q, xw, gw, acc4);
+      }
+      float acc[4];
+      acc_sum(acc4, acc);
+      write_terms(p, q, bop, jt, t, r0, r1, m0, m1, inv_s[m0], inv_s[m1], acc);
+    }
+  }
+  // padding codes [k1, kend): zero terms
+  const int npad = (int)(q.kend - q.k1), lo = (int)(q.k1 - q.k0);
+  const bool ter = p.ternary != 0;
+  for (int i = et; i < npad * p.M * p.T; i += kBuildThreads) {
+    const int row = i / npad, kl = lo + (i - row * npad);
+    uint8_t* blk = bop + (size_t)(kl >> 7) * p.NP * 128;
+    const int kap = decode_pos(kl & 127, ter);
+    blk[row * 128 + (((kap >> 4) ^ (row & 7)) << 4) + (kap & 15)] = 0;
+  }
+  fence_proxy_async_smem();   // generic-proxy stores -> the MMAs' async-proxy reads
+  named_bar_sync(3, kBuildThreads);
+}
+
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t c_full[kMaxRing], c_empty[kMaxRing];
@@ -115,6 +377,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   __shared__ uint32_t tmem_base;
   __shared__ int last[128];
   __shared__ float scale_s[kMaxDecodeM];   // 2^e_m
+  __shared__ float inv_s[kMaxFuseM];       // 2^-e_m (fused B operand)
+  __shared__ uint32_t xmax_u[kMaxFuseM];   // max |x[m]| bits (fused B operand)
   __shared__ int sblk[kMaxSpu + 1];         // first block of stage j of a tile
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -144,6 +408,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         mbar_init(&acc_empty[e][b], 128);
       }
     for (int j = 0; j <= spu; ++j) sblk[j] = stage_block(j, ncb, spu);
+    for (int m = 0; m < kMaxFuseM; ++m) xmax_u[m] = 0u;
     mbar_init(&b_full, 1);
     mbar_init(&mma_done[0], 1);
     mbar_init(&mma_done[1], 1);
@@ -158,7 +423,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   __syncthreads();
   tc_fence_after();
   pdl_launch_dependents();
-  if (warp >= kProducers || !p.early) pdl_wait();
+  // (the B operand builders of the fused path wait inside build_b_operand)
+  const bool builder = p.fused && warp >= kExpWarp0 && warp < kEpiWarp0;
+  if (!builder && (warp >= kProducers || !p.early)) pdl_wait();
   const uint32_t tmem = tmem_base;
   bool ok = true;
 
@@ -171,7 +438,11 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       // operand: after its first two stages when the codes may be read before
       // the preceding grid is done, before everything otherwise.
       int last_i = -1;
-      bool b_loaded = warp != 0;
+      bool b_loaded = warp != 0 || p.fused;   // fused: the expanders build it
+      // Fused: the first kFusePre stages go out at once, the rest once the B
+      // operand is built, so that the builders' loads do not queue behind a
+      // full ring of code copies.
+      bool b_ready = !p.fused;
       const int pre = p.early ? min(2 * kProducers, nstages) : 0;
       int u = 0, j = warp;
       while (j >= spu) { j -= spu; ++u; }
@@ -181,6 +452,11 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
           mbar_expect_tx(&b_full, p.b_bytes);
           bulk_g2s(bop, p.bimg + (size_t)kb0 * p.NP * 128, p.b_bytes, &b_full);
           b_loaded = true;
+        }
+        if (!b_ready && i >= kFusePre) {
+          ok = mbar_wait(&b_full, 0);
+          if (!ok) break;
+          b_ready = true;
         }
         const int slot = i % p.ring, r = i / p.ring;
         if (r > 0) ok = mbar_wait(&c_empty[slot], (r - 1) & 1);
@@ -205,7 +481,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         b_loaded = ok;
       }
       // Every copy this thread issued has landed before the CTA may exit.
-      if (warp == 0 && b_loaded && !mbar_wait(&b_full, 0)) ok = false;
+      if (warp == 0 && !p.fused && b_loaded && !mbar_wait(&b_full, 0)) ok = false;
       for (int i = last_i; i >= 0 && i > last_i - p.ring; i -= kProducers)
         if (!mbar_wait(&c_full[i % p.ring], (i / p.ring) & 1)) ok = false;
     }
@@ -273,6 +549,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
     // ------------------------------------------------------------ expanders
     // Set x = 2e + t expands stages i = e + 2t (mod 4) in order: TMEM slot
     // x, ring slots i mod ring (ring is a multiple of 4).
+    if (p.fused) {
+      build_b_operand(p, bop, kb0, ncb, tid - 32 * kExpWarp0, xmax_u, inv_s, scale_s);
+      if (tid == 32 * kExpWarp0) mbar_arrive(&b_full);
+    }
     const int x = (warp - kExpWarp0) >> 2, q = warp & 3, r = 32 * q + lane;
     const int ex = x / kSlots, tx = x - ex * kSlots;
     const uint32_t lane_addr = tmem + ((uint32_t)(32 * q) << 16);
@@ -341,8 +621,13 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
     const int q = warp & 3, r = 32 * q + lane, et = tid - 32 * kEpiWarp0;
     const int NR = p.ntiles * kTileRows;
     const int MT = p.M * p.T;
-    if (et < p.M) scale_s[et] = ldexpf(1.f, p.sexp[et]);
-    named_bar_sync(2, 128);
+    call_record_start(p.rec, p.call, blockIdx.x == 0 && et == 0);
+    if (p.fused) {   // scale_s was written by the B operand builders
+      ok = group_and(2, 128, mbar_wait(&b_full, 0));
+    } else {
+      if (et < p.M) scale_s[et] = ldexpf(1.f, p.sexp[et]);
+      named_bar_sync(2, 128);
+    }
     int kc[2] = {0, 0};
     for (int u = 0; u < nunits && ok; ++u) {
       // issuers with stages in this tile: both, unless the tile is one stage
@@ -402,7 +687,13 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       named_bar_sync(2, 128);
       for (int u0 = 0; u0 < nunits; u0 += 128) {
         const int u = u0 + et;
-        last[et] = u < nunits && atomicAdd(p.cnt + prow + u * p.P, 1u) == (uint32_t)(p.S - 1);
+        bool lt = false;
+        if (u < nunits) {
+          const uint32_t n = ticket_take(p.cnt + prow + u * p.P, p.call);
+          if (n == 0) call_record_fail(p.rec, p.call);
+          lt = n == (uint32_t)p.S;
+        }
+        last[et] = lt;
         named_bar_sync(2, 128);
         __threadfence();
         for (int uu = 0; uu < min(128, nunits - u0); ++uu) {
@@ -428,7 +719,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       }
     }
   }
-  if (!ok) atomicExch(p.err, 1u);
+  if (!ok) call_record_fail(p.rec, p.call);
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {
@@ -498,8 +789,22 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
   return best;
 }
 
+bool decode_fusable(const sdq_plan_s* pl, int M, const uint16_t* x) {
+  const Geometry& g = pl->geo;
+  if (M < 1 || M > kMaxFuseM || (reinterpret_cast<uintptr_t>(x) & 15u)) return false;
+  if (g.block % 16 != 0 || g.n_b % 8 != 0 || !pl->d_g_frag) return false;
+  const DecodeConfig& dc = decode_config(pl, M);
+  if (dc.S < 1) return false;
+  // MMA steps per builder warp for the widest chunk: (m, b) row tiles x code
+  // tiles x 16-deep steps over B, shared by the 16 warps.
+  const int64_t nbi = ((int64_t)dc.CB * kBlk + g.n_b - 1) / g.n_b + 1;
+  const int64_t rt = ((int64_t)M * nbi + 15) / 16;
+  const int64_t steps = rt * (g.n_b / 8) * (g.block / 16) / (kBuildThreads / 32);
+  return steps <= kMaxBuildSteps;
+}
+
 cudaError_t launch_decode(const sdq_plan_s* pl, const uint32_t* codes, const float* alpha, int M,
-                          float* y, void* ws, cudaStream_t st, int early) {
+                          float* y, void* ws, cudaStream_t st, int early, const uint16_t* x) {
   const Geometry& g = pl->geo;
   const DecodeConfig& dc = decode_config(pl, M);
   if (dc.S < 1) return cudaErrorNotSupported;   // the B operand of a k chunk does not fit
@@ -510,8 +815,13 @@ cudaError_t launch_decode(const sdq_plan_s* pl, const uint32_t* codes, const flo
   p.bimg = base + L.bimg;
   p.sexp = reinterpret_cast<const int*>(base + L.sexp);
   p.part = reinterpret_cast<float*>(base + L.part);
-  p.cnt = reinterpret_cast<uint32_t*>(base + L.cnt);
-  p.err = reinterpret_cast<uint32_t*>(base + L.err);
+  p.cnt = reinterpret_cast<uint64_t*>(base + L.cnt);
+  p.rec = reinterpret_cast<uint64_t*>(base + L.err);
+  p.call = next_call_number();
+  p.fused = x != nullptr;
+  p.x = x; p.g_frag = pl->d_g_frag; p.gnorm = pl->gnorm;
+  p.K = g.k_in; p.B = g.block; p.n_b = g.n_b; p.k_eff = g.k_eff;
+  if (p.fused) early = 0;   // x and the codes may come from the preceding grid
   p.M = M; p.T = dc.T; p.NP = dc.NP; p.S = dc.S; p.P = dc.P; p.CB = dc.CB;
   p.KB = (int)(g.k_eff_pad / kBlk); p.ring = dc.ring;
   tmem_split(dc.NP, &p.sb, &p.nbuf, &p.dbase);

@@ -46,7 +46,8 @@ struct PrefillParams {
   const uint32_t* codes;
   const float* alpha;
   float* y;
-  uint32_t* err;
+  uint64_t* rec;       // call record
+  uint64_t call;
   int M, N, ntiles, ngroups, wpg, nks, quantizer;
 };
 
@@ -95,6 +96,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   pdl_wait();
   pdl_launch_dependents();
+  call_record_start(p.rec, p.call, blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0);
   const uint32_t tmem = tmem_base;
   bool ok = true;
 
@@ -203,7 +205,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   }
-  if (!ok) atomicExch(p.err, 1u);
+  if (!ok) call_record_fail(p.rec, p.call);
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {
@@ -247,7 +249,8 @@ cudaError_t launch_prefill(const sdq_plan_s* pl, const uint32_t* codes, const fl
   if (cr != CUDA_SUCCESS) return cudaErrorInvalidValue;
   PrefillParams p;
   p.codes = codes; p.alpha = alpha; p.y = y;
-  p.err = reinterpret_cast<uint32_t*>(wbase + L.err);
+  p.rec = reinterpret_cast<uint64_t*>(wbase + L.err);
+  p.call = next_call_number();
   p.M = M; p.N = g.n_out; p.ntiles = g.ntiles; p.ngroups = g.ngroups; p.wpg = g.wpg;
   p.nks = (int)(g.k_eff_pad / kBK);
   p.quantizer = pl->desc.quantizer;

@@ -29,7 +29,6 @@ struct PrepParams {
   const uint16_t* g_hi;
   const uint16_t* g_lo;
   uint16_t* xtb;      // bf16 M x kpad (permuted)
-  uint32_t* err;      // the workspace error word, zeroed here
   int M, K, B, n_b, nblk;
   int64_t k_eff, kpad;
   int vec, ternary;
@@ -123,13 +122,12 @@ __global__ void __launch_bounds__(128) prep_kernel(PrepParams p) {
         p.xtb[(size_t)m * p.kpad + phys] = float_to_bf16_bits(acc[n][e]);
       }
     }
-  // Zero the K padding of this batch row, and the error word.
+  // Zero the K padding of this batch row.
   if (jt == 0 && bt == 0) {
     for (int64_t k = p.k_eff + tid; k < p.kpad; k += 128) {
       const int64_t phys = (k & ~int64_t(63)) | prefill_pos64((int)(k & 63), p.ternary);
       p.xtb[(size_t)m * p.kpad + phys] = 0;
     }
-    if (m == 0 && tid == 0) *p.err = 0u;
   }
 }
 
@@ -156,25 +154,22 @@ struct DecPrepParams {
   float* xt;          // M x kpad fp32
   uint8_t* bimg;      // e4m3 B operand image
   int* sexp;          // e_m per batch row
-  uint32_t* cnt;      // decode tickets and error word to zero
-  int ncnt;
   float gnorm;
   int M, K, B, n_b, nblk, T, NP, kc, ternary, vec;
   int64_t k_eff, kpad;
 };
 
-// MMA K position (within a 128-code block) of natural code kl: the inverse of
-// decode_stage_k.
-__device__ __forceinline__ int decode_pos(int kl, bool ternary) {
-  if (ternary) {
-    const int f = kl & 15;
-    return (kl & ~15) + 4 * (3 - (f & 3)) + (f >> 2);
-  }
-  const int f = kl & 31;
-  return (kl & ~31) + 4 * (7 - (f & 7)) + (f >> 3);
-}
-
 __device__ __forceinline__ float bf16_abs(uint32_t h) { return __uint_as_float((h & 0x7FFFu) << 16); }
+
+// 16-byte global -> shared copy that does not pass through registers; `bytes`
+// = 0 fills the destination with zeros.
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, uint32_t bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n"
+               :: "r"(smem_u32(dst)), "l"(src), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;\n" ::: "memory");
+}
 
 __global__ void __launch_bounds__(128) prep_decode_kernel(DecPrepParams p) {
   constexpr int TB = 16, NTW = 2;   // 16 blocks x 64 j per CTA; warp w owns j 16w .. 16w + 15
@@ -192,42 +187,26 @@ __global__ void __launch_bounds__(128) prep_decode_kernel(DecPrepParams p) {
   const int b0 = bt * TB, j0 = jt * 64, wcol = warp * 16;
   const uint16_t* xr = p.x + (size_t)m * p.K;
 
-  // max |x[m, :]| (loads issued before the tile loads)
-  float xmax = 0.f;
-  if (p.vec) {
-    for (int i = tid; i < p.K / 8; i += 128) {
-      const uint4 v = *reinterpret_cast<const uint4*>(xr + 8 * i);
-      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-      for (int q = 0; q < 4; ++q) xmax = fmaxf(xmax, fmaxf(bf16_abs(w[q]), bf16_abs(w[q] >> 16)));
-    }
-  } else {
-    for (int i = tid; i < p.K; i += 128) xmax = fmaxf(xmax, bf16_abs(xr[i]));
-  }
-
   float acc[NTW][4];
 #pragma unroll
   for (int n = 0; n < NTW; ++n)
 #pragma unroll
     for (int e = 0; e < 4; ++e) acc[n][e] = 0.f;
+  float xmax = 0.f;
   for (int kc0 = 0; kc0 < p.B; kc0 += p.kc) {
-    if (p.vec) {   // B % 32 == 0, rows 16-byte aligned
+    if (p.vec) {   // B % 32 == 0, rows 16-byte aligned: asynchronous 16-byte copies
       const int q8 = p.kc / 8;
       for (int i = tid; i < TB * q8; i += 128) {
         const int rr = i / q8, q = i - rr * q8, b = b0 + rr;
-        uint4 v = make_uint4(0, 0, 0, 0);
-        if (b < p.nblk) v = *reinterpret_cast<const uint4*>(xr + (size_t)b * p.B + kc0 + 8 * q);
-        *reinterpret_cast<uint4*>(xs + rr * ld + 8 * q) = v;
+        const bool v = b < p.nblk;
+        cp_async16(xs + rr * ld + 8 * q, v ? xr + (size_t)b * p.B + kc0 + 8 * q : xr, v ? 16u : 0u);
       }
       for (int i = tid; i < 64 * q8; i += 128) {
         const int rr = i / q8, q = i - rr * q8, j = j0 + rr;
-        uint4 vh = make_uint4(0, 0, 0, 0), vl = vh;
-        if (j < p.n_b) {
-          vh = *reinterpret_cast<const uint4*>(p.g_hi + (size_t)j * p.B + kc0 + 8 * q);
-          vl = *reinterpret_cast<const uint4*>(p.g_lo + (size_t)j * p.B + kc0 + 8 * q);
-        }
-        *reinterpret_cast<uint4*>(ghs + rr * ld + 8 * q) = vh;
-        *reinterpret_cast<uint4*>(gls + rr * ld + 8 * q) = vl;
+        const bool v = j < p.n_b;
+        const size_t off = v ? (size_t)j * p.B + kc0 + 8 * q : 0;
+        cp_async16(ghs + rr * ld + 8 * q, p.g_hi + off, v ? 16u : 0u);
+        cp_async16(gls + rr * ld + 8 * q, p.g_lo + off, v ? 16u : 0u);
       }
     } else {
       for (int i = tid; i < TB * p.kc; i += 128) {
@@ -241,6 +220,30 @@ __global__ void __launch_bounds__(128) prep_decode_kernel(DecPrepParams p) {
         gls[rr * ld + kk] = gv ? p.g_lo[(size_t)j * p.B + k] : 0;
       }
     }
+    if (kc0 == 0) {
+      // max |x[m, :]| while the tile copies are in flight; 8 independent
+      // 16-byte loads per thread at a time.
+      if (p.vec) {
+        const int nv = p.K / 8;
+        for (int i0 = tid; i0 < nv; i0 += 128 * 8) {
+          uint4 v[8];
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const int i = i0 + 128 * u;
+            v[u] = i < nv ? __ldg(reinterpret_cast<const uint4*>(xr) + i) : make_uint4(0, 0, 0, 0);
+          }
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const uint32_t w[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+#pragma unroll
+            for (int q = 0; q < 4; ++q) xmax = fmaxf(xmax, fmaxf(bf16_abs(w[q]), bf16_abs(w[q] >> 16)));
+          }
+        }
+      } else {
+        for (int i = tid; i < p.K; i += 128) xmax = fmaxf(xmax, bf16_abs(xr[i]));
+      }
+    }
+    if (p.vec) cp_async_wait_all();
     __syncthreads();
     for (int ks = 0; ks < p.kc; ks += 16) {
       uint32_t a[4];
@@ -299,8 +302,7 @@ __global__ void __launch_bounds__(128) prep_decode_kernel(DecPrepParams p) {
         }
       }
     }
-  // K padding of this batch row (x_tilde and its terms are 0 there), and the
-  // decode tickets and error word.
+  // K padding of this batch row (x_tilde and its terms are 0 there).
   if (jt == 0 && bt == 0) {
     for (int64_t k = p.k_eff + tid; k < p.kpad; k += 128) {
       p.xt[(size_t)m * p.kpad + k] = 0.f;
@@ -311,8 +313,6 @@ __global__ void __launch_bounds__(128) prep_decode_kernel(DecPrepParams p) {
         blk[row * 128 + (((kap >> 4) ^ (row & 7)) << 4) + (kap & 15)] = 0;
       }
     }
-    if (m == 0 && p.cnt)
-      for (int i = tid; i < p.ncnt; i += 128) p.cnt[i] = 0u;
   }
 }
 
@@ -330,8 +330,6 @@ cudaError_t launch_prep(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws
     p.xt = reinterpret_cast<float*>(base + L.xt);
     p.bimg = base + L.bimg;
     p.sexp = reinterpret_cast<int*>(base + L.sexp);
-    p.cnt = reinterpret_cast<uint32_t*>(base + L.cnt);
-    p.ncnt = g.ntiles + 1;   // the tile tickets and the error word that follows them
     p.gnorm = pl->gnorm;
     p.M = M; p.K = g.k_in; p.B = g.block; p.n_b = g.n_b; p.nblk = g.nblk;
     p.T = dc.T; p.NP = dc.NP;
@@ -354,7 +352,6 @@ cudaError_t launch_prep(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws
   p.vec = vec;
   const bool small = (int64_t)M * g.nblk < 4 * (int64_t)pl->sm_count;
   const int TB = small ? 16 : 64;
-  p.err = reinterpret_cast<uint32_t*>(base + L.err);
   dim3 grid((g.n_b + 63) / 64, (g.nblk + TB - 1) / TB, M);
   return small ? launch_pdl(prep_kernel<16>, grid, dim3(128), 0, st, p)
                : launch_pdl(prep_kernel<64>, grid, dim3(128), 0, st, p);

@@ -38,6 +38,19 @@ constexpr int kMaxDecodeM = 64;
 // with N up to 64 columns (M * T), so small batches take more terms.
 inline int decode_terms(int M) { return M <= 16 ? 4 : (M <= 21 ? 3 : 2); }
 
+// G in the order the decode kernel's B-operand builders load it (only when
+// B % 16 == 0 and n_b % 8 == 0): for code tile jt (rows j = 8 jt .. 8 jt + 7),
+// k batch kb of kbw = min(64, B) inputs and lane (g, t) of the warp MMA, the
+// run of R = kbw / 4 inputs i = kb kbw + t R + e (e < R) of row j = 8 jt + g
+// at element 2 R (32 (jt (B / kbw) + kb) + lane), as 32-bit words that
+// alternate a hi pair (inputs e, e + 1) and the lo pair of the same inputs.
+// Within the batch, input t R + 4 s + r is MMA K index 2t + (r & 1) + 8 (r >> 1)
+// of 16-deep step s, so that each lane's fragments are one contiguous run.
+#ifdef __CUDACC__
+__host__ __device__
+#endif
+inline int g_frag_batch(int B) { return B < 64 ? B : 64; }
+
 // Launch shape of the decode kernel for one batch size (chosen at plan time).
 // Grid = S * P CTAs, one per SM: CTA (s, p) contracts k chunk s (CB blocks
 // of 128 codes) against row tiles p, p + P, p + 2P, ...
@@ -59,5 +72,6 @@ struct sdq_plan_s {
   float* d_at;         // encode table, transposed: B x n_b (At[k][j] = A_enc[j][k])
   uint16_t* d_g_hi;    // G as bf16 hi part, n_b x B row-major
   uint16_t* d_g_lo;    // G - hi as bf16, n_b x B row-major
+  uint16_t* d_g_frag;  // G hi + lo in warp-fragment order (g_frag_index), or null
   sdq::DecodeConfig dcfg[sdq::kMaxDecodeM + 1];  // decode launch shape per batch size
 };
