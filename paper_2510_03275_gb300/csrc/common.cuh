@@ -258,16 +258,19 @@ __device__ __forceinline__ void call_record_fail(uint64_t* rec, uint64_t call) {
 
 // Split-K ticket of one row tile: bits 8..63 the call number, bits 0..7 the
 // arrivals of that call.  A ticket that carries another call number counts
-// as empty, so tickets need no reset between calls.  Returns this CTA's
-// arrival number (1..255), or 0 if the compare-and-swap did not settle within
-// its retry bound.
+// as empty, so tickets need no reset between calls: the first arrival of a
+// call installs (call, 1) by compare-and-swap, later ones add 1 (a ticket
+// that carries this call's number keeps it for the rest of the call).
+// Returns this CTA's arrival number (1..255), or 0 if the compare-and-swap
+// did not settle within its retry bound.
 __device__ __forceinline__ uint32_t ticket_take(uint64_t* tk, uint64_t call) {
   unsigned long long* p = reinterpret_cast<unsigned long long*>(tk);
+  const unsigned long long mine = (unsigned long long)call << 8;
   unsigned long long cur = *reinterpret_cast<volatile unsigned long long*>(p);
-  for (int it = 0; it < (1 << 20); ++it) {
-    const unsigned long long base = (cur >> 8) == call ? cur : ((unsigned long long)call << 8);
-    const unsigned long long prev = atomicCAS(p, cur, base + 1);
-    if (prev == cur) return (uint32_t)((base & 0xFFu) + 1);
+  for (int it = 0; it < 64; ++it) {
+    if ((cur >> 8) == call) return (uint32_t)((atomicAdd(p, 1ull) & 0xFFu) + 1);
+    const unsigned long long prev = atomicCAS(p, cur, mine + 1);
+    if (prev == cur) return 1;
     cur = prev;
   }
   return 0;

@@ -14,9 +14,11 @@
 //             row's packed words (no shared-memory round trip)
 //   B (smem)  the activations as T e4m3 terms per batch row m:
 //             x_tilde[m] * 2^-e_m = sum_t 16^-t q_t[m] (e_m from a bound on |x_tilde[m]|),
-//             N = M*T rows rounded up to 16, K-major, 128-byte swizzle,
-//             written for all of K by the decode prepare kernel; each CTA
-//             copies the part of its k chunk once
+//             N = M*T rows rounded up to 16, K-major, 128-byte swizzle:
+//             either written for all of K by the decode prepare kernel, each
+//             CTA copying the part of its k chunk once, or (small batches,
+//             `fused`) built by the CTA's expander warps for its k chunk from
+//             x itself, with a scale 2^e_m of its own (build_b_operand)
 //   D (TMEM)  fp32, 128 lanes x NP columns
 // so that y[m, r] = alpha_r / 2 * 2^e_m * sum_t 16^-t D[r, m T + t].
 //
@@ -43,14 +45,15 @@
 //                 TMEM lane quadrant) expands stages i = e + 2t (mod 4) into
 //                 TMEM slot x
 //   warps 20..23  epilogue: read and add the accumulators, combine the
-//                 terms, scale and store y, or store a split-K partial; after
-//                 the CTA's last tile, one fence and one ticket per tile, and
-//                 the last CTA of each tile sums its S partials in a fixed
-//                 order (deterministic)
+//                 terms, scale and store y, or store a split-K partial, fence
+//                 it and take the tile's ticket while the next tile's MMAs
+//                 run; the CTA with the last ticket of a tile sums its S
+//                 partials in a fixed order (deterministic)
 // With `early` set the producers start the code stream before waiting for
 // the preceding grid (codes are never written by the prep kernels).
-// Every mbarrier wait is bounded (about 2 s); a timeout sets the workspace
-// error word and the CTA drains its copies and MMAs before freeing TMEM.
+// Every mbarrier wait is bounded (about 2 s); a timeout writes the call
+// number into the workspace's call record and the CTA drains its copies and
+// MMAs before freeing TMEM.
 #include <algorithm>
 #include <cmath>
 
@@ -77,6 +80,7 @@ constexpr int kMaxFuseM = 4;                     // batch rows of the fused B op
 constexpr int kBuildThreads = 32 * 4 * kExpSets; // the expander warps build it
 constexpr int kMaxBuildSteps = 64;               // 16-deep MMA steps per warp (fusion bound)
 constexpr int kFusePre = 4;                      // code stages requested before the B operand is built
+constexpr int kRedWords = 64;                    // split-K sums summed CTA-wide: first 2048 tiles
 
 struct DecodeParams {
   const uint32_t* codes;
@@ -375,7 +379,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   __shared__ __align__(8) uint64_t a_full[2 * kSlots], a_empty[2 * kSlots];
   __shared__ __align__(8) uint64_t acc_full[2][2], acc_empty[2][2], b_full, mma_done[2];
   __shared__ uint32_t tmem_base;
-  __shared__ int last[128];
+  __shared__ int last[1];
+  __shared__ uint32_t red_bits[kRedWords];  // tiles whose split-K sum this CTA owes (all threads sum)
   __shared__ float scale_s[kMaxDecodeM];   // 2^e_m
   __shared__ float inv_s[kMaxFuseM];       // 2^-e_m (fused B operand)
   __shared__ uint32_t xmax_u[kMaxFuseM];   // max |x[m]| bits (fused B operand)
@@ -387,6 +392,12 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   const int ncb = min(p.CB, p.KB - kb0);                        // blocks of this chunk
   const int spu = max((ncb + p.sb - 1) / p.sb, min(2, ncb));   // stages per tile
   const int nunits = (p.ntiles - prow + p.P - 1) / p.P;         // row tiles of this CTA
+  // The CTAs of a row set (one per k chunk) walk its tiles in rotated orders,
+  // so that a different CTA finishes (and sums the split-K partials of) each
+  // tile: unit u is tile prow + ((u + rot) mod nunits) P.
+  // (Single-row sums, M = 1, done at once per tile, keep the plain order.)
+  const bool red_now = p.M == 1;
+  const int rot = red_now ? 0 : (int)(((int64_t)sidx * ((nunits + p.S - 1) / p.S)) % max(nunits, 1));
   const int nstages = nunits * spu;
   const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
   uint8_t* base = smem_raw + (sbase - smem_u32(smem_raw));
@@ -409,6 +420,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       }
     for (int j = 0; j <= spu; ++j) sblk[j] = stage_block(j, ncb, spu);
     for (int m = 0; m < kMaxFuseM; ++m) xmax_u[m] = 0u;
+    for (int w = 0; w < kRedWords; ++w) red_bits[w] = 0u;
     mbar_init(&b_full, 1);
     mbar_init(&mma_done[0], 1);
     mbar_init(&mma_done[1], 1);
@@ -462,7 +474,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         if (r > 0) ok = mbar_wait(&c_empty[slot], (r - 1) & 1);
         if (!ok) break;
         const int b0 = sblk[j], b1 = sblk[j + 1];
-        const int tile = prow + u * p.P;
+        const int tile = prow + (u + rot < nunits ? u + rot : u + rot - nunits) * p.P;
         const uint8_t* src = reinterpret_cast<const uint8_t*>(p.codes) +
                              ((size_t)tile * p.KB + kb0 + b0) * p.blk_bytes;
         const uint32_t bytes = (uint32_t)(b1 - b0) * p.blk_bytes;
@@ -621,6 +633,26 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
     const int q = warp & 3, r = 32 * q + lane, et = tid - 32 * kEpiWarp0;
     const int NR = p.ntiles * kTileRows;
     const int MT = p.M * p.T;
+    // a split-K sum costs M x ceil(S / 16) rounds of 16 loads per thread
+    auto reduce_tile = [&](int ut) {
+      const int row = (prow + ut * p.P) * kTileRows + r;
+      if (row >= p.n_out) return;
+      const float sa = 0.5f * __ldg(p.alpha + row);
+      const size_t sstride = (size_t)p.M * NR;
+      for (int mm = 0; mm < p.M; ++mm) {
+        const float* pr = p.part + (size_t)mm * NR + row;
+        float s0 = 0.f;
+        for (int k0 = 0; k0 < p.S; k0 += 16) {   // 16 loads in flight, summed in chunk order
+          float a[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) a[i] = k0 + i < p.S ? __ldcg(pr + (size_t)(k0 + i) * sstride) : 0.f;
+#pragma unroll
+          for (int i = 0; i < 16; ++i)
+            if (k0 + i < p.S) s0 += a[i];
+        }
+        p.y[(size_t)mm * p.n_out + row] = sa * s0;
+      }
+    };
     call_record_start(p.rec, p.call, blockIdx.x == 0 && et == 0);
     if (p.fused) {   // scale_s was written by the B operand builders
       ok = group_and(2, 128, mbar_wait(&b_full, 0));
@@ -640,7 +672,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       ok = group_and(2, 128, w);
       if (!ok) break;
       tc_fence_after();
-      const int row = (prow + u * p.P) * kTileRows + r;
+      const int ut = u + rot < nunits ? u + rot : u + rot - nunits;   // unit of this tile
+      const int row = (prow + ut * p.P) * kTileRows + r;
       const bool live = row < p.n_out;
       const float sa = live ? 0.5f * __ldg(p.alpha + row) : 0.f;
       const uint32_t lq = tmem + ((uint32_t)(32 * q) << 16);
@@ -678,50 +711,64 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       }
       kc[0] += in0;
       kc[1] += in1;
-    }
-    if (p.S > 1 && ok) {
-      // Split-K: one fence for all of this CTA's partials, then one ticket
-      // per tile; the CTA that takes the last ticket of a tile sums its S
-      // partials in k-chunk order.
-      __threadfence();
-      named_bar_sync(2, 128);
-      for (int u0 = 0; u0 < nunits; u0 += 128) {
-        const int u = u0 + et;
-        bool lt = false;
-        if (u < nunits) {
-          const uint32_t n = ticket_take(p.cnt + prow + u * p.P, p.call);
+      if (p.S > 1) {
+        // Split-K, per tile while the next tile's MMAs run: one thread fences
+        // (after the barrier that orders the other threads' partial stores
+        // before it) and takes the tile's ticket; the CTA with the last ticket
+        // sums the S partials in k-chunk order (deterministic): at once when
+        // that is one round of loads per thread, else after the main loop on
+        // all of the CTA's threads (the tiles a CTA finishes last come at the
+        // end of its rotated order).
+        named_bar_sync(2, 128);
+        if (et == 0) {
+          __threadfence();
+          const uint32_t n = ticket_take(p.cnt + prow + ut * p.P, p.call);
           if (n == 0) call_record_fail(p.rec, p.call);
-          lt = n == (uint32_t)p.S;
-        }
-        last[et] = lt;
-        named_bar_sync(2, 128);
-        __threadfence();
-        for (int uu = 0; uu < min(128, nunits - u0); ++uu) {
-          if (!last[uu]) continue;
-          const int row = (prow + (u0 + uu) * p.P) * kTileRows + r;
-          if (row >= p.n_out) continue;
-          const float sa = 0.5f * __ldg(p.alpha + row);
-          const size_t sstride = (size_t)p.M * NR;
-          for (int mm = 0; mm < p.M; ++mm) {
-            const float* pr = p.part + (size_t)mm * NR + row;
-            float s0 = 0.f;
-            int kk = 0;
-            for (; kk + 4 <= p.S; kk += 4) {
-              const float a0 = __ldcg(pr + (size_t)kk * sstride), a1 = __ldcg(pr + (size_t)(kk + 1) * sstride);
-              const float a2 = __ldcg(pr + (size_t)(kk + 2) * sstride), a3 = __ldcg(pr + (size_t)(kk + 3) * sstride);
-              s0 = (((s0 + a0) + a1) + a2) + a3;
-            }
-            for (; kk < p.S; ++kk) s0 += __ldcg(pr + (size_t)kk * sstride);
-            p.y[(size_t)mm * p.n_out + row] = sa * s0;
-          }
+          const bool won = n == (uint32_t)p.S;
+          if (won) __threadfence();
+          const bool defer = won && !red_now && ut < 32 * kRedWords;
+          if (defer) red_bits[ut >> 5] |= 1u << (ut & 31);
+          last[0] = won && !defer;
         }
         named_bar_sync(2, 128);
+        if (last[0]) reduce_tile(ut);
       }
     }
   }
   if (!ok) call_record_fail(p.rec, p.call);
   tc_fence_before();
   __syncthreads();
+  // Split-K sums won in the end-of-kernel ticket burst, by every thread of the
+  // CTA: (m, row) pairs, consecutive threads on consecutive rows; each pair
+  // adds its S partials in k-chunk order (deterministic) with 16 loads in
+  // flight.
+  if (p.S > 1 && ok && !red_now) {
+    const int NR = p.ntiles * kTileRows;
+    const size_t sstride = (size_t)p.M * NR;
+    for (int w = 0; w < kRedWords; ++w) {
+      uint32_t bits = red_bits[w];
+      while (bits) {
+        const int u = 32 * w + __ffs(bits) - 1;
+        bits &= bits - 1;
+        const int row0 = (prow + u * p.P) * kTileRows;
+        for (int i = tid; i < kTileRows * p.M; i += kThreads) {
+          const int mm = i / kTileRows, row = row0 + (i - mm * kTileRows);
+          if (row >= p.n_out) continue;
+          const float* pr = p.part + (size_t)mm * NR + row;
+          float s0 = 0.f;
+          for (int k0 = 0; k0 < p.S; k0 += 16) {
+            float a[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) a[j] = k0 + j < p.S ? __ldcg(pr + (size_t)(k0 + j) * sstride) : 0.f;
+#pragma unroll
+            for (int j = 0; j < 16; ++j)
+              if (k0 + j < p.S) s0 += a[j];
+          }
+          p.y[(size_t)mm * p.n_out + row] = 0.5f * __ldg(p.alpha + row) * s0;
+        }
+      }
+    }
+  }
   if (warp == 0) {
     __syncwarp();   // warp-collective: lane 0 ran the producer loop alone
     tc_fence_after();
@@ -758,7 +805,7 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
   tmem_split(best.NP, &sb, &nbuf, &dbase);
   const int slot_bytes = sb * blk_bytes;
   const double clk = 1.9e9, bw = 6.5e12, latency = 2.2e-6;   // loaded HBM latency
-  const double t_mma = std::max(38.0, best.NP * 0.4) / clk;     // per MMA, two issuers
+  const double t_mma = std::max(38.0, best.NP * 0.55) / clk;    // per MMA, two issuers
   const double code_bytes = (double)g.ntiles * kTileRows * g.k_eff_pad * g.bits / 8;
   double best_t = 1e30;
   for (int S = 1; S <= std::min(KB, sms); ++S) {
@@ -776,7 +823,16 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
       const double inflight = (double)grid * ring * slot_bytes;
       const double bw_eff = std::min(bw, inflight / latency);
       const double part_bytes = S > 1 ? 8.0 * S * M * g.ntiles * kTileRows : 0.0;
-      const double tail = S > 1 ? 2.5e-6 + (double)M * S * kTileRows * 4 / 40e9 : 0.0;
+      // split-K: the CTA that sums a tile reads S partials for each of its
+      // 128 M (m, row) pairs, in rounds of 16 loads (~1.2 us a round).  M = 1:
+      // summed per tile by the epilogue while MMAs go on (within the fixed
+      // split-K tail below).  Else M x 128 / 768 pairs per thread of the whole
+      // CTA after the main loop, about units / S tiles per CTA (rotated tile
+      // orders).
+      const bool now = M == 1;
+      const int rounds = (kTileRows * M + kThreads - 1) / kThreads * ((S + 15) / 16);
+      const double red = S <= 1 || now ? 0.0 : (double)((units + S - 1) / S) * rounds * 1.2e-6;
+      const double tail = S > 1 ? 2.5e-6 + red : 0.0;
       const double t_cta = units * (4.0 * CB * t_mma + spu * 90.0 / clk + 300.0 / clk);
       const double t = std::max(t_cta, (code_bytes + part_bytes) / bw_eff) + tail;
       if (t < best_t * 0.999) {
