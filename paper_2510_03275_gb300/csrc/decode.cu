@@ -81,6 +81,8 @@ constexpr int kBuildThreads = 32 * 4 * kExpSets; // the expander warps build it
 constexpr int kMaxBuildSteps = 64;               // 16-deep MMA steps per warp (fusion bound)
 constexpr int kFusePre = 4;                      // code stages requested before the B operand is built
 constexpr int kRedWords = 64;                    // split-K sums summed CTA-wide: first 2048 tiles
+static_assert(kMaxRing <= 32 && 2 * kSlots + 7 <= 16 && kRedWords == 64 && kMaxSpu < 160,
+              "the prologue's per-warp set-up assumes these bounds");
 
 struct DecodeParams {
   const uint32_t* codes;
@@ -404,28 +406,32 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   uint8_t* bop = base;                                          // ncb x NP x 128 bytes
   uint8_t* ring = base + p.b_bytes;                             // ring x slot_bytes
 
-  if (tid == 0) {
-    for (int i = 0; i < p.ring; ++i) {
-      mbar_init(&c_full[i], 1);
-      mbar_init(&c_empty[i], 4);     // one arrival per expander warp
+  // Set-up spread over warps 1.. (warp 0 allocates TMEM meanwhile).
+  if (warp == 1 && lane < p.ring) {
+    mbar_init(&c_full[lane], 1);
+    mbar_init(&c_empty[lane], 4);   // one arrival per expander warp
+  } else if (warp == 2) {
+    if (lane < 2 * kSlots) {
+      mbar_init(&a_full[lane], 4);
+      mbar_init(&a_empty[lane], 1);
+    } else if (lane < 2 * kSlots + 4) {
+      const int e = (lane - 2 * kSlots) >> 1, b = lane & 1;
+      mbar_init(&acc_full[e][b], 1);
+      mbar_init(&acc_empty[e][b], 128);
+    } else if (lane == 2 * kSlots + 4) {
+      mbar_init(&b_full, 1);
+    } else if (lane == 2 * kSlots + 5 || lane == 2 * kSlots + 6) {
+      mbar_init(&mma_done[lane - 2 * kSlots - 5], 1);
+    } else if (lane >= 16 && lane < 16 + kMaxFuseM) {
+      xmax_u[lane - 16] = 0u;
     }
-    for (int i = 0; i < 2 * kSlots; ++i) {
-      mbar_init(&a_full[i], 4);
-      mbar_init(&a_empty[i], 1);
-    }
-    for (int e = 0; e < 2; ++e)
-      for (int b = 0; b < 2; ++b) {
-        mbar_init(&acc_full[e][b], 1);
-        mbar_init(&acc_empty[e][b], 128);
-      }
-    for (int j = 0; j <= spu; ++j) sblk[j] = stage_block(j, ncb, spu);
-    for (int m = 0; m < kMaxFuseM; ++m) xmax_u[m] = 0u;
-    for (int w = 0; w < kRedWords; ++w) red_bits[w] = 0u;
-    mbar_init(&b_full, 1);
-    mbar_init(&mma_done[0], 1);
-    mbar_init(&mma_done[1], 1);
-    fence_mbar_init();
+  } else if (warp >= 3 && warp < 3 + (kMaxSpu + 32) / 32) {
+    const int j = tid - 96;
+    if (j <= spu) sblk[j] = stage_block(j, ncb, spu);
+  } else if (warp >= 8 && warp < 10) {
+    red_bits[tid - 256] = 0u;
   }
+  if (warp == 1 || warp == 2) fence_mbar_init();
   if (warp == 0) {
     __syncwarp();
     tmem_alloc(&tmem_base, 512);
