@@ -226,9 +226,9 @@ int sdq_read_prep(sdq_plan plan, int32_t M, const void* ws, float* xt_out, void*
  *     (cudaGetSymbolAddress, with that device current); make that first call
  *     before any stream capture.
  *   - All calls on a device share the array and it keeps the last call's
- *     contents; each call's prepare kernel re-zeroes what must start at
- *     zero.  Calls that overlap on the GPU (other streams or host threads)
- *     race on the array: serialize them.
+ *     contents, none of which needs resetting (see sdq_workspace_status).
+ *     Calls that overlap on the GPU (other streams or host threads) race on
+ *     the array: serialize them.
  *   - sdq_workspace_status is not available for these calls. */
 int sdq_linear_forward_noalloc(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha,
                                const uint16_t* x, int32_t M, float* y, void* stream);

@@ -4,16 +4,16 @@
 // a host runtime that owns every device allocation through its own pool
 // (and forbids cudaMalloc from third-party code), or a serving loop that
 // must not allocate device memory once it has started.  For them this file
-// keeps the decode scratch (x_tilde, the bf16 operand fragments, split-K
-// partials, counters and the error word) in one file-scope device array of
-// kNoAllocScratchBytes per GPU, reserved when the library is loaded and held
-// until the process exits.
+// keeps the decode scratch (x_tilde and the fp8 B operand of the two-kernel
+// route, split-K partials, tickets and the call record) in one file-scope
+// device array of kNoAllocScratchBytes per GPU, reserved when the library is
+// loaded and held until the process exits.
 //
 // The array is shared by every call on a device and keeps whatever the last
-// call left in it; the prepare kernel of each call zeroes the counters and
-// the error word before the contraction reads them, and everything else is
-// written before it is read.  Two calls that overlap on the GPU (different
-// streams, or different host threads) race on the array.
+// call left in it: tickets and the call record carry a process-wide call
+// number, so stale contents never count, and everything else is written
+// before it is read.  Two calls that overlap on the GPU (different streams,
+// or different host threads) race on the array.
 #include <mutex>
 
 #include "common.cuh"

@@ -21,8 +21,9 @@
 //               yields the codes in the permuted order the prep kernel also
 //               uses for A), then read the fp32 accumulator out of TMEM
 //               (tcgen05.ld), scale by alpha / 2 and store y.
-// Every wait on an mbarrier is bounded (about 2 s); a timeout sets the
-// workspace error word and the CTA finishes without further waits.
+// Every wait on an mbarrier is bounded (about 2 s); a timeout writes the call
+// number into the workspace's call record and the CTA finishes without
+// further waits.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
