@@ -192,6 +192,17 @@ __device__ __forceinline__ void mma_batch(const BuildGeo& q, const uint32_t (&xw
       mma_bf16_16816(acc[1], a, gw[4 * s + 1], gw[4 * s + 3]);
     }
 }
+// One accumulator (hi and lo parts of G alternate into it).
+__device__ __forceinline__ void mma_batch1(const BuildGeo& q, const uint32_t (&xw)[2][8], const uint32_t (&gw)[16],
+                                           float (&acc)[4]) {
+#pragma unroll
+  for (int s = 0; s < 4; ++s)
+    if (s < q.S4) {
+      const uint32_t a[4] = {xw[0][2 * s], xw[1][2 * s], xw[0][2 * s + 1], xw[1][2 * s + 1]};
+      mma_bf16_16816(acc, a, gw[4 * s], gw[4 * s + 2]);
+      mma_bf16_16816(acc, a, gw[4 * s + 1], gw[4 * s + 3]);
+    }
+}
 __device__ __forceinline__ void acc_sum(const float (&a)[2][4], float (&out)[4]) {
 #pragma unroll
   for (int e = 0; e < 4; ++e) out[e] = a[0][e] + a[1][e];
@@ -274,14 +285,17 @@ __device__ void build_b_operand(const DecodeParams& p, uint8_t* bop, int kb0, in
     const uint16_t* xa1 = p.x + t * q.R + (v1 ? (size_t)m1 * p.K + (size_t)(q.blo + g + 8 - m1 * q.nbi) * p.B : 0);
     uint32_t mx0 = 0u, mx1 = 0u;   // max |x| bits of rows g, g + 8
     float inv0 = 1.f, inv1 = 1.f;
-    for (int jt = ew; jt < JT; jt += NW) {
-      const bool first = jt == ew;
-      float acc4[2][4] = {};
+    // A warp takes two adjacent code tiles per pass over x (one x load
+    // feeds both), so that 16 warps cover 32 tiles (n_b = 256) in one item.
+    for (int jt = 2 * ew; jt < JT; jt += 2 * NW) {
+      const bool first = jt == 2 * ew, two = jt + 1 < JT;
+      float acc0[4] = {0.f, 0.f, 0.f, 0.f}, acc1[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int kb = 0; kb < 2; ++kb)
         if (kb < q.nkb) {
-          uint32_t xw[2][8], gw[16];
-          load_g_frags(p, q, jt, kb, lane, gw);
+          uint32_t xw[2][8], gw0[16], gw1[16];
+          load_g_frags(p, q, jt, kb, lane, gw0);
+          if (two) load_g_frags(p, q, jt + 1, kb, lane, gw1);
           load_x_frags(q, xa0, xa1, kb, xw);   // (again for later tiles: an L1 hit)
           if (first)
 #pragma unroll
@@ -289,10 +303,9 @@ __device__ void build_b_operand(const DecodeParams& p, uint8_t* bop, int kb0, in
               mx0 = bf16x2_absmax_bits(xw[0][w], mx0);
               mx1 = bf16x2_absmax_bits(xw[1][w], mx1);
             }
-          mma_batch(q, xw, gw, acc4);
+          mma_batch1(q, xw, gw0, acc0);
+          if (two) mma_batch1(q, xw, gw1, acc1);
         }
-      float acc[4];
-      acc_sum(acc4, acc);
       if (first) {   // max |x[m]| over the warp's fragments = over the whole chunk
 #pragma unroll
         for (int mm = 0; mm < kMaxFuseM; ++mm) {
@@ -306,7 +319,8 @@ __device__ void build_b_operand(const DecodeParams& p, uint8_t* bop, int kb0, in
           if (et == mm) scale_s[mm] = ldexpf(1.f, e);
         }
       }
-      write_terms(p, q, bop, jt, t, g, g + 8, m0, m1, inv0, inv1, acc);
+      write_terms(p, q, bop, jt, t, g, g + 8, m0, m1, inv0, inv1, acc0);
+      if (two) write_terms(p, q, bop, jt + 1, t, g, g + 8, m0, m1, inv0, inv1, acc1);
     }
   } else {
     pdl_wait();
@@ -464,6 +478,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       const int pre = p.early ? min(2 * kProducers, nstages) : 0;
       int u = 0, j = warp;
       while (j >= spu) { j -= spu; ++u; }
+      const uint64_t pol = l2_policy_evict_first();   // codes are read once per call
       for (int i = warp; i < nstages && ok; i += kProducers) {
         if (!b_loaded && i >= pre) {
           if (p.early) pdl_wait();
@@ -485,7 +500,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
                              ((size_t)tile * p.KB + kb0 + b0) * p.blk_bytes;
         const uint32_t bytes = (uint32_t)(b1 - b0) * p.blk_bytes;
         mbar_expect_tx(&c_full[slot], bytes);
-        bulk_g2s(ring + (size_t)slot * p.slot_bytes, src, bytes, &c_full[slot]);
+        bulk_g2s_hint(ring + (size_t)slot * p.slot_bytes, src, bytes, &c_full[slot], pol);
         last_i = i;
         j += kProducers;
         while (j >= spu) { j -= spu; ++u; }
