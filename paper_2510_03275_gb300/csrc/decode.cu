@@ -213,11 +213,15 @@ __device__ __forceinline__ uint32_t bf16x2_absmax_bits(uint32_t w, uint32_t cur)
   return max(cur, max(w & 0x7FFF0000u, (w << 16) & 0x7FFF0000u));
 }
 
-// T e4m3 terms of the lane's four x_tilde values of tile (rows r0, r1; codes 8 jt ..).
-template <int T>
-__device__ __forceinline__ void write_terms_t(const DecodeParams& p, const BuildGeo& q, uint8_t* bop, int jt, int t,
-                                              int r0, int r1, int m0, int m1, float inv0, float inv1,
-                                              const float (&acc)[4]) {
+// Row stride (floats) of the fp32 x_tilde scratch per (m, 128-code block):
+// 128 MMA positions + 4 of padding, so that lanes on different blocks hit
+// different banks.
+constexpr int kXtStride = 132;
+
+// The lane's four x_tilde values of tile (rows r0, r1; codes 8 jt ..) into
+// the scratch, at their MMA position: xs[(m ncb + block) kXtStride + kap].
+__device__ __forceinline__ void store_xt(const DecodeParams& p, const BuildGeo& q, float* xs, int ncb, int jt,
+                                         int t, int r0, int r1, int m0, int m1, const float (&acc)[4]) {
   const bool ter = p.ternary != 0;
 #pragma unroll
   for (int e = 0; e < 4; ++e) {
@@ -227,25 +231,43 @@ __device__ __forceinline__ void write_terms_t(const DecodeParams& p, const Build
     const int64_t k = (int64_t)(q.blo + rho - m * q.nbi) * p.n_b + jt * 8 + 2 * t + (e & 1);
     if (k < q.k0 || k >= q.k1) continue;
     const int kl = (int)(k - q.k0);
-    uint8_t* blk = bop + (size_t)(kl >> 7) * p.NP * 128;
-    const int kap = decode_pos(kl & 127, ter);
-    float v = acc[e] * (e < 2 ? inv0 : inv1);
-#pragma unroll
-    for (int tt = 0; tt < T; ++tt) {
-      const uint32_t qb = f32_to_e4m3(v);
-      const int row = m * T + tt;
-      blk[row * 128 + (((kap >> 4) ^ (row & 7)) << 4) + (kap & 15)] = (uint8_t)qb;
-      if (tt + 1 < T) v = (v - e4m3_to_f32(qb)) * 16.f;
-    }
+    xs[(m * ncb + (kl >> 7)) * kXtStride + decode_pos(kl & 127, ter)] = acc[e];
   }
 }
-__device__ __forceinline__ void write_terms(const DecodeParams& p, const BuildGeo& q, uint8_t* bop, int jt, int t,
-                                            int r0, int r1, int m0, int m1, float inv0, float inv1,
-                                            const float (&acc)[4]) {
-  switch (p.T) {
-    case 4: write_terms_t<4>(p, q, bop, jt, t, r0, r1, m0, m1, inv0, inv1, acc); break;
-    case 3: write_terms_t<3>(p, q, bop, jt, t, r0, r1, m0, m1, inv0, inv1, acc); break;
-    default: write_terms_t<2>(p, q, bop, jt, t, r0, r1, m0, m1, inv0, inv1, acc); break;
+
+// T e4m3 terms of 16 consecutive MMA positions (one 16-byte chunk of each
+// term row), packed and stored 16 bytes at a time.
+template <int T>
+__device__ __forceinline__ void chunk_terms(const DecodeParams& p, uint8_t* bop, const float* xs, int ncb, int m,
+                                            int blk, int c, float inv, int lim) {
+  const bool ter = p.ternary != 0;
+  const float4* src = reinterpret_cast<const float4*>(xs + (m * ncb + blk) * kXtStride + 16 * c);
+  float v[16];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float4 f = src[i];
+    v[4 * i] = f.x; v[4 * i + 1] = f.y; v[4 * i + 2] = f.z; v[4 * i + 3] = f.w;
+  }
+#pragma unroll
+  for (int i = 0; i < 16; ++i)   // padding codes (k >= K_eff) are 0; the scratch is not written there
+    v[i] = blk * kBlk + decode_stage_k(16 * c + i, ter) < lim ? v[i] * inv : 0.f;
+  uint8_t* base = bop + (size_t)blk * p.NP * 128;
+#pragma unroll
+  for (int tt = 0; tt < T; ++tt) {
+    uint32_t w[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      uint32_t b4 = 0;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t qb = f32_to_e4m3(v[4 * i + j]);
+        b4 |= qb << (8 * j);
+        if (tt + 1 < T) v[4 * i + j] = (v[4 * i + j] - e4m3_to_f32(qb)) * 16.f;
+      }
+      w[i] = b4;
+    }
+    const int row = m * T + tt;
+    *reinterpret_cast<uint4*>(base + row * 128 + ((c ^ (row & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
   }
 }
 
@@ -257,7 +279,7 @@ __device__ __forceinline__ int term_exponent(float mx, float gnorm) {
 
 // Called by the kBuildThreads expander threads before their first stage; it
 // waits for the preceding grid itself (x may come from it; G does not).
-__device__ void build_b_operand(const DecodeParams& p, uint8_t* bop, int kb0, int ncb, int et,
+__device__ void build_b_operand(const DecodeParams& p, uint8_t* bop, float* xs, int kb0, int ncb, int et,
                                 uint32_t* xmax_u, float* inv_s, float* scale_s) {
   BuildGeo q;
   q.k0 = (int64_t)kb0 * kBlk;
@@ -284,7 +306,6 @@ __device__ void build_b_operand(const DecodeParams& p, uint8_t* bop, int kb0, in
     const uint16_t* xa0 = p.x + t * q.R + (v0 ? (size_t)m0 * p.K + (size_t)(q.blo + g - m0 * q.nbi) * p.B : 0);
     const uint16_t* xa1 = p.x + t * q.R + (v1 ? (size_t)m1 * p.K + (size_t)(q.blo + g + 8 - m1 * q.nbi) * p.B : 0);
     uint32_t mx0 = 0u, mx1 = 0u;   // max |x| bits of rows g, g + 8
-    float inv0 = 1.f, inv1 = 1.f;
     // A warp takes two adjacent code tiles per pass over x (one x load
     // feeds both), so that 16 warps cover 32 tiles (n_b = 256) in one item.
     for (int jt = 2 * ew; jt < JT; jt += 2 * NW) {
@@ -314,13 +335,14 @@ __device__ void build_b_operand(const DecodeParams& p, uint8_t* bop, int kb0, in
 #pragma unroll
           for (int o = 16; o > 0; o >>= 1) v = max(v, __shfl_xor_sync(0xffffffffu, v, o));
           const int e = term_exponent(__uint_as_float(v), p.gnorm);
-          if (m0 == mm) inv0 = ldexpf(1.f, -e);
-          if (m1 == mm) inv1 = ldexpf(1.f, -e);
-          if (et == mm) scale_s[mm] = ldexpf(1.f, e);
+          if (et == mm) {
+            scale_s[mm] = ldexpf(1.f, e);
+            inv_s[mm] = ldexpf(1.f, -e);
+          }
         }
       }
-      write_terms(p, q, bop, jt, t, g, g + 8, m0, m1, inv0, inv1, acc0);
-      if (two) write_terms(p, q, bop, jt + 1, t, g, g + 8, m0, m1, inv0, inv1, acc1);
+      store_xt(p, q, xs, ncb, jt, t, g, g + 8, m0, m1, acc0);
+      if (two) store_xt(p, q, xs, ncb, jt + 1, t, g, g + 8, m0, m1, acc1);
     }
   } else {
     pdl_wait();
@@ -373,17 +395,22 @@ __device__ void build_b_operand(const DecodeParams& p, uint8_t* bop, int kb0, in
       }
       float acc[4];
       acc_sum(acc4, acc);
-      write_terms(p, q, bop, jt, t, r0, r1, m0, m1, inv_s[m0], inv_s[m1], acc);
+      store_xt(p, q, xs, ncb, jt, t, r0, r1, m0, m1, acc);
     }
   }
-  // padding codes [k1, kend): zero terms
-  const int npad = (int)(q.kend - q.k1), lo = (int)(q.k1 - q.k0);
-  const bool ter = p.ternary != 0;
-  for (int i = et; i < npad * p.M * p.T; i += kBuildThreads) {
-    const int row = i / npad, kl = lo + (i - row * npad);
-    uint8_t* blk = bop + (size_t)(kl >> 7) * p.NP * 128;
-    const int kap = decode_pos(kl & 127, ter);
-    blk[row * 128 + (((kap >> 4) ^ (row & 7)) << 4) + (kap & 15)] = 0;
+  // x_tilde (all of the chunk, in the scratch) -> e4m3 terms: one thread per
+  // (m, block, 16-position chunk), 16-byte stores, consecutive threads on
+  // consecutive chunks of a term row (no bank conflicts).
+  named_bar_sync(3, kBuildThreads);
+  const int lim = (int)(q.k1 - q.k0);
+  for (int task = et; task < p.M * ncb * 8; task += kBuildThreads) {
+    const int m = task / (ncb * 8), rem = task - m * ncb * 8, blk = rem >> 3, c = rem & 7;
+    const float inv = inv_s[m];
+    switch (p.T) {
+      case 4: chunk_terms<4>(p, bop, xs, ncb, m, blk, c, inv, lim); break;
+      case 3: chunk_terms<3>(p, bop, xs, ncb, m, blk, c, inv, lim); break;
+      default: chunk_terms<2>(p, bop, xs, ncb, m, blk, c, inv, lim); break;
+    }
   }
   fence_proxy_async_smem();   // generic-proxy stores -> the MMAs' async-proxy reads
   named_bar_sync(3, kBuildThreads);
@@ -583,7 +610,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
     // Set x = 2e + t expands stages i = e + 2t (mod 4) in order: TMEM slot
     // x, ring slots i mod ring (ring is a multiple of 4).
     if (p.fused) {
-      build_b_operand(p, bop, kb0, ncb, tid - 32 * kExpWarp0, xmax_u, inv_s, scale_s);
+      // scratch: the ring slots the first kFusePre stages do not use
+      float* xs = reinterpret_cast<float*>(ring + (size_t)kFusePre * p.slot_bytes);
+      build_b_operand(p, bop, xs, kb0, ncb, tid - 32 * kExpWarp0, xmax_u, inv_s, scale_s);
       if (tid == 32 * kExpWarp0) mbar_arrive(&b_full);
     }
     const int x = (warp - kExpWarp0) >> 2, q = warp & 3, r = 32 * q + lane;
@@ -877,7 +906,13 @@ bool decode_fusable(const sdq_plan_s* pl, int M, const uint16_t* x) {
   const int64_t nbi = ((int64_t)dc.CB * kBlk + g.n_b - 1) / g.n_b + 1;
   const int64_t rt = ((int64_t)M * nbi + 15) / 16;
   const int64_t steps = rt * (g.n_b / 8) * (g.block / 16) / (kBuildThreads / 32);
-  return steps <= kMaxBuildSteps;
+  if (steps > kMaxBuildSteps) return false;
+  // the fp32 x_tilde scratch lives in the ring slots the first kFusePre stages do not use
+  int sb = 0, nbuf = 0, dbase = 0;
+  tmem_split(dc.NP, &sb, &nbuf, &dbase);
+  const size_t slot = (size_t)sb * kTileRows * kBlk * g.bits / 8;
+  const size_t scratch = (size_t)M * dc.CB * kXtStride * sizeof(float);
+  return dc.ring > kFusePre && scratch <= (size_t)(dc.ring - kFusePre) * slot;
 }
 
 cudaError_t launch_decode(const sdq_plan_s* pl, const uint32_t* codes, const float* alpha, int M,
