@@ -193,12 +193,19 @@ def run_sdq(args, rank, world, dist):
     M = args.m
     layers, enc_ms = build_layer(P, W, torch, cfg)
     code_bytes = sum(l["code_bytes"] for l in layers)
-    # per-linear inputs / outputs / workspaces
+    # per-linear inputs / outputs / workspaces; the step's x and y each live in
+    # one buffer (views per linear), so a step moves them with one copy each
+    xs = [torch.from_numpy(W.activations(lay["lin"], M).view(np.int16)).view(torch.bfloat16)
+          for lay in layers]
+    x_all = torch.cat([x.reshape(-1) for x in xs]).cuda()
+    y_all = torch.empty(sum(M * lay["lin"].n_out for lay in layers), dtype=torch.float32, device="cuda")
+    xo = yo = 0
     for lay in layers:
         lin = lay["lin"]
-        bits = W.activations(lin, M)
-        lay["x"] = torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).cuda()
-        lay["y"] = torch.empty((M, lin.n_out), dtype=torch.float32, device="cuda")
+        lay["x"] = x_all[xo:xo + M * lin.k_in].view(M, lin.k_in)
+        lay["y"] = y_all[yo:yo + M * lin.n_out].view(M, lin.n_out)
+        xo += M * lin.k_in
+        yo += M * lin.n_out
         lay["ws"] = lay["plan"].alloc_workspace(M)
         lay["kernels"] = P.sdq_forward_kernels(lay["plan"].handle, M, lay["x"])
 
@@ -293,17 +300,17 @@ def run_sdq(args, rank, world, dist):
 
     # end to end through the C ABI with host buffers (pinned), eager calls
     e2e_steps = min(200, max(20, args.steps // 100))
-    hx = [lay["x"].cpu().pin_memory() for lay in layers]
-    hy = [torch.empty_like(lay["y"], device="cpu").pin_memory() for lay in layers]
-    h2d = sum(h.numel() * h.element_size() for h in hx)
-    d2h = sum(h.numel() * h.element_size() for h in hy)
+    hx = x_all.cpu().pin_memory()
+    hy = torch.empty_like(y_all, device="cpu").pin_memory()
+    h2d = hx.numel() * hx.element_size()
+    d2h = hy.numel() * hy.element_size()
 
     def e2e_step():
-        for lay, xh, yh in zip(layers, hx, hy):
-            lay["x"].copy_(xh, non_blocking=True)
+        x_all.copy_(hx, non_blocking=True)      # the step's inputs, host -> device
+        for lay in layers:
             P.sdq_linear_forward(lay["plan"].handle, lay["tiled"], lay["alpha"], lay["x"], M,
                                  lay["y"], lay["ws"], stream)
-            yh.copy_(lay["y"], non_blocking=True)
+        hy.copy_(y_all, non_blocking=True)      # the step's results, device -> host
 
     with torch.cuda.stream(stream):
         for _ in range(3):
@@ -335,7 +342,8 @@ def run_sdq(args, rank, world, dist):
         "clocks": clocks,
         "e2e": {"value": round(e2e_val, 1), "unit": "GB/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms, 4),
-                "how": "eager sdq_linear_forward per linear with pinned-host x in and y out"},
+                "how": "per step: one pinned-host -> device copy of all x, eager sdq_linear_forward "
+                       "per linear, one device -> pinned-host copy of all y"},
         "gpu_launches": sum(lay["kernels"] for lay in layers) * args.steps,
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
                      "unit": "GB/s", "frac": round(achieved / hbm, 4), "traffic": traffic,

@@ -4,6 +4,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_fp8.h>
+#include <atomic>
 #include <cstdint>
 
 #include "sdq_internal.h"
@@ -41,6 +42,17 @@ bool decode_fusable(const sdq_plan_s* p, int M, const uint16_t* x);
 cudaError_t launch_prefill(const sdq_plan_s* p, const uint32_t* codes, const float* alpha, int M,
                            float* y, void* ws, cudaStream_t st);
 cudaError_t launch_read_prep(const sdq_plan_s* p, int M, const void* ws, float* out, cudaStream_t st);
+
+// Raise `kernel`'s dynamic shared-memory limit to `bytes` once per device:
+// the setting is per function and device, and a constant value makes later
+// launches (and concurrent callers) skip the driver call.
+template <class Kern>
+cudaError_t smem_limit_once(Kern kernel, int bytes, int device, std::atomic<int>* done) {
+  if (device >= 0 && device < 64 && done[device].load(std::memory_order_acquire)) return cudaSuccess;
+  const cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess && device >= 0 && device < 64) done[device].store(1, std::memory_order_release);
+  return e;
+}
 
 // ------------------------------------------------------------------ device
 __device__ __forceinline__ float bf16_bits_to_float(uint16_t b) {

@@ -942,8 +942,8 @@ cudaError_t launch_decode(const sdq_plan_s* pl, const uint32_t* codes, const flo
   p.blk_bytes = (uint32_t)(kTileRows * kBlk * g.bits / 8);
   p.slot_bytes = p.sb * p.blk_bytes;
   p.b_bytes = (uint32_t)(dc.CB * dc.NP * 128);
-  cudaError_t e = cudaFuncSetAttribute(decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)dc.smem);
+  static std::atomic<int> smem_set[64];   // per device: limit raised to kSmemMax + 1 KB
+  cudaError_t e = smem_limit_once(decode_kernel, kSmemMax + 1024, pl->device, smem_set);
   if (e != cudaSuccess) return e;
   return launch_pdl(decode_kernel, dim3(dc.S * dc.P), dim3(kThreads), dc.smem, st, p);
 }

@@ -338,7 +338,9 @@ cudaError_t launch_prep(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws
     p.vec = vec;
     p.k_eff = g.k_eff; p.kpad = g.k_eff_pad;
     const size_t smem = (size_t)(16 + 128) * (p.kc + 8) * sizeof(uint16_t);
-    cudaError_t e = cudaFuncSetAttribute(prep_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    static std::atomic<int> smem_set[64];   // per device: limit raised to the largest kc's need
+    cudaError_t e = smem_limit_once(prep_decode_kernel, (16 + 128) * (256 + 8) * (int)sizeof(uint16_t),
+                                    pl->device, smem_set);
     if (e != cudaSuccess) return e;
     dim3 grid((g.n_b + 63) / 64, (g.nblk + 15) / 16, M);
     return launch_pdl(prep_decode_kernel, grid, dim3(128), smem, st, p);
