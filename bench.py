@@ -50,6 +50,22 @@ def parse():
 
 
 # ------------------------------------------------------------------ utils
+def max_over_ranks(x, dist):
+    """Largest x over all ranks (a job's step time is its slowest rank's)."""
+    if not dist:
+        return float(x)
+    import torch
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([float(x)], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(units_per_rank, world, ms_step):
+    """Whole-job throughput (G units / s): what all ranks processed over the step time."""
+    return units_per_rank * world / (ms_step * 1e-3) / 1e9
+
+
 def peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -254,12 +270,9 @@ def run_sdq(args, rank, world, dist):
     ms_total = ev0.elapsed_time(ev1)
     clocks = sampler.summary(t_wall0, t_wall1)
     sampler.stop()
-    if dist:
-        t = torch.tensor([ms_total], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_total = float(t.item())
+    ms_total = max_over_ranks(ms_total, dist)
     ms_step = ms_total / args.steps
-    value = code_bytes * world / (ms_step * 1e-3) / 1e9
+    value = job_rate(code_bytes, world, ms_step)
 
     # the decode kernel alone, event-timed per launch: the one-kernel forward
     # where the step uses it, else the contraction behind its prepare kernel
