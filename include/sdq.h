@@ -161,8 +161,7 @@ int sdq_unpack(sdq_plan plan, const uint32_t* codes_tiled, uint32_t* codes_plain
  * M x k_in row-major), written into the workspace `ws` for sdq_contract.
  * M <= 64: one kernel writes x_tilde in fp32 and, as the decode kernel's
  * tensor-core B operand, T e4m3 terms per batch row m with
- * x_tilde[m] 2^-e_m = sum_t 16^-t q_t[m] (T = 4 for M <= 16, 3 for M <= 21,
- * else 2); e_m is set from the bound |x_tilde[m, j]| <= gnorm max_k |x[m, k]|,
+ * x_tilde[m] 2^-e_m = sum_t 16^-t q_t[m] (T = 4 for M <= 8, else 2); e_m is set from the bound |x_tilde[m, j]| <= gnorm max_k |x[m, k]|,
  * gnorm = max_j sum_k |G[j, k]|, so that no thread block waits for another.
  * M > 64: x_tilde is written in bf16 in the permuted K order the prefill
  * kernel reads.  Kernels are launched with programmatic dependent launch. */

@@ -34,9 +34,12 @@ int build_tables(const sdq_layer_desc* d, const int8_t* signs, float* a_enc, flo
 
 constexpr int kMaxDecodeM = 64;
 
-// e4m3 terms per activation on the decode path: the MMA cost does not grow
-// with N up to 64 columns (M * T), so small batches take more terms.
-inline int decode_terms(int M) { return M <= 16 ? 4 : (M <= 21 ? 3 : 2); }
+// e4m3 terms per activation on the decode path.  Up to N = M T = 32 MMA
+// columns the accumulators stay double-buffered and the MMA costs the same,
+// so batches up to 8 take four terms (~2^-16 relative); larger ones take two
+// (~2^-8, the level of the single bf16 rounding of x_tilde on the prefill
+// path).
+inline int decode_terms(int M) { return M <= 8 ? 4 : 2; }
 
 // G in the order the decode kernel's B-operand builders load it (only when
 // B % 16 == 0 and n_b % 8 == 0): for code tile jt (rows j = 8 jt .. 8 jt + 7),
