@@ -273,7 +273,12 @@ __device__ __forceinline__ void chunk_terms(const DecodeParams& p, uint8_t* bop,
 
 __device__ __forceinline__ int term_exponent(float mx, float gnorm) {
   int e = 0;
-  if (mx > 0.f) frexpf(mx * gnorm / 448.f, &e);   // bound * 2^-e < 448
+  if (mx > 0.f) {   // bound = mx gnorm < 2^(e1 + e2) without forming it (no overflow)
+    int e1 = 0, e2 = 0;
+    frexpf(mx, &e1);
+    frexpf(gnorm, &e2);
+    e = e1 + e2 - 8;   // bound * 2^-e < 256 < 448
+  }
   return max(e, -120);
 }
 

@@ -274,7 +274,12 @@ __global__ void __launch_bounds__(128) prep_decode_kernel(DecPrepParams p) {
   if (tid == 0) {
     const float mx = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
     int e = 0;
-    if (mx > 0.f) frexpf(mx * p.gnorm / 448.f, &e);   // bound * 2^-e < 448
+    if (mx > 0.f) {   // bound = mx gnorm < 2^(e1 + e2) without forming it (no overflow)
+      int e1 = 0, e2 = 0;
+      frexpf(mx, &e1);
+      frexpf(p.gnorm, &e2);
+      e = e1 + e2 - 8;   // bound * 2^-e < 256 < 448
+    }
     e = max(e, -120);
     e_s = e;
     if (jt == 0 && bt == 0) p.sexp[m] = e;
