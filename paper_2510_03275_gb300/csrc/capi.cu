@@ -5,6 +5,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <new>
+#include <numeric>
 #include <vector>
 
 #include "common.cuh"
@@ -87,7 +88,8 @@ extern "C" int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_sig
 
   const size_t tab = (size_t)g.n_b * g.block;
   std::vector<float> a_enc(tab), gm(tab), at(tab);
-  st = build_tables(desc, had_signs, a_enc.data(), gm.data());
+  std::vector<double> dt(tab);
+  st = build_tables(desc, had_signs, a_enc.data(), gm.data(), dt.data());
   if (st != SDQ_OK) return st;
   for (int j = 0; j < g.n_b; ++j)
     for (int k = 0; k < g.block; ++k) at[(size_t)k * g.n_b + j] = a_enc[(size_t)j * g.block + k];
@@ -121,8 +123,48 @@ extern "C" int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_sig
         }
   }
 
+  // Polyphase table of D^T (poly_stride) when D^T has that structure to fp64
+  // rounding and the table is small.
+  std::vector<uint32_t> poly;
+  const int B = g.block, pp = g.n_b / std::gcd(g.n_b, g.block), pq = g.block / std::gcd(g.n_b, g.block);
+  const size_t poly_bytes = (size_t)pp * poly_stride(B) * 8;
+  if (B % 16 == 0 && g.n_b % 8 == 0 && B <= kMaxPolyBlock && poly_bytes <= (size_t)kMaxPolyBytes) {
+    double mx = 0.0, dev = 0.0;
+    for (size_t i = 0; i < tab; ++i) mx = std::max(mx, std::fabs(dt[i]));
+    for (int j = 0; j < g.n_b; ++j)
+      for (int i = 0; i < B; ++i) {
+        const int src = (int)(((int64_t)i - (int64_t)pq * (j / pp)) % B + B) % B;
+        dev = std::max(dev, std::fabs(dt[(size_t)j * B + i] - dt[(size_t)(j % pp) * B + src]));
+      }
+    if (dev <= 1e-12 * mx) {
+      poly.assign(poly_bytes / 4 + B, 0u);
+      for (int r = 0; r < pp; ++r)
+        for (int d = 0; d < 2 * B; ++d) {
+          uint32_t hi = 0, lo = 0;
+          for (int h = 0; h < 2; ++h) {   // taps d and d + 1 (mod B): low and high halves
+            double v = dt[(size_t)r * B + (d + h) % B];
+            if (std::fabs(v) < 0x1p-46) v = 0.0;   // fp64 noise on exact zeros
+            const uint16_t vh = host_bf16(v), vl = host_bf16(v - host_bf16_value(vh));
+            hi |= (uint32_t)vh << (16 * h);
+            lo |= (uint32_t)vl << (16 * h);
+          }
+          const size_t e = (size_t)r * poly_stride(B) + d;
+          poly[2 * e] = hi;
+          poly[2 * e + 1] = lo;
+        }
+      const bool had = desc->hadamard != 0;
+      for (int k = 0; k < B; ++k) {
+        const float sk = had ? (float)((had_signs ? (double)had_signs[k] : 1.0) / std::sqrt((double)B)) : 1.0f;
+        std::memcpy(&poly[poly_bytes / 4 + k], &sk, 4);
+      }
+    }
+  }
+
   sdq_plan_s* p = new (std::nothrow) sdq_plan_s();
   if (!p) return SDQ_ERR_ALLOC;
+  p->poly_p = pp;
+  p->poly_q = pq;
+  p->poly_bytes = (int)poly_bytes;
   p->desc = *desc;
   p->geo = g;
   p->device = dev;
@@ -131,7 +173,8 @@ extern "C" int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_sig
   if (cudaMalloc(&p->d_at, sizeof(float) * tab) != cudaSuccess ||
       cudaMalloc(&p->d_g_hi, sizeof(uint16_t) * tab) != cudaSuccess ||
       cudaMalloc(&p->d_g_lo, sizeof(uint16_t) * tab) != cudaSuccess ||
-      (!gfrag.empty() && cudaMalloc(&p->d_g_frag, sizeof(uint16_t) * gfrag.size()) != cudaSuccess)) {
+      (!gfrag.empty() && cudaMalloc(&p->d_g_frag, sizeof(uint16_t) * gfrag.size()) != cudaSuccess) ||
+      (!poly.empty() && cudaMalloc(&p->d_poly, sizeof(uint32_t) * poly.size()) != cudaSuccess)) {
     sdq_plan_destroy(p);
     return SDQ_ERR_ALLOC;
   }
@@ -139,7 +182,9 @@ extern "C" int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_sig
       cudaMemcpy(p->d_g_hi, ghi.data(), sizeof(uint16_t) * tab, cudaMemcpyHostToDevice) != cudaSuccess ||
       cudaMemcpy(p->d_g_lo, glo.data(), sizeof(uint16_t) * tab, cudaMemcpyHostToDevice) != cudaSuccess ||
       (!gfrag.empty() && cudaMemcpy(p->d_g_frag, gfrag.data(), sizeof(uint16_t) * gfrag.size(),
-                                    cudaMemcpyHostToDevice) != cudaSuccess)) {
+                                    cudaMemcpyHostToDevice) != cudaSuccess) ||
+      (!poly.empty() && cudaMemcpy(p->d_poly, poly.data(), sizeof(uint32_t) * poly.size(),
+                                   cudaMemcpyHostToDevice) != cudaSuccess)) {
     sdq_plan_destroy(p);
     return SDQ_ERR_CUDA;
   }
@@ -155,6 +200,7 @@ extern "C" int sdq_plan_destroy(sdq_plan p) {
   if (p->d_g_hi && (e2 = cudaFree(p->d_g_hi)) != cudaSuccess) e = e2;
   if (p->d_g_lo && (e2 = cudaFree(p->d_g_lo)) != cudaSuccess) e = e2;
   if (p->d_g_frag && (e2 = cudaFree(p->d_g_frag)) != cudaSuccess) e = e2;
+  if (p->d_poly && (e2 = cudaFree(p->d_poly)) != cudaSuccess) e = e2;
   delete p;
   return cuda_status(e);
 }

@@ -97,8 +97,10 @@ struct DecodeParams {
   // Fused path (fused = 1): the B operand is built in the kernel from x.
   const uint16_t* x;     // M x K bf16 bits
   const uint16_t* g_frag; // G = D^T Had^T, bf16 hi + lo, warp-fragment order (g_frag_batch)
+  const uint32_t* poly;  // polyphase table of D^T (poly_stride), then B floats d_k / sqrt(B)
   float gnorm;           // max_j sum_i |G[j, i]| (with margin)
   int fused, K, B, n_b;
+  int use_poly, poly_p, poly_q, poly_bytes, fwht;
   int64_t k_eff;
   int M, T, NP, S, P, CB, KB, ring, sb, nbuf, dbase;
   int n_out, ntiles, ngroups, ternary, early;
@@ -129,18 +131,23 @@ __device__ __forceinline__ float bf16_mag(uint32_t h) { return __uint_as_float((
 // Fused B operand (small decode batches): the expander warps compute x_tilde
 // for this CTA's k chunk only,
 //   x_tilde[m, b n_b + j] = sum_i G[j, i] x[m, b B + i]      (G = D^T Had^T)
-// on warp MMAs (bf16 x exact, G as bf16 hi + lo, fp32 accumulation), and
-// write its T e4m3 terms into the shared-memory B image, laid out as the
-// decode prepare kernel lays out the global one.  The term scale 2^e_m is
-// this CTA's own, from the bound |x_tilde[m, k]| <= gnorm max |x[m, i]| over
-// the input blocks the chunk reads; the epilogue applies it to this CTA's
-// products only, so no CTA waits for another.
+// on warp MMAs with fp32 accumulation, and writes its T e4m3 terms into the
+// shared-memory B image, laid out as the decode prepare kernel lays out the
+// global one.  The term scale 2^e_m is this CTA's own, from the bound
+// |x_tilde[m, k]| <= gnorm max |x[m, i]| over the input blocks the chunk
+// reads; the epilogue applies it to this CTA's products only, so no CTA
+// waits for another.  Two ways to the same x_tilde:
+//   polyphase (B <= 256, use_poly): u = Had^T x_b by a fast Walsh-Hadamard
+//     transform, then x_tilde = D^T u with D^T's entries looked up in its
+//     polyphase table (a few KB in shared memory); u and D^T as bf16 hi + lo
+//   dense: G x_b with bf16 x exact and G as bf16 hi + lo, G's fragments
+//     streamed from the plan's fragment-ordered copy (n_b B 4 bytes)
 //
 // MMA tiles are 16 (m, b) rows x 8 codes j.  Per k batch of kbw inputs each
-// lane loads one contiguous run of x per row and one of G (the plan's
-// fragment-ordered copy), 16 bytes at a time: input t R + 4 s + r of the batch
-// is MMA K index 2t + (r & 1) + 8 (r >> 1) of step s, for x and G alike, which
-// leaves the dot products unchanged.
+// lane takes one contiguous run of the inputs (x or u) per row and of the
+// matching G or D^T entries: input t R + 4 s + r of the batch is MMA K index
+// 2t + (r & 1) + 8 (r >> 1) of step s, for both operands, which leaves the
+// dot products unchanged.
 struct BuildGeo {
   int64_t k0, k1, kend;   // chunk codes [k0, kend), with a value below k1
   int blo, nbi, rows;     // first input block, input blocks, (m, b) rows (m-major)
@@ -192,27 +199,10 @@ __device__ __forceinline__ void mma_batch(const BuildGeo& q, const uint32_t (&xw
       mma_bf16_16816(acc[1], a, gw[4 * s + 1], gw[4 * s + 3]);
     }
 }
-// One accumulator (hi and lo parts of G alternate into it).
-__device__ __forceinline__ void mma_batch1(const BuildGeo& q, const uint32_t (&xw)[2][8], const uint32_t (&gw)[16],
-                                           float (&acc)[4]) {
-#pragma unroll
-  for (int s = 0; s < 4; ++s)
-    if (s < q.S4) {
-      const uint32_t a[4] = {xw[0][2 * s], xw[1][2 * s], xw[0][2 * s + 1], xw[1][2 * s + 1]};
-      mma_bf16_16816(acc, a, gw[4 * s], gw[4 * s + 2]);
-      mma_bf16_16816(acc, a, gw[4 * s + 1], gw[4 * s + 3]);
-    }
-}
 __device__ __forceinline__ void acc_sum(const float (&a)[2][4], float (&out)[4]) {
 #pragma unroll
   for (int e = 0; e < 4; ++e) out[e] = a[0][e] + a[1][e];
 }
-// max of |bf16| over the halves of a word, as an order-preserving integer
-// (the magnitude bits of a non-negative float)
-__device__ __forceinline__ uint32_t bf16x2_absmax_bits(uint32_t w, uint32_t cur) {
-  return max(cur, max(w & 0x7FFF0000u, (w << 16) & 0x7FFF0000u));
-}
-
 // Row stride (floats) of the fp32 x_tilde scratch per (m, 128-code block):
 // 128 MMA positions + 4 of padding, so that lanes on different blocks hit
 // different banks.
@@ -271,6 +261,160 @@ __device__ __forceinline__ void chunk_terms(const DecodeParams& p, uint8_t* bop,
   }
 }
 
+// Polyphase build: u = Had^T x_b of one (m, b) row, V = B / 32 inputs per
+// lane (lanes beyond B / V idle), by a fast Walsh-Hadamard transform with
+// the sign and 1 / sqrt(B) scale applied first; stored as bf16 hi + lo rows
+// of stride us; returns the lane's max |x|.
+template <int V>
+__device__ __forceinline__ float row_transform(const DecodeParams& p, const uint16_t* xr, bool act, int lane,
+                                               uint16_t* uhi, uint16_t* ulo) {
+  float v[V];
+  uint32_t w[(V + 1) / 2];
+#pragma unroll
+  for (int i = 0; i < (V + 1) / 2; ++i) w[i] = 0u;
+  if (act) {
+    if constexpr (V == 8) {
+      const uint4 t4 = __ldg(reinterpret_cast<const uint4*>(xr));
+      w[0] = t4.x; w[1] = t4.y; w[2] = t4.z; w[3] = t4.w;
+    } else if constexpr (V == 4) {
+      const uint2 t2 = __ldg(reinterpret_cast<const uint2*>(xr));
+      w[0] = t2.x; w[1] = t2.y;
+    } else if constexpr (V == 2) {
+      w[0] = __ldg(reinterpret_cast<const uint32_t*>(xr));
+    } else {
+      w[0] = __ldg(reinterpret_cast<const unsigned short*>(xr));
+    }
+  }
+  float mx = 0.f;
+#pragma unroll
+  for (int e = 0; e < V; ++e) {
+    v[e] = __uint_as_float((e & 1) ? (w[e >> 1] & 0xFFFF0000u) : (w[e >> 1] << 16));
+    mx = fmaxf(mx, fabsf(v[e]));
+  }
+  if (act) {
+    const float* sg = reinterpret_cast<const float*>(p.poly) + p.poly_bytes / 4 + lane * V;
+#pragma unroll
+    for (int e = 0; e < V; ++e) v[e] *= __ldg(sg + e);
+  }
+  if (p.fwht) {
+#pragma unroll
+    for (int h = 1; h < V; h <<= 1)   // butterflies within the lane
+#pragma unroll
+      for (int e = 0; e < V; ++e)
+        if (!(e & h)) {
+          const float a = v[e], b = v[e + h];
+          v[e] = a + b;
+          v[e + h] = a - b;
+        }
+    for (int o = 1; o < p.B / V; o <<= 1)   // across lanes: index bit o * V
+#pragma unroll
+      for (int e = 0; e < V; ++e) {
+        const float other = __shfl_xor_sync(0xffffffffu, v[e], o);
+        v[e] = (lane & o) ? other - v[e] : v[e] + other;
+      }
+  }
+  if (lane * V < p.B) {
+    uint16_t hb[V], lb[V];
+#pragma unroll
+    for (int e = 0; e < V; ++e) {
+      hb[e] = float_to_bf16_bits(v[e]);
+      lb[e] = float_to_bf16_bits(v[e] - bf16_bits_to_float(hb[e]));
+    }
+    if constexpr (V == 1) {
+      uhi[lane] = hb[0];
+      ulo[lane] = lb[0];
+    } else {
+      uint32_t hw[V / 2], lw[V / 2];
+#pragma unroll
+      for (int i = 0; i < V / 2; ++i) {
+        hw[i] = (uint32_t)hb[2 * i] | ((uint32_t)hb[2 * i + 1] << 16);
+        lw[i] = (uint32_t)lb[2 * i] | ((uint32_t)lb[2 * i + 1] << 16);
+      }
+      if constexpr (V == 8) {
+        reinterpret_cast<uint4*>(uhi)[lane] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+        reinterpret_cast<uint4*>(ulo)[lane] = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+      } else if constexpr (V == 4) {
+        reinterpret_cast<uint2*>(uhi)[lane] = make_uint2(hw[0], hw[1]);
+        reinterpret_cast<uint2*>(ulo)[lane] = make_uint2(lw[0], lw[1]);
+      } else {
+        reinterpret_cast<uint32_t*>(uhi)[lane] = hw[0];
+        reinterpret_cast<uint32_t*>(ulo)[lane] = lw[0];
+      }
+    }
+  }
+  return mx;
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];\n"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]) : "r"(addr));
+}
+
+// x_tilde = D^T u of the polyphase build, for B a compile-time constant:
+// warp items (16-row tile rt of (m, b) rows, code tiles jt, jt + 1), 16-deep
+// steps s over the inputs in natural order.  A = u hi and lo rows by
+// ldmatrix; the lane's code row j = r + p m takes taps D^T[r][(i - q m)
+// mod B] for i = 16 s + 2t (+1, +8, +9) from one table base and the step's
+// constant offset.  u hi D hi goes to one accumulator, u lo D hi + u hi D lo
+// to another (the lo x lo term is below fp32 rounding of the sum).
+template <int B>
+__device__ __forceinline__ void poly_items(const DecodeParams& p, const BuildGeo& q, float* xs, int ncb,
+                                           const uint16_t* uhi, const uint16_t* ulo, const uint2* ptab,
+                                           int ew, int lane) {
+  constexpr int S = B / 16, US = B + 8, ST = poly_stride(B), NW = kBuildThreads / 32;
+  const int g = lane >> 2, t = lane & 3;
+  const int JT = p.n_b / 8, JP = (JT + 1) / 2, RT = (q.rows + 15) / 16;
+  const bool ter = p.ternary != 0;
+  const int lim = (int)(q.k1 - q.k0), k0 = (int)q.k0;
+  const int lrow = (lane & 7) + 8 * ((lane >> 3) & 1), lcol = 8 * (lane >> 4);   // ldmatrix row of this lane
+  for (int it = ew; it < RT * JP; it += NW) {
+    const int rt = it / JP, jt = 2 * (it - rt * JP);
+    const bool two = jt + 1 < JT;
+    const uint32_t ah_at = smem_u32(uhi + (rt * 16 + lrow) * US + lcol);
+    const uint32_t al_at = smem_u32(ulo + (rt * 16 + lrow) * US + lcol);
+    const int j0 = 8 * jt + g, j1 = j0 + 8;
+    const uint2* pb0 = ptab + (j0 % p.poly_p) * ST + ((2 * t - p.poly_q * (j0 / p.poly_p)) & (B - 1));
+    const uint2* pb1 = ptab + (j1 % p.poly_p) * ST + ((2 * t - p.poly_q * (j1 / p.poly_p)) & (B - 1));
+    float h0[4] = {0.f, 0.f, 0.f, 0.f}, l0[4] = {0.f, 0.f, 0.f, 0.f};
+    float h1[4] = {0.f, 0.f, 0.f, 0.f}, l1[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+      uint32_t ah[4], al[4];
+      ldsm_x4(ah_at + 32 * s, ah);
+      ldsm_x4(al_at + 32 * s, al);
+      const uint2 e0 = pb0[16 * s], f0 = pb0[16 * s + 8];
+      mma_bf16_16816(h0, ah, e0.x, f0.x);
+      mma_bf16_16816(l0, al, e0.x, f0.x);
+      mma_bf16_16816(l0, ah, e0.y, f0.y);
+      if (two) {
+        const uint2 e1 = pb1[16 * s], f1 = pb1[16 * s + 8];
+        mma_bf16_16816(h1, ah, e1.x, f1.x);
+        mma_bf16_16816(l1, al, e1.x, f1.x);
+        mma_bf16_16816(l1, ah, e1.y, f1.y);
+      }
+    }
+    // accumulator element e: (m, b) row rt 16 + g + 8 (e >> 1), code 8 jt + 2t + (e & 1)
+#pragma unroll
+    for (int hh = 0; hh < 2; ++hh) {
+      const int rho = rt * 16 + g + 8 * hh;
+      if (rho >= q.rows) continue;
+      const int m = rho / q.nbi;
+      const int off = (q.blo + rho - m * q.nbi) * p.n_b - k0 + 8 * jt + 2 * t;   // chunk-local code
+      float* xm = xs + m * ncb * kXtStride;
+#pragma unroll
+      for (int c = 0; c < 2; ++c)
+#pragma unroll
+        for (int tile = 0; tile < 2; ++tile) {
+          if (tile == 1 && !two) continue;
+          const int kl = off + 8 * tile + c;
+          if ((unsigned)kl >= (unsigned)lim) continue;
+          const float v = tile ? h1[2 * hh + c] + l1[2 * hh + c] : h0[2 * hh + c] + l0[2 * hh + c];
+          xm[(kl >> 7) * kXtStride + decode_pos(kl & 127, ter)] = v;
+        }
+    }
+  }
+}
+
 __device__ __forceinline__ int term_exponent(float mx, float gnorm) {
   int e = 0;
   if (mx > 0.f) {   // bound = mx gnorm < 2^(e1 + e2) without forming it (no overflow)
@@ -301,53 +445,50 @@ __device__ void build_b_operand(const DecodeParams& p, uint8_t* bop, float* xs, 
   constexpr int NW = kBuildThreads / 32;
   const int JT = p.n_b / 8;
 
-  if (q.rows <= 16 && q.nkb <= 2) {
-    // One row tile, B <= 128: every warp holds all of x's chunk in its A
-    // fragments, so each takes max |x[m]| from them (no cross-warp step); the
-    // G fragments of the warp's first code tile are loaded before the wait.
+  if (p.use_poly) {
+    // Polyphase build.  The table goes to shared memory before the wait (a
+    // plan constant); then each warp transforms (m, b) rows u = Had^T x_b
+    // (bf16 hi + lo rows behind the fp32 scratch) and adds max |x| into
+    // xmax_u; after one barrier the warps take (row tile, code tile pair)
+    // items of x_tilde = D^T u on warp MMAs.
+    const int B = p.B, us = B + 8, RT = (q.rows + 15) / 16;
+    uint16_t* uhi = reinterpret_cast<uint16_t*>(xs + (size_t)p.M * p.CB * kXtStride);
+    uint16_t* ulo = uhi + (size_t)16 * RT * us;
+    uint2* ptab = reinterpret_cast<uint2*>(ulo + (size_t)16 * RT * us);
+    for (int i = et; i < p.poly_bytes / 16; i += kBuildThreads)
+      reinterpret_cast<uint4*>(ptab)[i] = __ldg(reinterpret_cast<const uint4*>(p.poly) + i);
     pdl_wait();
-    const bool v0 = g < q.rows, v1 = g + 8 < q.rows;
-    const int m0 = v0 ? g / q.nbi : 0, m1 = v1 ? (g + 8) / q.nbi : 0;
-    const uint16_t* xa0 = p.x + t * q.R + (v0 ? (size_t)m0 * p.K + (size_t)(q.blo + g - m0 * q.nbi) * p.B : 0);
-    const uint16_t* xa1 = p.x + t * q.R + (v1 ? (size_t)m1 * p.K + (size_t)(q.blo + g + 8 - m1 * q.nbi) * p.B : 0);
-    uint32_t mx0 = 0u, mx1 = 0u;   // max |x| bits of rows g, g + 8
-    // A warp takes two adjacent code tiles per pass over x (one x load
-    // feeds both), so that 16 warps cover 32 tiles (n_b = 256) in one item.
-    for (int jt = 2 * ew; jt < JT; jt += 2 * NW) {
-      const bool first = jt == 2 * ew, two = jt + 1 < JT;
-      float acc0[4] = {0.f, 0.f, 0.f, 0.f}, acc1[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int kb = 0; kb < 2; ++kb)
-        if (kb < q.nkb) {
-          uint32_t xw[2][8], gw0[16], gw1[16];
-          load_g_frags(p, q, jt, kb, lane, gw0);
-          if (two) load_g_frags(p, q, jt + 1, kb, lane, gw1);
-          load_x_frags(q, xa0, xa1, kb, xw);   // (again for later tiles: an L1 hit)
-          if (first)
-#pragma unroll
-            for (int w = 0; w < 8; ++w) {
-              mx0 = bf16x2_absmax_bits(xw[0][w], mx0);
-              mx1 = bf16x2_absmax_bits(xw[1][w], mx1);
-            }
-          mma_batch1(q, xw, gw0, acc0);
-          if (two) mma_batch1(q, xw, gw1, acc1);
-        }
-      if (first) {   // max |x[m]| over the warp's fragments = over the whole chunk
-#pragma unroll
-        for (int mm = 0; mm < kMaxFuseM; ++mm) {
-          if (mm >= p.M) break;
-          uint32_t v = max(v0 && m0 == mm ? mx0 : 0u, v1 && m1 == mm ? mx1 : 0u);
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) v = max(v, __shfl_xor_sync(0xffffffffu, v, o));
-          const int e = term_exponent(__uint_as_float(v), p.gnorm);
-          if (et == mm) {
-            scale_s[mm] = ldexpf(1.f, e);
-            inv_s[mm] = ldexpf(1.f, -e);
-          }
-        }
+    const int V = B >= 32 ? B / 32 : 1;
+    for (int rho = ew; rho < 16 * RT; rho += NW) {
+      const bool in = rho < q.rows;
+      const int m = in ? rho / q.nbi : 0;
+      const bool act = in && lane * V < B;
+      const uint16_t* xr = p.x + (size_t)m * p.K + (size_t)(q.blo + rho - m * q.nbi) * B + lane * V;
+      uint16_t* rh = uhi + (size_t)rho * us;
+      uint16_t* rl = ulo + (size_t)rho * us;
+      float mx;
+      switch (V) {
+        case 8: mx = row_transform<8>(p, xr, act, lane, rh, rl); break;
+        case 4: mx = row_transform<4>(p, xr, act, lane, rh, rl); break;
+        case 2: mx = row_transform<2>(p, xr, act, lane, rh, rl); break;
+        default: mx = row_transform<1>(p, xr, act, lane, rh, rl); break;
       }
-      store_xt(p, q, xs, ncb, jt, t, g, g + 8, m0, m1, acc0);
-      if (two) store_xt(p, q, xs, ncb, jt + 1, t, g, g + 8, m0, m1, acc1);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      if (in && lane == 0) atomicMax(xmax_u + m, __float_as_uint(mx));   // non-negative: integer order
+    }
+    named_bar_sync(3, kBuildThreads);
+    if (et < p.M) {
+      const int e = term_exponent(__uint_as_float(xmax_u[et]), p.gnorm);
+      scale_s[et] = ldexpf(1.f, e);
+      inv_s[et] = ldexpf(1.f, -e);
+    }
+    switch (B) {
+      case 16: poly_items<16>(p, q, xs, ncb, uhi, ulo, ptab, ew, lane); break;
+      case 32: poly_items<32>(p, q, xs, ncb, uhi, ulo, ptab, ew, lane); break;
+      case 64: poly_items<64>(p, q, xs, ncb, uhi, ulo, ptab, ew, lane); break;
+      case 128: poly_items<128>(p, q, xs, ncb, uhi, ulo, ptab, ew, lane); break;
+      default: poly_items<256>(p, q, xs, ncb, uhi, ulo, ptab, ew, lane); break;
     }
   } else {
     pdl_wait();
@@ -900,24 +1041,36 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
   return best;
 }
 
-bool decode_fusable(const sdq_plan_s* pl, int M, const uint16_t* x) {
+// How the decode kernel would build its B operand at batch M: 2 polyphase,
+// 1 dense G, 0 not at all (the scratch does not fit the free ring slots, or
+// the build would take too many MMA steps per warp).
+int fused_build(const sdq_plan_s* pl, int M) {
   const Geometry& g = pl->geo;
-  if (M < 1 || M > kMaxFuseM || (reinterpret_cast<uintptr_t>(x) & 15u)) return false;
-  if (g.block % 16 != 0 || g.n_b % 8 != 0 || !pl->d_g_frag) return false;
+  if (M < 1 || M > kMaxFuseM) return 0;
+  if (g.block % 16 != 0 || g.n_b % 8 != 0 || !pl->d_g_frag) return 0;
   const DecodeConfig& dc = decode_config(pl, M);
-  if (dc.S < 1) return false;
+  if (dc.S < 1) return 0;
   // MMA steps per builder warp for the widest chunk: (m, b) row tiles x code
   // tiles x 16-deep steps over B, shared by the 16 warps.
   const int64_t nbi = ((int64_t)dc.CB * kBlk + g.n_b - 1) / g.n_b + 1;
   const int64_t rt = ((int64_t)M * nbi + 15) / 16;
   const int64_t steps = rt * (g.n_b / 8) * (g.block / 16) / (kBuildThreads / 32);
-  if (steps > kMaxBuildSteps) return false;
-  // the fp32 x_tilde scratch lives in the ring slots the first kFusePre stages do not use
+  if (steps > kMaxBuildSteps) return 0;
+  // the fp32 x_tilde scratch (and the polyphase build's u rows and table)
+  // lives in the ring slots the first kFusePre stages do not use
   int sb = 0, nbuf = 0, dbase = 0;
   tmem_split(dc.NP, &sb, &nbuf, &dbase);
   const size_t slot = (size_t)sb * kTileRows * kBlk * g.bits / 8;
+  if (dc.ring <= kFusePre) return 0;
+  const size_t room = (size_t)(dc.ring - kFusePre) * slot;
   const size_t scratch = (size_t)M * dc.CB * kXtStride * sizeof(float);
-  return dc.ring > kFusePre && scratch <= (size_t)(dc.ring - kFusePre) * slot;
+  const size_t poly = (size_t)2 * 16 * rt * (g.block + 8) * sizeof(uint16_t) + (size_t)pl->poly_bytes;
+  if (pl->d_poly && scratch + poly <= room) return 2;
+  return scratch <= room ? 1 : 0;
+}
+
+bool decode_fusable(const sdq_plan_s* pl, int M, const uint16_t* x) {
+  return (reinterpret_cast<uintptr_t>(x) & 15u) == 0 && fused_build(pl, M) != 0;
 }
 
 cudaError_t launch_decode(const sdq_plan_s* pl, const uint32_t* codes, const float* alpha, int M,
@@ -937,6 +1090,9 @@ cudaError_t launch_decode(const sdq_plan_s* pl, const uint32_t* codes, const flo
   p.call = next_call_number();
   p.fused = x != nullptr;
   p.x = x; p.g_frag = pl->d_g_frag; p.gnorm = pl->gnorm;
+  p.use_poly = p.fused && fused_build(pl, M) == 2;
+  p.poly = pl->d_poly; p.poly_p = pl->poly_p; p.poly_q = pl->poly_q; p.poly_bytes = pl->poly_bytes;
+  p.fwht = pl->desc.hadamard != 0;
   p.K = g.k_in; p.B = g.block; p.n_b = g.n_b; p.k_eff = g.k_eff;
   if (p.fused) early = 0;   // x and the codes may come from the preceding grid
   p.M = M; p.T = dc.T; p.NP = dc.NP; p.S = dc.S; p.P = dc.P; p.CB = dc.CB;

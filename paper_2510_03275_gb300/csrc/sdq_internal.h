@@ -30,7 +30,8 @@ int validate(const sdq_layer_desc* d, Geometry* g);
 // Host fp64 construction of the tables (see tables.cpp).
 //   a_enc: n_b x B row-major, A_enc[j][k] = fp32(sum_k' U[j][k'] Had[k][k'])
 //   g:     n_b x B row-major, G[j][k]     = fp32(sum_k' Dt[j][k'] Had[k][k'])
-int build_tables(const sdq_layer_desc* d, const int8_t* signs, float* a_enc, float* g);
+//   dt:    n_b x B row-major, D^T itself in fp64 (optional)
+int build_tables(const sdq_layer_desc* d, const int8_t* signs, float* a_enc, float* g, double* dt = nullptr);
 
 constexpr int kMaxDecodeM = 64;
 
@@ -54,6 +55,24 @@ __host__ __device__
 #endif
 inline int g_frag_batch(int B) { return B < 64 ? B : 64; }
 
+// Polyphase table of D^T for the decode kernel's own activation build.
+// With n_b / B = p / q in lowest terms, band-limited resampling commutes with
+// a cyclic shift of q inputs (p codes), so row r + p m of D^T is row r
+// shifted by q m:  D^T[r + p m][i] = D^T[r][(i - q m) mod B]  (checked at plan
+// time), and x_tilde = D^T (Had^T x_b) needs only D^T's first p rows.  Entry
+// r * poly_stride(B) + d, d < 2B, holds the pair (D^T[r][d mod B],
+// D^T[r][(d + 1) mod B]) as a bf16x2 word (hi) and the pair's bf16
+// remainders (lo), so that a run of taps from any start d < B needs no
+// wrap-around; after the p * poly_stride(B) entries come B floats
+// s_k = d_k / sqrt(B) (1 without the Hadamard transform).  A stride of 8
+// (mod 16) entries puts a warp's lookups of two phases in different banks.
+#ifdef __CUDACC__
+__host__ __device__
+#endif
+constexpr int poly_stride(int B) { return 2 * B + 8; }
+constexpr int kMaxPolyBlock = 256;       // B of the polyphase build (8 inputs per lane)
+constexpr int kMaxPolyBytes = 16 * 1024; // table entries, without the B floats
+
 // Launch shape of the decode kernel for one batch size (chosen at plan time).
 // Grid = S * P CTAs, one per SM: CTA (s, p) contracts k chunk s (CB blocks
 // of 128 codes) against row tiles p, p + P, p + 2P, ...
@@ -76,5 +95,8 @@ struct sdq_plan_s {
   uint16_t* d_g_hi;    // G as bf16 hi part, n_b x B row-major
   uint16_t* d_g_lo;    // G - hi as bf16, n_b x B row-major
   uint16_t* d_g_frag;  // G hi + lo in warp-fragment order (g_frag_index), or null
+  uint32_t* d_poly;    // polyphase table of D^T (poly_stride), or null
+  int poly_p, poly_q;  // n_b / B = poly_p / poly_q in lowest terms
+  int poly_bytes;      // bytes of the table's entries (the B floats follow)
   sdq::DecodeConfig dcfg[sdq::kMaxDecodeM + 1];  // decode launch shape per batch size
 };

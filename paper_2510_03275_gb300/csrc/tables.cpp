@@ -71,7 +71,7 @@ void fwht(double* v, int n) {
 
 }  // namespace
 
-int build_tables(const sdq_layer_desc* desc, const int8_t* signs, float* a_enc, float* gout) {
+int build_tables(const sdq_layer_desc* desc, const int8_t* signs, float* a_enc, float* gout, double* dt_out) {
   Geometry g;
   int st = validate(desc, &g);
   if (st != SDQ_OK) return st;
@@ -117,6 +117,7 @@ int build_tables(const sdq_layer_desc* desc, const int8_t* signs, float* a_enc, 
       }
     }
   }
+  if (dt_out) std::memcpy(dt_out, Dt.data(), sizeof(double) * Dt.size());
   // Right-multiply by Had^T: row j -> d_k / sqrt(B) * (H_B row_j)[k].
   std::vector<double> row(B);
   for (int which = 0; which < 2; ++which) {

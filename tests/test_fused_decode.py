@@ -22,8 +22,8 @@ def torch_cuda():
     return torch
 
 
-def _layer(sdq, torch, n, k, b, osr, q, seed):
-    d = sdq.LayerDesc(n, k, b, Fraction(osr), q, 1, 0)
+def _layer(sdq, torch, n, k, b, osr, q, seed, hadamard=1):
+    d = sdq.LayerDesc(n, k, b, Fraction(osr), q, hadamard, 0)
     rng = np.random.default_rng(seed)
     signs = np.where(rng.random(b) < 0.5, -1, 1).astype(np.int8)
     plan = sdq.Plan(d, signs)
@@ -47,9 +47,12 @@ def _rel(a, b):
 
 # Shapes the fused path takes: ragged N, K_eff not a multiple of 128 (padding
 # inside the last chunk), OSR 2.5 / 1.5 (128-code blocks straddle input
-# blocks), B = 16 and 256.
+# blocks), B = 16, 64 and 256 (the polyphase build with 1, 2 and 8 inputs per
+# lane), and OSR 17/16, whose 17 phases make the polyphase table too large:
+# the dense-G build.
 FUSED_SHAPES = [(33, 384, 128, Fraction(5, 2)), (100, 1024, 128, Fraction(3, 2)),
-                (300, 2048, 128, 2), (129, 272, 16, Fraction(5, 2)), (64, 1024, 256, 2)]
+                (300, 2048, 128, 2), (129, 272, 16, Fraction(5, 2)), (64, 1024, 256, 2),
+                (77, 640, 64, Fraction(9, 4)), (70, 512, 128, Fraction(17, 16))]
 
 
 @pytest.mark.parametrize("q", [O.TERNARY, O.BINARY])
@@ -79,6 +82,22 @@ def test_fused_forward_matches_oracle_and_two_kernel_path(sdq, torch_cuda, q, m,
     e1, e2 = _rel(y1.cpu().numpy(), yr), _rel(y2.cpu().numpy(), yr)
     assert e1 <= 1e-3 and e2 <= 1e-3, (e1, e2)
     assert _rel(y1.cpu().numpy(), y2.cpu().numpy()) <= 1e-3
+
+
+@pytest.mark.parametrize("m", [1, 3])
+@pytest.mark.parametrize("shape", [(300, 2048, 128, 2), (129, 272, 16, Fraction(5, 2)),
+                                   (70, 512, 128, Fraction(17, 16))])
+def test_fused_forward_without_hadamard(sdq, torch_cuda, m, shape):
+    """Layers encoded without the Hadamard rotation (G = D^T): the one-kernel
+    build skips the Walsh-Hadamard transform and matches the oracle."""
+    torch = torch_cuda
+    n, k, b, osr = shape
+    plan, d, signs, codes, alpha, tiled = _layer(sdq, torch, n, k, b, osr, O.TERNARY, seed=n + m, hadamard=0)
+    bits, x = _x(torch, m, k, seed=5 * m + 2)
+    assert sdq.sdq_forward_kernels(plan.handle, m, x) == 1
+    y = plan.forward(tiled, torch.from_numpy(alpha).cuda(), x).cpu().numpy()
+    yr = O.forward_code_domain(W.bf16_to_float(bits), codes, alpha, b, d.n_b, signs, hadamard=False)
+    assert _rel(y, yr) <= 1e-3
 
 
 def test_fused_forward_ignores_workspace_contents(sdq, torch_cuda):

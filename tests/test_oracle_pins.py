@@ -318,6 +318,26 @@ def test_decimation_adjoint_is_upsample_over_osr_plus_rank1():
     assert np.abs(Dt - U * B / nb - want).max() < 1e-13
 
 
+@pytest.mark.parametrize("B,osr", [(16, Fraction(5, 2)), (128, 2), (128, Fraction(3, 2)), (64, Fraction(9, 4)),
+                                   (256, 2), (2, Fraction(3, 2))])
+def test_decimation_adjoint_is_polyphase(B, osr):
+    """Band-limited resampling commutes with shifts that land on both grids:
+    n_b / B = p / q, a cyclic shift of the n_b codes by p is one of the B
+    outputs by q, so row r + p m of D^T is row r rolled by q m (the structure
+    the decode kernel's polyphase table stores)."""
+    nb = int(B * osr)
+    p, q = osr.numerator, osr.denominator
+    rng = np.random.default_rng(B + nb)
+    v = rng.standard_normal((3, nb))
+    lhs = O.resample(np.roll(v, p, axis=1), B)
+    rhs = np.roll(O.resample(v, B), q, axis=1)
+    assert np.abs(lhs - rhs).max() < 1e-12 * np.abs(rhs).max()
+    Dt = O.resample_matrix(nb, B)
+    for j in range(nb):
+        r, m = j % p, j // p
+        assert np.abs(Dt[j] - np.roll(Dt[r], q * m)).max() < 1e-13
+
+
 def test_canonical_and_f64_encoders_agree():
     """The fp32 canonical encoder and the fp64 FFT reading pick the same codes
     except where an integrator value lands within rounding of a threshold."""
