@@ -225,28 +225,29 @@ __device__ __forceinline__ void store_xt(const DecodeParams& p, const BuildGeo& 
   }
 }
 
-// T e4m3 terms of 16 consecutive MMA positions (one 16-byte chunk of each
-// term row), packed and stored 16 bytes at a time.
-template <int T>
+// T e4m3 terms of W = 16 or 8 consecutive MMA positions (all or half of one
+// 16-byte chunk of each term row), packed and stored W bytes at a time.
+// Position 16 c + h W + i of block blk, batch row m.
+template <int T, int W>
 __device__ __forceinline__ void chunk_terms(const DecodeParams& p, uint8_t* bop, const float* xs, int ncb, int m,
-                                            int blk, int c, float inv, int lim) {
+                                            int blk, int c, int h, float inv, int lim) {
   const bool ter = p.ternary != 0;
-  const float4* src = reinterpret_cast<const float4*>(xs + (m * ncb + blk) * kXtStride + 16 * c);
-  float v[16];
+  const float4* src = reinterpret_cast<const float4*>(xs + (m * ncb + blk) * kXtStride + 16 * c + W * h);
+  float v[W];
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
+  for (int i = 0; i < W / 4; ++i) {
     const float4 f = src[i];
     v[4 * i] = f.x; v[4 * i + 1] = f.y; v[4 * i + 2] = f.z; v[4 * i + 3] = f.w;
   }
 #pragma unroll
-  for (int i = 0; i < 16; ++i)   // padding codes (k >= K_eff) are 0; the scratch is not written there
-    v[i] = blk * kBlk + decode_stage_k(16 * c + i, ter) < lim ? v[i] * inv : 0.f;
+  for (int i = 0; i < W; ++i)   // padding codes (k >= K_eff) are 0; the scratch is not written there
+    v[i] = blk * kBlk + decode_stage_k(16 * c + W * h + i, ter) < lim ? v[i] * inv : 0.f;
   uint8_t* base = bop + (size_t)blk * p.NP * 128;
 #pragma unroll
   for (int tt = 0; tt < T; ++tt) {
-    uint32_t w[4];
+    uint32_t w[W / 4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
+    for (int i = 0; i < W / 4; ++i) {
       uint32_t b4 = 0;
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
@@ -257,7 +258,27 @@ __device__ __forceinline__ void chunk_terms(const DecodeParams& p, uint8_t* bop,
       w[i] = b4;
     }
     const int row = m * T + tt;
-    *reinterpret_cast<uint4*>(base + row * 128 + ((c ^ (row & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+    uint8_t* dst = base + row * 128 + ((c ^ (row & 7)) << 4) + W * h;
+    if constexpr (W == 16)
+      *reinterpret_cast<uint4*>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+    else
+      *reinterpret_cast<uint2*>(dst) = make_uint2(w[0], w[1]);
+  }
+}
+
+template <int W>
+__device__ __forceinline__ void all_terms(const DecodeParams& p, uint8_t* bop, const float* xs, int ncb, int et,
+                                          const float* inv_s, int lim) {
+  constexpr int PER = 128 / W;   // tasks per (m, block)
+  for (int task = et; task < p.M * ncb * PER; task += kBuildThreads) {
+    const int m = task / (ncb * PER), rem = task - m * ncb * PER, blk = rem / PER, cw = rem % PER;
+    const int c = cw / (16 / W), h = cw % (16 / W);
+    const float inv = inv_s[m];
+    switch (p.T) {
+      case 4: chunk_terms<4, W>(p, bop, xs, ncb, m, blk, c, h, inv, lim); break;
+      case 3: chunk_terms<3, W>(p, bop, xs, ncb, m, blk, c, h, inv, lim); break;
+      default: chunk_terms<2, W>(p, bop, xs, ncb, m, blk, c, h, inv, lim); break;
+    }
   }
 }
 
@@ -353,30 +374,32 @@ __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
 // x_tilde = D^T u of the polyphase build, for B a compile-time constant:
 // warp items (16-row tile rt of (m, b) rows, code tiles jt, jt + 1), 16-deep
 // steps s over the inputs in natural order.  A = u hi and lo rows by
-// ldmatrix; the lane's code row j = r + p m takes taps D^T[r][(i - q m)
-// mod B] for i = 16 s + 2t (+1, +8, +9) from one table base and the step's
-// constant offset.  u hi D hi goes to one accumulator, u lo D hi + u hi D lo
-// to another (the lo x lo term is below fp32 rounding of the sum).
+// ldmatrix; code row j = r + p m takes taps D^T[r][(i - q m) mod B] for
+// i = 16 s + 2t (+1, +8, +9) at table entry jbase[j] + 2t + 16 s (+8): one
+// base per lane and tile, constant offsets per step.  u hi D hi, u lo D hi
+// and u hi D lo go to three accumulators (short dependency chains); the
+// lo x lo term is below fp32 rounding of the sum.  rowoff / rowxm give each
+// (m, b) row's chunk-local first code and scratch offset (rowoff is far
+// negative for rows past the chunk's).
 template <int B>
-__device__ __forceinline__ void poly_items(const DecodeParams& p, const BuildGeo& q, float* xs, int ncb,
+__device__ __forceinline__ void poly_items(const DecodeParams& p, const BuildGeo& q, float* xs,
                                            const uint16_t* uhi, const uint16_t* ulo, const uint2* ptab,
-                                           int ew, int lane) {
-  constexpr int S = B / 16, US = B + 8, ST = poly_stride(B), NW = kBuildThreads / 32;
+                                           const int* jbase, const int* rowoff, const int* rowxm, int ew, int lane) {
+  constexpr int S = B / 16, US = B + 8, NW = kBuildThreads / 32;
   const int g = lane >> 2, t = lane & 3;
   const int JT = p.n_b / 8, JP = (JT + 1) / 2, RT = (q.rows + 15) / 16;
   const bool ter = p.ternary != 0;
-  const int lim = (int)(q.k1 - q.k0), k0 = (int)q.k0;
+  const int lim = (int)(q.k1 - q.k0);
   const int lrow = (lane & 7) + 8 * ((lane >> 3) & 1), lcol = 8 * (lane >> 4);   // ldmatrix row of this lane
   for (int it = ew; it < RT * JP; it += NW) {
-    const int rt = it / JP, jt = 2 * (it - rt * JP);
+    const int rt = it < JP ? 0 : it / JP, jt = 2 * (it - rt * JP);
     const bool two = jt + 1 < JT;
     const uint32_t ah_at = smem_u32(uhi + (rt * 16 + lrow) * US + lcol);
     const uint32_t al_at = smem_u32(ulo + (rt * 16 + lrow) * US + lcol);
-    const int j0 = 8 * jt + g, j1 = j0 + 8;
-    const uint2* pb0 = ptab + (j0 % p.poly_p) * ST + ((2 * t - p.poly_q * (j0 / p.poly_p)) & (B - 1));
-    const uint2* pb1 = ptab + (j1 % p.poly_p) * ST + ((2 * t - p.poly_q * (j1 / p.poly_p)) & (B - 1));
-    float h0[4] = {0.f, 0.f, 0.f, 0.f}, l0[4] = {0.f, 0.f, 0.f, 0.f};
-    float h1[4] = {0.f, 0.f, 0.f, 0.f}, l1[4] = {0.f, 0.f, 0.f, 0.f};
+    const uint2* pb0 = ptab + jbase[8 * jt + g] + 2 * t;
+    const uint2* pb1 = ptab + (two ? jbase[8 * jt + 8 + g] : 0) + 2 * t;
+    float h0[4] = {0.f, 0.f, 0.f, 0.f}, a0[4] = {0.f, 0.f, 0.f, 0.f}, b0[4] = {0.f, 0.f, 0.f, 0.f};
+    float h1[4] = {0.f, 0.f, 0.f, 0.f}, a1[4] = {0.f, 0.f, 0.f, 0.f}, b1[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int s = 0; s < S; ++s) {
       uint32_t ah[4], al[4];
@@ -384,31 +407,29 @@ __device__ __forceinline__ void poly_items(const DecodeParams& p, const BuildGeo
       ldsm_x4(al_at + 32 * s, al);
       const uint2 e0 = pb0[16 * s], f0 = pb0[16 * s + 8];
       mma_bf16_16816(h0, ah, e0.x, f0.x);
-      mma_bf16_16816(l0, al, e0.x, f0.x);
-      mma_bf16_16816(l0, ah, e0.y, f0.y);
+      mma_bf16_16816(a0, al, e0.x, f0.x);
+      mma_bf16_16816(b0, ah, e0.y, f0.y);
       if (two) {
         const uint2 e1 = pb1[16 * s], f1 = pb1[16 * s + 8];
         mma_bf16_16816(h1, ah, e1.x, f1.x);
-        mma_bf16_16816(l1, al, e1.x, f1.x);
-        mma_bf16_16816(l1, ah, e1.y, f1.y);
+        mma_bf16_16816(a1, al, e1.x, f1.x);
+        mma_bf16_16816(b1, ah, e1.y, f1.y);
       }
     }
     // accumulator element e: (m, b) row rt 16 + g + 8 (e >> 1), code 8 jt + 2t + (e & 1)
 #pragma unroll
     for (int hh = 0; hh < 2; ++hh) {
       const int rho = rt * 16 + g + 8 * hh;
-      if (rho >= q.rows) continue;
-      const int m = rho / q.nbi;
-      const int off = (q.blo + rho - m * q.nbi) * p.n_b - k0 + 8 * jt + 2 * t;   // chunk-local code
-      float* xm = xs + m * ncb * kXtStride;
+      const int off = rowoff[rho] + 8 * jt + 2 * t;   // chunk-local code
+      float* xm = xs + rowxm[rho];
 #pragma unroll
       for (int c = 0; c < 2; ++c)
 #pragma unroll
         for (int tile = 0; tile < 2; ++tile) {
           if (tile == 1 && !two) continue;
-          const int kl = off + 8 * tile + c;
+          const int kl = off + 8 * tile + c, e = 2 * hh + c;
           if ((unsigned)kl >= (unsigned)lim) continue;
-          const float v = tile ? h1[2 * hh + c] + l1[2 * hh + c] : h0[2 * hh + c] + l0[2 * hh + c];
+          const float v = tile ? h1[e] + (a1[e] + b1[e]) : h0[e] + (a0[e] + b0[e]);
           xm[(kl >> 7) * kXtStride + decode_pos(kl & 127, ter)] = v;
         }
     }
@@ -455,8 +476,13 @@ __device__ void build_b_operand(const DecodeParams& p, uint8_t* bop, float* xs, 
     uint16_t* uhi = reinterpret_cast<uint16_t*>(xs + (size_t)p.M * p.CB * kXtStride);
     uint16_t* ulo = uhi + (size_t)16 * RT * us;
     uint2* ptab = reinterpret_cast<uint2*>(ulo + (size_t)16 * RT * us);
+    int* jbase = reinterpret_cast<int*>(ptab + p.poly_bytes / 8);   // n_b entries
+    int* rowoff = jbase + p.n_b;                                      // 16 RT (m, b) rows
+    int* rowxm = rowoff + 16 * RT;
     for (int i = et; i < p.poly_bytes / 16; i += kBuildThreads)
       reinterpret_cast<uint4*>(ptab)[i] = __ldg(reinterpret_cast<const uint4*>(p.poly) + i);
+    for (int j = et; j < p.n_b; j += kBuildThreads)   // code row j = r + p m: phase row r, taps from -q m
+      jbase[j] = (j % p.poly_p) * poly_stride(B) + ((-p.poly_q * (j / p.poly_p)) & (B - 1));
     pdl_wait();
     const int V = B >= 32 ? B / 32 : 1;
     for (int rho = ew; rho < 16 * RT; rho += NW) {
@@ -475,7 +501,11 @@ __device__ void build_b_operand(const DecodeParams& p, uint8_t* bop, float* xs, 
       }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-      if (in && lane == 0) atomicMax(xmax_u + m, __float_as_uint(mx));   // non-negative: integer order
+      if (lane == 0) {
+        if (in) atomicMax(xmax_u + m, __float_as_uint(mx));   // non-negative: integer order
+        rowoff[rho] = in ? (q.blo + rho - m * q.nbi) * p.n_b - (int)q.k0 : -(1 << 30);
+        rowxm[rho] = m * ncb * kXtStride;
+      }
     }
     named_bar_sync(3, kBuildThreads);
     if (et < p.M) {
@@ -484,11 +514,11 @@ __device__ void build_b_operand(const DecodeParams& p, uint8_t* bop, float* xs, 
       inv_s[et] = ldexpf(1.f, -e);
     }
     switch (B) {
-      case 16: poly_items<16>(p, q, xs, ncb, uhi, ulo, ptab, ew, lane); break;
-      case 32: poly_items<32>(p, q, xs, ncb, uhi, ulo, ptab, ew, lane); break;
-      case 64: poly_items<64>(p, q, xs, ncb, uhi, ulo, ptab, ew, lane); break;
-      case 128: poly_items<128>(p, q, xs, ncb, uhi, ulo, ptab, ew, lane); break;
-      default: poly_items<256>(p, q, xs, ncb, uhi, ulo, ptab, ew, lane); break;
+      case 16: poly_items<16>(p, q, xs, uhi, ulo, ptab, jbase, rowoff, rowxm, ew, lane); break;
+      case 32: poly_items<32>(p, q, xs, uhi, ulo, ptab, jbase, rowoff, rowxm, ew, lane); break;
+      case 64: poly_items<64>(p, q, xs, uhi, ulo, ptab, jbase, rowoff, rowxm, ew, lane); break;
+      case 128: poly_items<128>(p, q, xs, uhi, ulo, ptab, jbase, rowoff, rowxm, ew, lane); break;
+      default: poly_items<256>(p, q, xs, uhi, ulo, ptab, jbase, rowoff, rowxm, ew, lane); break;
     }
   } else {
     pdl_wait();
@@ -546,18 +576,14 @@ __device__ void build_b_operand(const DecodeParams& p, uint8_t* bop, float* xs, 
   }
   // x_tilde (all of the chunk, in the scratch) -> e4m3 terms: one thread per
   // (m, block, 16-position chunk), 16-byte stores, consecutive threads on
-  // consecutive chunks of a term row (no bank conflicts).
+  // consecutive chunks of a term row (no bank conflicts); per half chunk, 8-byte
+  // stores, when whole chunks would leave half the builders idle.
   named_bar_sync(3, kBuildThreads);
   const int lim = (int)(q.k1 - q.k0);
-  for (int task = et; task < p.M * ncb * 8; task += kBuildThreads) {
-    const int m = task / (ncb * 8), rem = task - m * ncb * 8, blk = rem >> 3, c = rem & 7;
-    const float inv = inv_s[m];
-    switch (p.T) {
-      case 4: chunk_terms<4>(p, bop, xs, ncb, m, blk, c, inv, lim); break;
-      case 3: chunk_terms<3>(p, bop, xs, ncb, m, blk, c, inv, lim); break;
-      default: chunk_terms<2>(p, bop, xs, ncb, m, blk, c, inv, lim); break;
-    }
-  }
+  if (p.M * ncb * 8 <= kBuildThreads / 2)   // too few 16-position tasks for the builders: halve them
+    all_terms<8>(p, bop, xs, ncb, et, inv_s, lim);
+  else
+    all_terms<16>(p, bop, xs, ncb, et, inv_s, lim);
   fence_proxy_async_smem();   // generic-proxy stores -> the MMAs' async-proxy reads
   named_bar_sync(3, kBuildThreads);
 }
@@ -1064,7 +1090,8 @@ int fused_build(const sdq_plan_s* pl, int M) {
   if (dc.ring <= kFusePre) return 0;
   const size_t room = (size_t)(dc.ring - kFusePre) * slot;
   const size_t scratch = (size_t)M * dc.CB * kXtStride * sizeof(float);
-  const size_t poly = (size_t)2 * 16 * rt * (g.block + 8) * sizeof(uint16_t) + (size_t)pl->poly_bytes;
+  const size_t poly = (size_t)2 * 16 * rt * (g.block + 8) * sizeof(uint16_t) + (size_t)pl->poly_bytes +
+                      sizeof(int) * ((size_t)g.n_b + 2 * 16 * rt);
   if (pl->d_poly && scratch + poly <= room) return 2;
   return scratch <= room ? 1 : 0;
 }
