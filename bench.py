@@ -42,7 +42,7 @@ def parse():
     ap.add_argument("--impl", default="sdq", choices=["sdq", "reference"])
     ap.add_argument("--m", type=int, default=1, help="decode batch")
     ap.add_argument("--no-extras", action="store_true", help="skip encode/prefill/sweep/cpu legs")
-    ap.add_argument("--linears", default="", help="comma list of cfg4 linears to run (default: all 7)")
+    ap.add_argument("--linears", default="", help="comma list of llama-70b-layer linears to run (default: all 7)")
     ap.add_argument("--eager", action="store_true",
                     help="launch every step eagerly instead of replaying a CUDA graph (same kernels; "
                          "for profilers that cannot follow stream capture)")
@@ -344,7 +344,7 @@ def run_sdq(args, rank, world, dist):
         "n_gpus": world, "steps": args.steps, "warmup": max(3, args.warmup),
         "ms_per_step": round(ms_step, 5), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "u2-codes/e4m3-mma/f32-acc", "data": "synthetic",
-        "config": {"workload": "llama70b-layer decode (cfg4): q/o 8192x8192, k/v 1024x8192, "
+        "config": {"workload": "llama70b-layer decode: q/o 8192x8192, k/v 1024x8192, "
                                "gate/up 28672x8192, down 8192x28672; OSR 2 ternary B=128"
                                + (f" [only {args.linears}]" if args.linears else ""),
                    "decode_batch": M, "code_bytes_per_step": code_bytes,
@@ -440,7 +440,7 @@ def prefill_leg(P, W, torch, layers, stream, tf_burst, tf_sus, peak_src):
 # -------------------------------------------------------- oracle (CPU) legs
 class OracleSample:
     """Seeded inputs for the oracle's code-domain forward (decode, M=1) on
-    `rows` rows of every cfg4 linear, prepared once; `run()` times one pass."""
+    `rows` rows of every llama-70b-layer linear, prepared once; `run()` times one pass."""
 
     def __init__(self, rows):
         import numpy as np
@@ -482,13 +482,13 @@ def cpu_baseline_leg(sample_rows=256, min_secs=10.0):
     return {"value": round(smp.nbytes * passes / secs / 1e9, 4), "unit": "GB/s", "cores": cores,
             "kind": "oracle",
             "sample": f"oracle forward_code_domain (fp64 numpy), decode M=1, {sample_rows} rows of "
-                      f"each of the 7 cfg4 linears ({smp.nbytes} code bytes) x {passes} passes = "
+                      f"each of the 7 llama-70b-layer linears ({smp.nbytes} code bytes) x {passes} passes = "
                       f"{secs:.1f} s; numpy default threads on {cores} host cores"}
 
 
 def run_reference(args, rank, world):
     """The oracle as the reference arm: each step is the code-domain forward on
-    a bounded row sample of every cfg4 linear (GB/s of codes processed)."""
+    a bounded row sample of every llama-70b-layer linear (GB/s of codes processed)."""
     if rank != 0:
         return None
     rows = 64 if args.steps <= 2000 else 16
@@ -506,11 +506,11 @@ def run_reference(args, rank, world):
             "ms_per_step": round(secs / args.steps * 1e3, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic",
-            "config": {"workload": "llama70b-layer decode (cfg4), M=1; oracle on a bounded "
+            "config": {"workload": "llama70b-layer decode, M=1; oracle on a bounded "
                                    f"sample of {rows} rows per linear per step"},
             "cpu_baseline": {"value": round(val, 4), "unit": "GB/s", "cores": cores,
                              "kind": "oracle",
-                             "sample": f"{rows} rows of each of the 7 cfg4 linears per step"},
+                             "sample": f"{rows} rows of each of the 7 llama-70b-layer linears per step"},
             "e2e": {"value": round(val, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
 

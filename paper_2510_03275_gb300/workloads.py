@@ -8,22 +8,22 @@ The paper evaluates on pretrained OPT / LLaMA checkpoints with WikiText2 / C4
 (section 4.1); none of those are available, so synthetic weights with the
 same linear shapes stand in for them:
 
-* cfg0  one 256 x 512 linear, W ~ N(0, 0.02), B = 512, OSR 2, ternary, M = 1.
-* cfg1  OPT-125M decoder linears (q/k/v/o 768x768, fc1 3072x768, fc2
+* single-256x512  one 256 x 512 linear, W ~ N(0, 0.02), B = 512, OSR 2, ternary, M = 1.
+* opt-125m  OPT-125M decoder linears (q/k/v/o 768x768, fc1 3072x768, fc2
         768x3072), W ~ N(0, 0.02) with round(0.005 K) outlier input columns
         scaled x20, OSR 2.5, binary, M in {1, 16}.
-* cfg2  LLaMA-7B decoder linears (q/k/v/o 4096^2, gate/up 11008x4096, down
+* llama-7b-layer  LLaMA-7B decoder linears (q/k/v/o 4096^2, gate/up 11008x4096, down
         4096x11008), Student-t(5) scaled to std 0.02 times a per-row factor
         log-uniform in [0.5, 2], OSR 2, ternary, M in {1, 4, 16, 64}.
-* cfg3  LLaMA-13B 4-layer stack (q/k/v/o 5120^2, gate/up 13824x5120, down
+* llama-13b-4layers  LLaMA-13B 4-layer stack (q/k/v/o 5120^2, gate/up 13824x5120, down
         5120x13824), N(0, sigma_l) with sigma_l log-uniform in [0.01, 0.03]
         per linear, MultiOSR in {1.5, 2, 2.5, 3}, ternary, M = 8 and 2048.
-* cfg4  LLaMA-70B decoder layer (q/o 8192^2, k/v 1024x8192, gate/up
+* llama-70b-layer  LLaMA-70B decoder layer (q/o 8192^2, k/v 1024x8192, gate/up
         28672x8192, down 8192x28672), Student-t(5) scaled to std 0.015,
         OSR 2, ternary, M = 4096 (prefill) and 1..64 (decode).
 
 Activations: x ~ N(0, 1) rounded to bf16.  Hadamard sign vectors: +-1 drawn
-uniformly.  Seeds: ``20251003 + 1000 * cfg + linear`` (weights; activations
+uniformly.  Seeds: ``20251003 + 1000 * index + linear`` (weights; activations
 ``+ 250``; Hadamard signs ``+ 500``).  Matrices are (N, K) = (out, in).
 """
 from __future__ import annotations
@@ -83,10 +83,10 @@ def _llama_layer(cfg, hidden, ffn, kv, osr, dist, std, layer=0, prefix=""):
 
 
 def config(index: int, multiosr=None) -> Config:
-    """The synthetic workload ``index`` (0..4).  For cfg3 the per-linear OSR
+    """The synthetic workload ``index`` (0..4).  For llama-13b-4layers the per-linear OSR
     map comes from ``multiosr`` (a callable taking the list of (params,
     variance) per layer, see ``paper_2510_03275_gb300.multiosr``); without it
-    every cfg3 linear uses OSR 2."""
+    every llama-13b-4layers linear uses OSR 2."""
     if index == 0:
         c = Config(0, "single-256x512", 512, TERNARY, decode_batches=(1,))
         c.linears = [Linear("lin", 256, 512, Fraction(2), "normal", 0.02, _seed(0, 0))]
@@ -167,7 +167,7 @@ def _weight_rowblock(lin: Linear, b: int, rb: int) -> np.ndarray:
 
 
 def outlier_columns(lin: Linear) -> np.ndarray:
-    """The round(0.005 K) input columns scaled x20 in cfg1."""
+    """The round(0.005 K) input columns scaled x20 in opt-125m."""
     cnt = int(round(0.005 * lin.k_in))
     return np.sort(np.random.default_rng([lin.seed, 4242]).permutation(lin.k_in)[:cnt])
 

@@ -155,7 +155,7 @@ def test_pack_unpack_bit_exact(sdq, torch_cuda, q, n, keff):
 
 
 def test_pack_full_size_sampled_tiles(sdq, torch_cuda):
-    """cfg4 gate (28672 x 16384 codes): round trip, and a seeded sample of
+    """llama-70b-layer gate (28672 x 16384 codes): round trip, and a seeded sample of
     (tile, k group) slabs compared with the oracle's tiled layout of the same
     128 rows."""
     torch = torch_cuda
@@ -255,7 +255,7 @@ def test_forward_decode_small(sdq, torch_cuda, q, m, shape):
     assert err <= min(TOL, bound), err
 
 
-def test_forward_encoded_cfg0_and_cfg1(sdq, torch_cuda):
+def test_forward_encoded_single_and_opt125m(sdq, torch_cuda):
     """End to end: GPU encode -> pack -> forward vs the oracle's encode and
     fp64 dense forward x . W_hat^T on configs 0 and 1."""
     torch = torch_cuda
