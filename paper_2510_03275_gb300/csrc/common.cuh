@@ -281,21 +281,29 @@ __device__ __forceinline__ void call_record_fail(uint64_t* rec, uint64_t call) {
   atomicExch(reinterpret_cast<unsigned long long*>(rec), (unsigned long long)call);
 }
 
-// Split-K ticket of one row tile: bits 8..63 the call number, bits 0..7 the
+__device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;\n" ::: "memory"); }
+
+// Split-K ticket of one row tile: bits 16..63 the call number, bits 0..15 the
 // arrivals of that call.  A ticket that carries another call number counts
-// as empty, so tickets need no reset between calls: the first arrival of a
-// call installs (call, 1) by compare-and-swap, later ones add 1 (a ticket
-// that carries this call's number keeps it for the rest of the call).
-// Returns this CTA's arrival number (1..255), or 0 if the compare-and-swap
-// did not settle within its retry bound.
+// as empty, so tickets need no reset between calls.  One acq_rel fence (after
+// the CTA barrier that orders the other threads' partial stores before it)
+// publishes the CTA's partials; then every arrival adds 1, and an add that
+// found another call's number installs (call, 1) by compare-and-swap or
+// joins the call that another arrival installed meanwhile.  (Such adds never
+// carry into the call field: a call leaves at most 2 S arrivals in a ticket,
+// far below 2^16.)  The last arrival fences again before reading the other
+// CTAs' partials.  Returns this CTA's arrival number (1..S), or 0 if the
+// compare-and-swap did not settle within its retry bound.
 __device__ __forceinline__ uint32_t ticket_take(uint64_t* tk, uint64_t call) {
   unsigned long long* p = reinterpret_cast<unsigned long long*>(tk);
-  const unsigned long long mine = (unsigned long long)call << 8;
-  unsigned long long cur = *reinterpret_cast<volatile unsigned long long*>(p);
+  fence_acq_rel_gpu();
+  const unsigned long long old = atomicAdd(p, 1ull);
+  if ((old >> 16) == call) return (uint32_t)(old & 0xFFFFu) + 1;
+  unsigned long long cur = old + 1;   // another call's ticket, with our add in it
   for (int it = 0; it < 64; ++it) {
-    if ((cur >> 8) == call) return (uint32_t)((atomicAdd(p, 1ull) & 0xFFu) + 1);
-    const unsigned long long prev = atomicCAS(p, cur, mine + 1);
+    const unsigned long long prev = atomicCAS(p, cur, (call << 16) | 1ull);
     if (prev == cur) return 1;
+    if ((prev >> 16) == call) return (uint32_t)(atomicAdd(p, 1ull) & 0xFFFFu) + 1;
     cur = prev;
   }
   return 0;

@@ -934,20 +934,19 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       kc[0] += in0;
       kc[1] += in1;
       if (p.S > 1) {
-        // Split-K, per tile while the next tile's MMAs run: one thread fences
-        // (after the barrier that orders the other threads' partial stores
-        // before it) and takes the tile's ticket; the CTA with the last ticket
-        // sums the S partials in k-chunk order (deterministic): at once when
-        // that is one round of loads per thread, else after the main loop on
-        // all of the CTA's threads (the tiles a CTA finishes last come at the
-        // end of its rotated order).
+        // Split-K, per tile while the next tile's MMAs run: one thread takes
+        // the tile's ticket (after the barrier that orders the other threads'
+        // partial stores before the ticket's release fence); the CTA with the
+        // last ticket fences again and sums the S partials in k-chunk order
+        // (deterministic): at once for M = 1, else after the main loop on all
+        // of the CTA's threads (the tiles a CTA finishes last come at the end
+        // of its rotated order).
         named_bar_sync(2, 128);
         if (et == 0) {
-          __threadfence();
           const uint32_t n = ticket_take(p.cnt + prow + ut * p.P, p.call);
           if (n == 0) call_record_fail(p.rec, p.call);
           const bool won = n == (uint32_t)p.S;
-          if (won) __threadfence();
+          if (won) fence_acq_rel_gpu();
           const bool defer = won && !red_now && ut < 32 * kRedWords;
           if (defer) red_bits[ut >> 5] |= 1u << (ut & 31);
           last[0] = won && !defer;
