@@ -1025,7 +1025,18 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
   int sb = 0, nbuf = 0, dbase = 0;
   tmem_split(best.NP, &sb, &nbuf, &dbase);
   const int slot_bytes = sb * blk_bytes;
-  const double clk = 1.9e9, bw = 6.5e12, latency = 2.2e-6;   // loaded HBM latency
+  // M = 1 constants fitted to measured launches: each split-K tile costs
+  // its epilogue (partial stores, a release fence and a ticket round trip
+  // while the code stream loads HBM) beyond its MMAs, and the ring's copies
+  // see a longer loaded latency.  Fewer, longer tiles per CTA measured
+  // faster both alone and inside the 7-linear layer step (8192 x 8192:
+  // S = 4 instead of 9, 31.0 -> 27.5 us per launch); for 8192 x 28672 the
+  // configurations that were faster alone were slower inside the step, and
+  // these constants keep S = 19 there.  Larger batches keep the earlier
+  // constants.
+  const double clk = 1.9e9, bw = 6.5e12;
+  const double latency = M == 1 ? 3.0e-6 : 2.2e-6;             // loaded HBM latency
+  const double t_tile = M == 1 ? 0.5e-6 : 0.0;                 // per split-K tile
   const double t_mma = std::max(38.0, best.NP * 0.55) / clk;    // per MMA, two issuers
   const double code_bytes = (double)g.ntiles * kTileRows * g.k_eff_pad * g.bits / 8;
   double best_t = 1e30;
@@ -1054,7 +1065,7 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
       const int rounds = (kTileRows * M + kThreads - 1) / kThreads * ((S + 15) / 16);
       const double red = S <= 1 || now ? 0.0 : (double)((units + S - 1) / S) * rounds * 1.2e-6;
       const double tail = S > 1 ? 2.5e-6 + red : 0.0;
-      const double t_cta = units * (4.0 * CB * t_mma + spu * 90.0 / clk + 300.0 / clk);
+      const double t_cta = units * (4.0 * CB * t_mma + spu * 90.0 / clk + 300.0 / clk + (S > 1 ? t_tile : 0.0));
       const double t = std::max(t_cta, (code_bytes + part_bytes) / bw_eff) + tail;
       if (t < best_t * 0.999) {
         best_t = t;
