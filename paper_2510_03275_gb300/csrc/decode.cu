@@ -103,8 +103,8 @@ struct DecodeParams {
   int use_poly, poly_p, poly_q, poly_bytes, fwht;
   int64_t k_eff;
   int M, T, NP, S, P, CB, KB, ring, sb, nbuf, dbase;
-  int n_out, ntiles, ngroups, ternary, early;
-  uint32_t blk_bytes, slot_bytes, b_bytes;
+  int n_out, ntiles, ngroups, ternary, early, stream;
+  uint32_t blk_bytes, slot_bytes, b_bytes;   // b_bytes: resident image (0 when streamed)
 };
 
 // Bounded wait whose outcome is the same for all lanes of the warp (the
@@ -588,6 +588,9 @@ __device__ void build_b_operand(const DecodeParams& p, uint8_t* bop, float* xs, 
   named_bar_sync(3, kBuildThreads);
 }
 
+// kStream: the B operand comes with each stage (p.stream); one instantiation
+// per mode keeps the resident mode's code free of the streamed bookkeeping.
+template <bool kStream>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t c_full[kMaxRing], c_empty[kMaxRing];
@@ -622,7 +625,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   // Set-up spread over warps 1.. (warp 0 allocates TMEM meanwhile).
   if (warp == 1 && lane < p.ring) {
     mbar_init(&c_full[lane], 1);
-    mbar_init(&c_empty[lane], 4);   // one arrival per expander warp
+    mbar_init(&c_empty[lane], kStream ? 5 : 4);   // one arrival per expander warp (+ the MMAs' commit)
   } else if (warp == 2) {
     if (lane < 2 * kSlots) {
       mbar_init(&a_full[lane], 4);
@@ -669,7 +672,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       // operand: after its first two stages when the codes may be read before
       // the preceding grid is done, before everything otherwise.
       int last_i = -1;
-      bool b_loaded = warp != 0 || p.fused;   // fused: the expanders build it
+      bool b_loaded = warp != 0 || p.fused || kStream;   // fused: the expanders build it
+      if (kStream && warp == 0) mbar_arrive(&b_full);   // streamed: nothing resident to wait for
       // Fused: the first kFusePre stages go out at once, the rest once the B
       // operand is built, so that the builders' loads do not queue behind a
       // full ring of code copies.
@@ -698,8 +702,16 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         const uint8_t* src = reinterpret_cast<const uint8_t*>(p.codes) +
                              ((size_t)tile * p.KB + kb0 + b0) * p.blk_bytes;
         const uint32_t bytes = (uint32_t)(b1 - b0) * p.blk_bytes;
-        mbar_expect_tx(&c_full[slot], bytes);
-        bulk_g2s_hint(ring + (size_t)slot * p.slot_bytes, src, bytes, &c_full[slot], pol);
+        uint8_t* dst = ring + (size_t)slot * p.slot_bytes;
+        if constexpr (kStream) {   // the stage's B rows behind the slot's code area
+          const uint32_t bb = (uint32_t)(b1 - b0) * p.NP * 128;
+          mbar_expect_tx(&c_full[slot], bytes + bb);
+          bulk_g2s_hint(dst, src, bytes, &c_full[slot], pol);
+          bulk_g2s(dst + (size_t)p.sb * p.blk_bytes, p.bimg + (size_t)(kb0 + b0) * p.NP * 128, bb, &c_full[slot]);
+        } else {
+          mbar_expect_tx(&c_full[slot], bytes);
+          bulk_g2s_hint(dst, src, bytes, &c_full[slot], pol);
+        }
         last_i = i;
         j += kProducers;
         while (j >= spu) { j -= spu; ++u; }
@@ -737,6 +749,11 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       while (j >= spu) { j -= spu; ++u; }
       bool first = true;
       uint32_t dt = 0;
+      int last_c = -1;   // last stage whose slot this thread released by commit
+      // streamed: B rows of stage i in ring slot i mod ring, behind its codes
+      const uint64_t sd0 = sw128_desc(sbase + p.b_bytes + (uint32_t)p.sb * p.blk_bytes);
+      const uint64_t sstep = (uint64_t)(p.slot_bytes >> 4);
+      int slot = e;
       for (int i = e, jj = 0; i < nstages && ok; i += 2, ++jj) {
         if (first) {
           buf = p.nbuf == 2 ? (k & 1) : 0;
@@ -751,7 +768,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         if (!ok) break;
         tc_fence_after();
         const int b0 = sblk[j], nb = sblk[j + 1] - b0;
-        uint64_t bd = bd0 + (uint64_t)b0 * bstep;
+        uint64_t bd;
+        if constexpr (kStream) bd = sd0 + (uint64_t)slot * sstep;
+        else bd = bd0 + (uint64_t)b0 * bstep;
         uint32_t at = abase + (uint32_t)(jj & 1) * aslot;
         for (int bb = 0; bb < nb; ++bb, at += 32, bd += bstep) {
           umma_f8_ts(dt, at, bd, idesc, (first && bb == 0) ? 0u : 1u);
@@ -760,6 +779,12 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
           umma_f8_ts(dt, at + 24, bd + 6, idesc, 1u);
         }
         umma_commit(&a_empty[a]);
+        if constexpr (kStream) {   // the slot's B rows are free once these MMAs are done
+          umma_commit(&c_empty[slot]);
+          last_c = i;
+          slot += 2;
+          if (slot >= p.ring) slot -= p.ring;
+        }
         const int u0 = u;
         j += 2;
         while (j >= spu) { j -= spu; ++u; }
@@ -776,6 +801,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       const int njs = (nstages - e + 1) / 2;   // stages of this pipeline
       for (int jj = max(0, njs - kSlots); jj < njs; ++jj)
         if (!mbar_wait(&a_empty[kSlots * e + jj % kSlots], (jj / kSlots) & 1)) ok = false;
+      // Streamed B: the slot commits of the last stages, which no producer
+      // waits for (the expanders arrived before these stages' MMAs).
+      for (int i = last_c; i >= 0 && i + p.ring >= nstages; i -= 2)
+        if (!mbar_wait(&c_empty[i % p.ring], (i / p.ring) & 1)) ok = false;
     }
   } else if (warp < kEpiWarp0) {
     // ------------------------------------------------------------ expanders
@@ -1040,11 +1069,17 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
   const double t_mma = std::max(38.0, best.NP * 0.55) / clk;    // per MMA, two issuers
   const double code_bytes = (double)g.ntiles * kTileRows * g.k_eff_pad * g.bits / 8;
   double best_t = 1e30;
+  // Streamed B (batches past the one-kernel route): each stage's slot holds
+  // its blocks' B rows too, so chunks are not bounded by a resident image
+  // and the split-K partials (S M N floats) can stay small.
+  const int nmode = M > kMaxFuseM ? 2 : 1;
+  for (int stream = 0; stream < nmode; ++stream)
   for (int S = 1; S <= std::min(KB, sms); ++S) {
     const int CB = (KB + S - 1) / S;
     if ((S - 1) * CB >= KB) continue;                      // no empty chunk
-    const int b_bytes = CB * best.NP * 128;
-    int ring = std::min(kMaxRing, (kSmemMax - 2048 - b_bytes) / slot_bytes);
+    const int b_bytes = stream ? 0 : CB * best.NP * 128;
+    const int sbytes = stream ? sb * (blk_bytes + best.NP * 128) : slot_bytes;
+    int ring = std::min(kMaxRing, (kSmemMax - 2048 - b_bytes) / sbytes);
     ring -= ring % kExpSets;          // each ring slot belongs to one expander set
     if (ring < kExpSets) continue;
     const int spu = std::max((CB + sb - 1) / sb, std::min(2, CB));
@@ -1052,7 +1087,7 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
     for (int P = 1; P <= std::min(g.ntiles, sms / S); ++P) {
       const int grid = S * P;
       const int units = (g.ntiles + P - 1) / P;
-      const double inflight = (double)grid * ring * slot_bytes;
+      const double inflight = (double)grid * ring * slot_bytes;   // code bytes in flight
       const double bw_eff = std::min(bw, inflight / latency);
       const double part_bytes = S > 1 ? 8.0 * S * M * g.ntiles * kTileRows : 0.0;
       // split-K: the CTA that sums a tile reads S partials for each of its
@@ -1069,8 +1104,8 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
       const double t = std::max(t_cta, (code_bytes + part_bytes) / bw_eff) + tail;
       if (t < best_t * 0.999) {
         best_t = t;
-        best.S = S; best.P = P; best.CB = CB; best.ring = ring;
-        best.smem = std::max<size_t>(kSmemMin, 1024 + (size_t)b_bytes + (size_t)ring * slot_bytes);
+        best.S = S; best.P = P; best.CB = CB; best.ring = ring; best.stream = stream;
+        best.smem = std::max<size_t>(kSmemMin, 1024 + (size_t)b_bytes + (size_t)ring * sbytes);
       }
     }
   }
@@ -1132,18 +1167,25 @@ cudaError_t launch_decode(const sdq_plan_s* pl, const uint32_t* codes, const flo
   p.fwht = pl->desc.hadamard != 0;
   p.K = g.k_in; p.B = g.block; p.n_b = g.n_b; p.k_eff = g.k_eff;
   if (p.fused) early = 0;   // x and the codes may come from the preceding grid
+  p.stream = !p.fused && dc.stream;
+  if (p.stream) early = 0;  // every stage carries B rows written by the preceding grid
   p.M = M; p.T = dc.T; p.NP = dc.NP; p.S = dc.S; p.P = dc.P; p.CB = dc.CB;
   p.KB = (int)(g.k_eff_pad / kBlk); p.ring = dc.ring;
   tmem_split(dc.NP, &p.sb, &p.nbuf, &p.dbase);
   p.n_out = g.n_out; p.ntiles = g.ntiles; p.ngroups = g.ngroups; p.ternary = g.bits == 2;
   p.early = early;
   p.blk_bytes = (uint32_t)(kTileRows * kBlk * g.bits / 8);
-  p.slot_bytes = p.sb * p.blk_bytes;
-  p.b_bytes = (uint32_t)(dc.CB * dc.NP * 128);
-  static std::atomic<int> smem_set[64];   // per device: limit raised to kSmemMax + 1 KB
-  cudaError_t e = smem_limit_once(decode_kernel, kSmemMax + 1024, pl->device, smem_set);
+  p.slot_bytes = p.sb * (p.blk_bytes + (p.stream ? (uint32_t)dc.NP * 128 : 0u));
+  p.b_bytes = p.stream ? 0u : (uint32_t)(dc.CB * dc.NP * 128);
+  static std::atomic<int> smem_set[2][64];   // per mode and device: limit raised to kSmemMax + 1 KB
+  if (p.stream) {
+    cudaError_t e = smem_limit_once(decode_kernel<true>, kSmemMax + 1024, pl->device, smem_set[1]);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(decode_kernel<true>, dim3(dc.S * dc.P), dim3(kThreads), dc.smem, st, p);
+  }
+  cudaError_t e = smem_limit_once(decode_kernel<false>, kSmemMax + 1024, pl->device, smem_set[0]);
   if (e != cudaSuccess) return e;
-  return launch_pdl(decode_kernel, dim3(dc.S * dc.P), dim3(kThreads), dc.smem, st, p);
+  return launch_pdl(decode_kernel<false>, dim3(dc.S * dc.P), dim3(kThreads), dc.smem, st, p);
 }
 
 }  // namespace sdq

@@ -80,6 +80,8 @@ struct DecodeConfig {
   int M, T, NP;           // batch, e4m3 terms per activation, MMA N (M*T rounded up to 16)
   int S, P, CB;           // k chunks, CTAs per k chunk, 128-code blocks per chunk
   int ring;               // code stages in the shared-memory ring
+  int stream;             // 1: each stage's slot also carries its blocks' B operand
+                          // rows (no resident per-chunk image; larger batches)
   size_t smem;            // dynamic shared memory of the decode kernel
 };
 
