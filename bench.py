@@ -368,17 +368,29 @@ def run_sdq(args, rank, world, dist):
         "encode": {"ms_per_layer": round(enc_ms, 3), "what": "sdq_encode_rows + sdq_pack, 7 linears"},
     }
     if not args.no_extras and rank == 0:
-        out["decode_sweep"] = decode_sweep(P, W, torch, layers, stream)
+        out["decode_sweep"] = decode_sweep(P, W, torch, layers, stream, hbm, tf_burst, peak_src)
         out["prefill"] = prefill_leg(P, W, torch, layers, stream, tf_burst, tf_sus, peak_src)
         out["cpu_baseline"] = cpu_baseline_leg()
     return out
 
 
-def decode_sweep(P, W, torch, layers, stream):
+def sweep_roofline(code_bytes, ops, ms, hbm_gbs, fp8_tflops):
+    """Bound and fraction of one batch size of the decode sweep: the time the
+    codes need at the HBM peak against the time the algorithmic add/sub work
+    (2 M N K_eff flop-equivalents) needs at the fp8 tensor peak; whichever is
+    longer is the bound, and frac = that time / the measured time."""
+    t_hbm = code_bytes / (hbm_gbs * 1e9)
+    t_ten = ops / (fp8_tflops * 1e12)
+    bound, t = ("hbm", t_hbm) if t_hbm >= t_ten else ("tensor", t_ten)
+    return {"bound": bound, "frac": round(t / (ms * 1e-3), 4)}
+
+
+def decode_sweep(P, W, torch, layers, stream, hbm_gbs, tf_bf16, peak_src):
     import numpy as np
-    res = {}
+    res, roof = {}, {}
+    fp8 = 2.0 * tf_bf16   # e4m3 dense peak: the measured bf16 peak x the nominal 2x ratio
     for M in (1, 2, 4, 8, 16, 32, 64):
-        tot_b, tot_ms = 0, 0.0
+        tot_b, tot_ms, tot_ops = 0, 0.0, 0.0
         for lay in layers:
             lin = lay["lin"]
             x = torch.from_numpy(W.activations(lin, M).view(np.int16)).view(torch.bfloat16).cuda()
@@ -399,9 +411,13 @@ def decode_sweep(P, W, torch, layers, stream):
             torch.cuda.synchronize()
             tot_ms += sum(a.elapsed_time(b) for a, b in evs) / len(evs)
             tot_b += lay["code_bytes"]
+            tot_ops += 2.0 * M * lin.n_out * lay["plan"].k_eff
         res[str(M)] = round(tot_b / (tot_ms * 1e-3) / 1e9, 1)
+        roof[str(M)] = sweep_roofline(tot_b, tot_ops, tot_ms, hbm_gbs, fp8)
     return {"unit": "weight GB/s (sdq_linear_forward per linear, inputs on the device, per batch size)",
-            "values": res}
+            "values": res, "roofline": roof,
+            "peaks": {"hbm_gbs": hbm_gbs, "fp8_tflops": fp8,
+                      "source": peak_src + " (fp8 = bf16 x 2, nominal ratio)"}}
 
 
 def prefill_leg(P, W, torch, layers, stream, tf_burst, tf_sus, peak_src):

@@ -55,6 +55,20 @@ def test_job_rate_counts_all_ranks():
     assert bench.max_over_ranks(2.5, None) == 2.5
 
 
+def test_sweep_roofline_bound_and_fraction():
+    """Per-batch decode roofline: the longer of the HBM time of the codes and
+    the fp8 tensor time of the 2 M N K_eff add/sub work bounds the batch."""
+    sys.path.insert(0, ROOT)
+    import bench
+    # 1 GB of codes at 1000 GB/s = 1 ms; 2 GFLOP at 1 TFLOP/s = 2 ms; measured 4 ms
+    assert bench.sweep_roofline(1e9, 2e9, 4.0, 1000.0, 1.0) == {"bound": "tensor", "frac": 0.5}
+    assert bench.sweep_roofline(1e9, 0.5e9, 2.0, 1000.0, 1.0) == {"bound": "hbm", "frac": 0.5}
+    # the LLaMA-70B layer at M = 64 against this pool's peaks is still HBM-bound
+    codes, ops = 427819008, 2.0 * 64 * 427819008 * 4   # 4 codes per byte (2-bit ternary)
+    r = bench.sweep_roofline(codes, ops, 1.0, 6783.5, 2 * 1903.9)
+    assert r["bound"] == "hbm"
+
+
 def test_reference_arm_under_torchrun_world2():
     env = dict(os.environ, CUDA_VISIBLE_DEVICES="")
     cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node=2",
