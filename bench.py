@@ -22,6 +22,7 @@ import argparse
 import hashlib
 import json
 import os
+import re
 import subprocess
 import sys
 import threading
@@ -133,19 +134,39 @@ class ClockSampler:
                 "samples": len(sel)}
 
 
+def code_text(src):
+    """C++/CUDA source without comments and empty lines, runs of blanks
+    collapsed: the part of a kernel source that a profile depends on."""
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    out = []
+    for line in src.splitlines():
+        i = line.find("//")
+        if i >= 0 and line.count('"', 0, i) % 2 == 0:
+            line = line[:i]
+        line = " ".join(line.split())
+        if line:
+            out.append(line)
+    return "\n".join(out) + "\n"
+
+
+def source_hash(src_files):
+    h = hashlib.sha256()
+    for p in src_files:
+        with open(p) as f:
+            h.update(code_text(f.read()).encode())
+    return h.hexdigest()[:16]
+
+
 def profile_traffic(src_files):
     """dram bytes per launch from the committed ncu summary, if it was taken
-    on the current kernel source (sha256 recorded in the summary)."""
+    on the current kernel code (a sha256 of the sources without comments,
+    recorded in the summary)."""
     try:
         with open(PROFILE_DECODE) as f:
             txt = f.read()
     except OSError:
         return None, None
-    h = hashlib.sha256()
-    for p in src_files:
-        with open(p, "rb") as f:
-            h.update(f.read())
-    cur = h.hexdigest()[:16]
+    cur = source_hash(src_files)
     vals = {}
     for line in txt.splitlines():
         if ":" in line and line.strip().startswith(("source_sha256", "traffic_bytes_per_launch",

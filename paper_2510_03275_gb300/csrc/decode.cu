@@ -15,10 +15,13 @@
 //   B (smem)  the activations as T e4m3 terms per batch row m:
 //             x_tilde[m] * 2^-e_m = sum_t 16^-t q_t[m] (e_m from a bound on |x_tilde[m]|),
 //             N = M*T rows rounded up to 16, K-major, 128-byte swizzle:
-//             either written for all of K by the decode prepare kernel, each
-//             CTA copying the part of its k chunk once, or (small batches,
-//             `fused`) built by the CTA's expander warps for its k chunk from
-//             x itself, with a scale 2^e_m of its own (build_b_operand)
+//             either written for all of K by the decode prepare kernel and
+//             then copied by each CTA, the part of its k chunk at once
+//             (resident) or each stage's blocks with the stage's codes
+//             (streamed, larger batches: decode_kernel<true>), or (small
+//             batches, `fused`) built by the CTA's expander warps for its k
+//             chunk from x itself, with a scale 2^e_m of its own
+//             (build_b_operand)
 //   D (TMEM)  fp32, 128 lanes x NP columns
 // so that y[m, r] = alpha_r / 2 * 2^e_m * sum_t 16^-t D[r, m T + t].
 //
@@ -35,9 +38,9 @@
 // CTA (k chunk s, row set p) of one SM, 24 warps:
 //   warps 0, 1    lane 0 of warp e streams pipeline e's stages (one 128-row
 //                 tile x up to sb * 128 codes = contiguous slabs of the tiled
-//                 layout) into its shared-memory ring slots with bulk copies;
-//                 warp 0 also owns the TMEM allocation and copies the chunk's
-//                 B operand
+//                 layout, plus their B rows when streamed) into its
+//                 shared-memory ring slots with bulk copies; warp 0 also owns
+//                 the TMEM allocation and copies a resident B operand
 //   warps 2, 3    lane 0 of warp 2 + e issues pipeline e's MMAs, commits to
 //                 the stage's TMEM slot and, after its last stage of a row
 //                 tile, to its accumulator

@@ -69,6 +69,18 @@ def test_sweep_roofline_bound_and_fraction():
     assert r["bound"] == "hbm"
 
 
+def test_profile_hash_ignores_comments_only():
+    """The ncu summary stays valid across comment edits of the kernel source,
+    not across code edits (a string holding // is code)."""
+    sys.path.insert(0, ROOT)
+    import bench
+    a = 'int f() {  // note\n  /* block\n comment */ return 1;\n}\n'
+    b = '// header\nint f() {\n\n  return 1;   \n}\n'
+    assert bench.code_text(a) == bench.code_text(b)
+    assert bench.code_text('int g = 2;\n') != bench.code_text('int g = 3;\n')
+    assert "//x" in bench.code_text('const char* s = "//x";\n')
+
+
 def test_reference_arm_under_torchrun_world2():
     env = dict(os.environ, CUDA_VISIBLE_DEVICES="")
     cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node=2",
