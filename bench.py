@@ -507,6 +507,23 @@ def _cores():
     return len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
 
 
+def _host_threads():
+    """The host the oracle runs on: logical CPUs, the ones this process may
+    use, and the BLAS thread pools numpy would use (threadpoolctl when it is
+    installed, else the environment's thread settings)."""
+    import numpy  # noqa: F401  (loads the BLAS whose pools are reported)
+    info = {"cpu_count": os.cpu_count(), "affinity": _cores()}
+    pools = []
+    try:
+        from threadpoolctl import threadpool_info
+        pools = [{"api": d.get("internal_api"), "threads": d.get("num_threads")} for d in threadpool_info()]
+    except Exception:
+        pass
+    info["blas"] = pools or {k: os.environ.get(k, "unset") for k in
+                             ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS")}
+    return info
+
+
 def cpu_baseline_leg(sample_rows=256, min_secs=10.0):
     """The oracle timed on the host cores: repeated passes over a bounded
     sample until about `min_secs` of CPU work."""
@@ -517,7 +534,7 @@ def cpu_baseline_leg(sample_rows=256, min_secs=10.0):
         passes += 1
     cores = _cores()
     return {"value": round(smp.nbytes * passes / secs / 1e9, 4), "unit": "GB/s", "cores": cores,
-            "kind": "oracle",
+            "kind": "oracle", "host": _host_threads(),
             "sample": f"oracle forward_code_domain (fp64 numpy), decode M=1, {sample_rows} rows of "
                       f"each of the 7 llama-70b-layer linears ({smp.nbytes} code bytes) x {passes} passes = "
                       f"{secs:.1f} s; numpy default threads on {cores} host cores"}
@@ -546,7 +563,7 @@ def run_reference(args, rank, world):
             "config": {"workload": "llama70b-layer decode, M=1; oracle on a bounded "
                                    f"sample of {rows} rows per linear per step"},
             "cpu_baseline": {"value": round(val, 4), "unit": "GB/s", "cores": cores,
-                             "kind": "oracle",
+                             "kind": "oracle", "host": _host_threads(),
                              "sample": f"{rows} rows of each of the 7 llama-70b-layer linears per step"},
             "e2e": {"value": round(val, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
