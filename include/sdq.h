@@ -136,6 +136,28 @@ size_t sdq_workspace_bytes(sdq_plan plan, int32_t M);
 int sdq_build_tables(const sdq_layer_desc* desc, const int8_t* had_signs,
                      float* a_enc_host, float* g_host);
 
+/* Host-only (no GPU needed): the polyphase table of D^T that the decode
+ * kernel's own activation transform reads (sdq_linear_forward at small
+ * batches; section 3.5 with Algorithm 1's Resample).  With n_b / block =
+ * p / q in lowest terms, band-limited resampling commutes with a cyclic
+ * shift of q inputs, so row r + p m of D^T (n_b x block, the adjoint of the
+ * decimation) is row r shifted by q m: D^T[r + p m][i] =
+ * D^T[r][(i - q m) mod block].  Writes p and q (p_out, q_out) and the
+ * table's size in uint32 words (words_out; each may be NULL), and, when
+ * `table_host` is not NULL, the table: for r < p and d < 2 block, words
+ * 2 (r (2 block + 8) + d) and +1 = the bf16x2 pair (D^T[r][d mod block],
+ * D^T[r][(d + 1) mod block]) (first element in the low half) and the bf16x2
+ * pair of their remainders after the first rounding; rows padded to
+ * 2 block + 8 entries with zeros; then `block` fp32 bit patterns
+ * d_k / sqrt(block) (1 without the Hadamard rotation).  Returns
+ * SDQ_ERR_UNSUPPORTED when the kernel would not use a table (block not a
+ * multiple of 16 or above 256, n_b not a multiple of 8, more than 16 KB of
+ * entries, or D^T not polyphase to 1e-12 of its largest entry),
+ * SDQ_ERR_WORKSPACE when capacity_words is too small, and the errors of
+ * sdq_build_tables. */
+int sdq_build_poly_table(const sdq_layer_desc* desc, const int8_t* had_signs, uint32_t* table_host,
+                         size_t capacity_words, size_t* words_out, int32_t* p_out, int32_t* q_out);
+
 /* Algorithm 1 without compensation, on every row of W (device, fp32,
  * n_out x k_in row-major).  Writes codes in the plain layout
  * (sdq_plain_bytes) and alpha (device, fp32[n_out]).  Bit-exact contract:

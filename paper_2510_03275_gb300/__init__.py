@@ -21,7 +21,7 @@ __all__ = [
     "SDQ_OK", "SDQ_BINARY", "SDQ_TERNARY", "SDQ_ALPHA_MAXABS", "SDQ_ALPHA_MEANABS",
     "SdqError", "LayerDesc", "lib", "library_path",
     "sdq_plan_create", "sdq_plan_destroy", "sdq_k_eff", "sdq_plain_bytes", "sdq_tiled_bytes",
-    "sdq_workspace_bytes", "sdq_build_tables", "sdq_encode_rows", "sdq_pack", "sdq_unpack",
+    "sdq_workspace_bytes", "sdq_build_tables", "sdq_build_poly_table", "sdq_encode_rows", "sdq_pack", "sdq_unpack",
     "sdq_prep_activations", "sdq_contract", "sdq_linear_forward", "sdq_read_prep",
     "sdq_workspace_status", "sdq_linear_forward_noalloc", "sdq_noalloc_scratch_bytes",
     "sdq_forward_kernels", "sdq_status_string", "Plan",
@@ -81,6 +81,8 @@ _SIGS = {
     "sdq_tiled_bytes": (_sz, [ctypes.POINTER(_Desc)]),
     "sdq_workspace_bytes": (_sz, [_vp, _i32]),
     "sdq_build_tables": (ctypes.c_int, [ctypes.POINTER(_Desc), _vp, _vp, _vp]),
+    "sdq_build_poly_table": (ctypes.c_int, [ctypes.POINTER(_Desc), _vp, _vp, _sz, ctypes.POINTER(_sz),
+                                            ctypes.POINTER(_i32), ctypes.POINTER(_i32)]),
     "sdq_encode_rows": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp]),
     "sdq_pack": (ctypes.c_int, [_vp, _vp, _vp, _vp]),
     "sdq_unpack": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp]),
@@ -173,6 +175,23 @@ def sdq_build_tables(desc: LayerDesc, had_signs=None):
                                 a.ctypes.data_as(_vp), g.ctypes.data_as(_vp))
     _check(st, "sdq_build_tables")
     return a, g
+
+
+def sdq_build_poly_table(desc: LayerDesc, had_signs=None):
+    """Host-only: (table as a uint32 numpy array, p, q) -- the polyphase table
+    of D^T the decode kernel's own activation transform reads (layout in
+    include/sdq.h); raises SdqError when the structure does not apply."""
+    import numpy as np
+    words, pp, qq = _sz(0), _i32(0), _i32(0)
+    signs = None if had_signs is None else np.ascontiguousarray(had_signs, dtype=np.int8)
+    sp = None if signs is None else signs.ctypes.data_as(_vp)
+    _check(lib().sdq_build_poly_table(ctypes.byref(desc.c()), sp, None, 0, ctypes.byref(words),
+                                      ctypes.byref(pp), ctypes.byref(qq)), "sdq_build_poly_table")
+    table = np.zeros(words.value, np.uint32)
+    _check(lib().sdq_build_poly_table(ctypes.byref(desc.c()), sp, table.ctypes.data_as(_vp), table.size,
+                                      ctypes.byref(words), ctypes.byref(pp), ctypes.byref(qq)),
+           "sdq_build_poly_table")
+    return table, pp.value, qq.value
 
 
 def sdq_encode_rows(plan, W, codes_plain, alpha, stream=None):

@@ -34,6 +34,51 @@ double host_bf16_value(uint16_t b) {
 
 int cuda_status(cudaError_t e) { return e == cudaSuccess ? SDQ_OK : SDQ_ERR_CUDA; }
 
+// The polyphase table of D^T (layout: poly_stride in sdq_internal.h) from
+// D^T itself (n_b x B, fp64).  Sets p, q (n_b / B = p / q in lowest terms)
+// always; fills `poly` and returns SDQ_OK when the decode kernel can use it:
+// B a multiple of 16 up to kMaxPolyBlock, n_b a multiple of 8, the entries
+// within kMaxPolyBytes, and D^T polyphase to 1e-12 of its largest entry.
+int build_poly_table(const Geometry& g, const sdq_layer_desc* desc, const int8_t* had_signs,
+                     const std::vector<double>& dt, std::vector<uint32_t>* poly, int* p_out, int* q_out) {
+  const int B = g.block, pp = g.n_b / std::gcd(g.n_b, g.block), pq = g.block / std::gcd(g.n_b, g.block);
+  *p_out = pp;
+  *q_out = pq;
+  const size_t poly_bytes = (size_t)pp * poly_stride(B) * 8;
+  if (B % 16 != 0 || g.n_b % 8 != 0 || B > kMaxPolyBlock || poly_bytes > (size_t)kMaxPolyBytes)
+    return SDQ_ERR_UNSUPPORTED;
+  const size_t tab = (size_t)g.n_b * B;
+  double mx = 0.0, dev = 0.0;
+  for (size_t i = 0; i < tab; ++i) mx = std::max(mx, std::fabs(dt[i]));
+  for (int j = 0; j < g.n_b; ++j)
+    for (int i = 0; i < B; ++i) {
+      const int src = (int)(((int64_t)i - (int64_t)pq * (j / pp)) % B + B) % B;
+      dev = std::max(dev, std::fabs(dt[(size_t)j * B + i] - dt[(size_t)(j % pp) * B + src]));
+    }
+  if (dev > 1e-12 * mx) return SDQ_ERR_UNSUPPORTED;
+  poly->assign(poly_bytes / 4 + B, 0u);
+  for (int r = 0; r < pp; ++r)
+    for (int d = 0; d < 2 * B; ++d) {
+      uint32_t hi = 0, lo = 0;
+      for (int h = 0; h < 2; ++h) {   // taps d and d + 1 (mod B): low and high halves
+        double v = dt[(size_t)r * B + (d + h) % B];
+        if (std::fabs(v) < 0x1p-46) v = 0.0;   // fp64 noise on exact zeros
+        const uint16_t vh = host_bf16(v), vl = host_bf16(v - host_bf16_value(vh));
+        hi |= (uint32_t)vh << (16 * h);
+        lo |= (uint32_t)vl << (16 * h);
+      }
+      const size_t e = (size_t)r * poly_stride(B) + d;
+      (*poly)[2 * e] = hi;
+      (*poly)[2 * e + 1] = lo;
+    }
+  const bool had = desc->hadamard != 0;
+  for (int k = 0; k < B; ++k) {
+    const float sk = had ? (float)((had_signs ? (double)had_signs[k] : 1.0) / std::sqrt((double)B)) : 1.0f;
+    std::memcpy(&(*poly)[poly_bytes / 4 + k], &sk, 4);
+  }
+  return SDQ_OK;
+}
+
 }  // namespace
 
 uint64_t next_call_number() {
@@ -124,41 +169,11 @@ extern "C" int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_sig
   }
 
   // Polyphase table of D^T (poly_stride) when D^T has that structure to fp64
-  // rounding and the table is small.
+  // rounding and the table is small (else the decode build streams G).
   std::vector<uint32_t> poly;
-  const int B = g.block, pp = g.n_b / std::gcd(g.n_b, g.block), pq = g.block / std::gcd(g.n_b, g.block);
-  const size_t poly_bytes = (size_t)pp * poly_stride(B) * 8;
-  if (B % 16 == 0 && g.n_b % 8 == 0 && B <= kMaxPolyBlock && poly_bytes <= (size_t)kMaxPolyBytes) {
-    double mx = 0.0, dev = 0.0;
-    for (size_t i = 0; i < tab; ++i) mx = std::max(mx, std::fabs(dt[i]));
-    for (int j = 0; j < g.n_b; ++j)
-      for (int i = 0; i < B; ++i) {
-        const int src = (int)(((int64_t)i - (int64_t)pq * (j / pp)) % B + B) % B;
-        dev = std::max(dev, std::fabs(dt[(size_t)j * B + i] - dt[(size_t)(j % pp) * B + src]));
-      }
-    if (dev <= 1e-12 * mx) {
-      poly.assign(poly_bytes / 4 + B, 0u);
-      for (int r = 0; r < pp; ++r)
-        for (int d = 0; d < 2 * B; ++d) {
-          uint32_t hi = 0, lo = 0;
-          for (int h = 0; h < 2; ++h) {   // taps d and d + 1 (mod B): low and high halves
-            double v = dt[(size_t)r * B + (d + h) % B];
-            if (std::fabs(v) < 0x1p-46) v = 0.0;   // fp64 noise on exact zeros
-            const uint16_t vh = host_bf16(v), vl = host_bf16(v - host_bf16_value(vh));
-            hi |= (uint32_t)vh << (16 * h);
-            lo |= (uint32_t)vl << (16 * h);
-          }
-          const size_t e = (size_t)r * poly_stride(B) + d;
-          poly[2 * e] = hi;
-          poly[2 * e + 1] = lo;
-        }
-      const bool had = desc->hadamard != 0;
-      for (int k = 0; k < B; ++k) {
-        const float sk = had ? (float)((had_signs ? (double)had_signs[k] : 1.0) / std::sqrt((double)B)) : 1.0f;
-        std::memcpy(&poly[poly_bytes / 4 + k], &sk, 4);
-      }
-    }
-  }
+  int pp = 0, pq = 0;
+  if (build_poly_table(g, desc, had_signs, dt, &poly, &pp, &pq) != SDQ_OK) poly.clear();
+  const size_t poly_bytes = (size_t)pp * poly_stride(g.block) * 8;
 
   sdq_plan_s* p = new (std::nothrow) sdq_plan_s();
   if (!p) return SDQ_ERR_ALLOC;
@@ -190,6 +205,29 @@ extern "C" int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_sig
   }
   for (int M = 1; M <= kMaxDecodeM; ++M) p->dcfg[M] = decode_config_search(p, M);
   *out = p;
+  return SDQ_OK;
+}
+
+extern "C" int sdq_build_poly_table(const sdq_layer_desc* desc, const int8_t* had_signs, uint32_t* table,
+                                    size_t capacity_words, size_t* words_out, int32_t* p_out, int32_t* q_out) {
+  if (!desc) return SDQ_ERR_INVALID_ARG;
+  Geometry g;
+  int st = validate(desc, &g);
+  if (st != SDQ_OK) return st;
+  std::vector<double> dt((size_t)g.n_b * g.block);
+  st = build_tables(desc, had_signs, nullptr, nullptr, dt.data());
+  if (st != SDQ_OK) return st;
+  std::vector<uint32_t> poly;
+  int pp = 0, pq = 0;
+  st = build_poly_table(g, desc, had_signs, dt, &poly, &pp, &pq);
+  if (p_out) *p_out = pp;
+  if (q_out) *q_out = pq;
+  if (words_out) *words_out = poly.size();
+  if (st != SDQ_OK) return st;
+  if (table) {
+    if (capacity_words < poly.size()) return SDQ_ERR_WORKSPACE;
+    std::memcpy(table, poly.data(), sizeof(uint32_t) * poly.size());
+  }
   return SDQ_OK;
 }
 

@@ -101,3 +101,52 @@ def test_tables_match_oracle(sdq, block, osr, signs, had):
     nb = d.n_b
     assert np.array_equal(a, O.encode_table(block, nb, signs, bool(had)))
     assert np.abs(g - O.decode_table(block, nb, signs, bool(had))).max() < 1e-6
+
+
+def _bf16(h):
+    return (np.asarray(h, np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+@pytest.mark.parametrize("block,osr", [(16, Fraction(5, 2)), (128, Fraction(2)), (128, Fraction(3, 2)),
+                                       (64, Fraction(9, 4)), (256, Fraction(2)), (32, Fraction(1))])
+@pytest.mark.parametrize("had", [1, 0])
+def test_poly_table_matches_oracle(sdq, block, osr, had):
+    """The decode kernel's polyphase table of D^T (host-built): its p phase
+    rows, each shifted by q m, give every row of the oracle's D^T to bf16
+    hi + lo precision; padding is zero; the trailing floats are d_k / sqrt(B)
+    (1 without the rotation)."""
+    rng = np.random.default_rng(block + 7 * had)
+    signs = np.where(rng.random(block) < 0.5, -1, 1).astype(np.int8)
+    d = sdq.LayerDesc(16, block, block, osr, 2, had)
+    t, p, q = sdq.sdq_build_poly_table(d, signs)
+    assert Fraction(p, q) == Fraction(osr)
+    st = 2 * block + 8
+    assert t.size == 2 * p * st + block
+    ent = t[:2 * p * st].reshape(p, st, 2)
+    assert not ent[:, 2 * block:, :].any()
+    hi, lo = ent[:, :2 * block, 0], ent[:, :2 * block, 1]
+    first = _bf16(hi & 0xFFFF) + _bf16(lo & 0xFFFF)     # tap d mod B
+    second = _bf16(hi >> 16) + _bf16(lo >> 16)          # tap d + 1 mod B
+    Dt = O.resample_matrix(d.n_b, block)                 # D^T, n_b x B
+    tol = 2.0 ** -15 * np.abs(Dt).max()
+    idx = np.arange(2 * block)
+    for r in range(p):
+        assert np.abs(first[r] - Dt[r, idx % block]).max() <= tol
+        assert np.abs(second[r] - Dt[r, (idx + 1) % block]).max() <= tol
+    for j in range(d.n_b):   # every row from its phase: D^T[r + p m][i] = row r at (i - q m) mod B
+        r, m = j % p, j // p
+        start = (-q * m) % block
+        assert np.abs(first[r, start:start + block] - Dt[j, :]).max() <= tol
+    scale = t[2 * p * st:].view(np.float32).astype(np.float64)
+    want = signs / np.sqrt(block) if had else np.ones(block)
+    assert np.abs(scale - want).max() <= 1e-7
+
+
+@pytest.mark.parametrize("block,osr", [(512, Fraction(2)), (128, Fraction(17, 16)), (8, Fraction(2))])
+def test_poly_table_unsupported(sdq, block, osr):
+    """No table where the decode kernel streams G instead: B above 256, 17
+    phases (more than 16 KB of entries), B not a multiple of 16."""
+    d = sdq.LayerDesc(16, block, block, osr, 2, 1)
+    with pytest.raises(sdq.SdqError) as e:
+        sdq.sdq_build_poly_table(d)
+    assert e.value.status == -2   # SDQ_ERR_UNSUPPORTED
