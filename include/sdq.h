@@ -158,6 +158,17 @@ int sdq_build_tables(const sdq_layer_desc* desc, const int8_t* had_signs,
 int sdq_build_poly_table(const sdq_layer_desc* desc, const int8_t* had_signs, uint32_t* table_host,
                          size_t capacity_words, size_t* words_out, int32_t* p_out, int32_t* q_out);
 
+/* Host-only (no GPU needed): the launch shape the decode contraction takes
+ * at batch M (1..64) on a device with `sm_count` SMs, as sdq_plan_create
+ * chooses it.  Writes 13 int64 values to `out_host`: T (e4m3 terms per
+ * activation), NP (MMA N), S (k chunks), P (CTAs per chunk), CB (128-code
+ * blocks per chunk), ring (stages in the shared-memory ring), streamed (1
+ * when each stage carries its B operand rows), dynamic shared memory bytes,
+ * sb (blocks per stage), nbuf (accumulators per pipeline), bytes per ring
+ * slot, bytes of the resident B operand (0 when streamed), and the kernel's
+ * shared-memory limit.  SDQ_ERR_UNSUPPORTED if no shape fits. */
+int sdq_decode_launch_shape(const sdq_layer_desc* desc, int32_t M, int32_t sm_count, int64_t* out_host);
+
 /* Algorithm 1 without compensation, on every row of W (device, fp32,
  * n_out x k_in row-major).  Writes codes in the plain layout
  * (sdq_plain_bytes) and alpha (device, fp32[n_out]).  Bit-exact contract:

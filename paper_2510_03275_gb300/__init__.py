@@ -21,7 +21,7 @@ __all__ = [
     "SDQ_OK", "SDQ_BINARY", "SDQ_TERNARY", "SDQ_ALPHA_MAXABS", "SDQ_ALPHA_MEANABS",
     "SdqError", "LayerDesc", "lib", "library_path",
     "sdq_plan_create", "sdq_plan_destroy", "sdq_k_eff", "sdq_plain_bytes", "sdq_tiled_bytes",
-    "sdq_workspace_bytes", "sdq_build_tables", "sdq_build_poly_table", "sdq_encode_rows", "sdq_pack", "sdq_unpack",
+    "sdq_workspace_bytes", "sdq_build_tables", "sdq_build_poly_table", "sdq_decode_launch_shape", "sdq_encode_rows", "sdq_pack", "sdq_unpack",
     "sdq_prep_activations", "sdq_contract", "sdq_linear_forward", "sdq_read_prep",
     "sdq_workspace_status", "sdq_linear_forward_noalloc", "sdq_noalloc_scratch_bytes",
     "sdq_forward_kernels", "sdq_status_string", "Plan",
@@ -83,6 +83,7 @@ _SIGS = {
     "sdq_build_tables": (ctypes.c_int, [ctypes.POINTER(_Desc), _vp, _vp, _vp]),
     "sdq_build_poly_table": (ctypes.c_int, [ctypes.POINTER(_Desc), _vp, _vp, _sz, ctypes.POINTER(_sz),
                                             ctypes.POINTER(_i32), ctypes.POINTER(_i32)]),
+    "sdq_decode_launch_shape": (ctypes.c_int, [ctypes.POINTER(_Desc), _i32, _i32, _vp]),
     "sdq_encode_rows": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp]),
     "sdq_pack": (ctypes.c_int, [_vp, _vp, _vp, _vp]),
     "sdq_unpack": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp]),
@@ -192,6 +193,19 @@ def sdq_build_poly_table(desc: LayerDesc, had_signs=None):
                                       ctypes.byref(words), ctypes.byref(pp), ctypes.byref(qq)),
            "sdq_build_poly_table")
     return table, pp.value, qq.value
+
+
+_SHAPE_KEYS = ("T", "NP", "S", "P", "CB", "ring", "streamed", "smem", "sb", "nbuf", "slot_bytes",
+               "b_bytes", "smem_limit")
+
+
+def sdq_decode_launch_shape(desc: LayerDesc, M: int, sm_count: int) -> dict:
+    """Host-only: the decode launch shape at batch M (include/sdq.h)."""
+    import numpy as np
+    out = np.zeros(len(_SHAPE_KEYS), np.int64)
+    _check(lib().sdq_decode_launch_shape(ctypes.byref(desc.c()), M, sm_count, out.ctypes.data_as(_vp)),
+           "sdq_decode_launch_shape")
+    return dict(zip(_SHAPE_KEYS, (int(v) for v in out)))
 
 
 def sdq_encode_rows(plan, W, codes_plain, alpha, stream=None):

@@ -1145,6 +1145,31 @@ int fused_build(const sdq_plan_s* pl, int M) {
   return scratch <= room ? 1 : 0;
 }
 
+}  // namespace sdq
+
+// Host-only launch-shape query (sizing and tests; see include/sdq.h).
+extern "C" int sdq_decode_launch_shape(const sdq_layer_desc* desc, int32_t M, int32_t sm_count, int64_t* out) {
+  using namespace sdq;
+  if (!desc || !out || M < 1 || M > kMaxDecodeM || sm_count < 1) return SDQ_ERR_INVALID_ARG;
+  sdq_plan_s pl{};
+  const int st = validate(desc, &pl.geo);
+  if (st != SDQ_OK) return st;
+  pl.desc = *desc;
+  pl.sm_count = sm_count;
+  const DecodeConfig dc = decode_config_search(&pl, M);
+  if (dc.S < 1) return SDQ_ERR_UNSUPPORTED;
+  int sb = 0, nbuf = 0, dbase = 0;
+  tmem_split(dc.NP, &sb, &nbuf, &dbase);
+  const int64_t blk = (int64_t)kTileRows * kBlk * pl.geo.bits / 8;
+  const int64_t v[13] = {dc.T, dc.NP, dc.S, dc.P, dc.CB, dc.ring, dc.stream, (int64_t)dc.smem, sb, nbuf,
+                         sb * (blk + (dc.stream ? (int64_t)dc.NP * 128 : 0)),
+                         dc.stream ? 0 : (int64_t)dc.CB * dc.NP * 128, kSmemMax + 1024};
+  for (int i = 0; i < 13; ++i) out[i] = v[i];
+  return SDQ_OK;
+}
+
+namespace sdq {
+
 bool decode_fusable(const sdq_plan_s* pl, int M, const uint16_t* x) {
   return (reinterpret_cast<uintptr_t>(x) & 15u) == 0 && fused_build(pl, M) != 0;
 }

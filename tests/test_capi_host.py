@@ -150,3 +150,42 @@ def test_poly_table_unsupported(sdq, block, osr):
     with pytest.raises(sdq.SdqError) as e:
         sdq.sdq_build_poly_table(d)
     assert e.value.status == -2   # SDQ_ERR_UNSUPPORTED
+
+
+def _launch_shapes():
+    seen = {}
+    for ci in range(5):
+        cfg = W.config(ci)
+        for lin in cfg.linears:
+            seen[(lin.n_out, lin.k_in, cfg.block, Fraction(lin.osr), cfg.quantizer)] = None
+    seen[(77, 640, 64, Fraction(9, 4), 2)] = None
+    seen[(129, 272, 16, Fraction(5, 2), 1)] = None
+    seen[(5, 4096, 1024, Fraction(4), 2)] = None
+    return list(seen)
+
+
+@pytest.mark.parametrize("sms", [152, 148, 132, 20])
+def test_decode_launch_shapes_fit(sdq, sms):
+    """Every decode launch shape the plan would choose keeps the kernel's
+    invariants: at most one CTA per SM, k chunks covering K with none empty,
+    a ring of 4..24 stages in multiples of 4, TMEM columns within 512, the
+    B operand and ring within the shared-memory limit, stage copies within
+    the mbarrier transaction count, and a streamed B operand only past the
+    one-kernel route (M > 4)."""
+    for n, k, b, osr, qz in _launch_shapes():
+        d = sdq.LayerDesc(n, k, b, osr, qz, 1, 0)
+        kb = -(-sdq.sdq_k_eff(d) // 128)
+        blk = 128 * 128 * qz // 8
+        for m in range(1, 65):
+            s = sdq.sdq_decode_launch_shape(d, m, sms)
+            assert s["T"] == (4 if m <= 8 else 2) and s["NP"] == -(-(m * s["T"]) // 16) * 16
+            assert 1 <= s["S"] and 1 <= s["P"] and s["S"] * s["P"] <= sms
+            assert (s["S"] - 1) * s["CB"] < kb <= s["S"] * s["CB"]
+            assert 4 <= s["ring"] <= 24 and s["ring"] % 4 == 0
+            assert 2 * 2 * 32 * s["sb"] + 2 * s["nbuf"] * s["NP"] <= 512
+            assert s["streamed"] in (0, 1) and (m > 4 or not s["streamed"])
+            assert s["slot_bytes"] == s["sb"] * (blk + (s["NP"] * 128 if s["streamed"] else 0))
+            assert s["b_bytes"] == (0 if s["streamed"] else s["CB"] * s["NP"] * 128)
+            assert 1024 + s["b_bytes"] + s["ring"] * s["slot_bytes"] <= s["smem"] <= s["smem_limit"]
+            assert s["slot_bytes"] < (1 << 20)
+            assert max(-(-s["CB"] // s["sb"]), min(2, s["CB"])) <= 128   # stages per row tile
