@@ -22,7 +22,7 @@ What it computes (SDQ-LLM, arXiv 2510.03275):
 * Storage accounting, eq. (14).
 * The packed code layouts (plain and tiled) of the C-ABI header.
 
-Readings of points the paper leaves open (every one is listed in the design doc):
+Readings of points the paper leaves open:
 
 * Integrator: eq. (8) ``i_n = i_{n-1} + x_n - y_{n-1}`` (accumulating form);
   Algorithm 1's SDQuant body writes the integrator without the accumulation,
