@@ -2,9 +2,9 @@
 
 Codes, alpha and packed layouts must be bit-exact.  Layer outputs must be
 within max |y - y_ref| / max |y_ref| <= 1e-2 of the oracle's fp64 forward on
-the same codes (the bar of the task); the fp8 activation expansion is
-expected to do far better (about 2^-12 with three terms, 2^-8 with two),
-which is also asserted.
+the same codes (the accuracy bar for layer outputs); the fp8 activation
+expansion is expected to do far better (about 2^-16 per element with four
+terms, M <= 8, and 2^-8 with two), which is also asserted.
 """
 from fractions import Fraction
 
