@@ -205,8 +205,11 @@ int sdq_prep_activations(sdq_plan plan, const uint16_t* x, int32_t M,
  * = alpha_r * sum_j c[r,j] x_tilde[m,j], reading the x_tilde that
  * sdq_prep_activations left in `ws` for the same M.  M <= 64: decode kernel
  * (tcgen05 fp8 MMAs with the codes expanded into tensor memory as the A
- * operand, split-K over thread blocks with a deterministic last-block
- * reduction).  M > 64: tcgen05 bf16 prefill kernel. */
+ * operand and the prepared fp8 terms as the B operand, copied once per k
+ * chunk or, for larger batches, streamed with each stage of codes;
+ * split-K over thread blocks with a deterministic last-block reduction; the
+ * launch shape is chosen per batch size at plan creation and can be queried
+ * with sdq_decode_launch_shape).  M > 64: tcgen05 bf16 prefill kernel. */
 int sdq_contract(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha, int32_t M,
                  float* y, void* ws, size_t ws_bytes, void* stream);
 
