@@ -392,6 +392,10 @@ def run_sdq(args, rank, world, dist):
         out["decode_sweep"] = decode_sweep(P, W, torch, layers, stream, hbm, tf_burst, peak_src)
         out["prefill"] = prefill_leg(P, W, torch, layers, stream, tf_burst, tf_sus, peak_src)
         out["cpu_baseline"] = cpu_baseline_leg()
+        try:
+            out["encode"]["cpu"] = encode_cpu_leg()
+        except Exception as e:   # a reported comparison only: never fail the run on it
+            out["encode"]["cpu"] = {"unavailable": f"{type(e).__name__}: {e}"[:200]}
     return out
 
 
@@ -538,6 +542,28 @@ def cpu_baseline_leg(sample_rows=256, min_secs=10.0):
             "sample": f"oracle forward_code_domain (fp64 numpy), decode M=1, {sample_rows} rows of "
                       f"each of the 7 llama-70b-layer linears ({smp.nbytes} code bytes) x {passes} passes = "
                       f"{secs:.1f} s; numpy default threads on {cores} host cores"}
+
+
+def encode_cpu_leg(rows=64):
+    """The oracle's canonical fp32 encoder (the bit-exact contract of
+    sdq_encode_rows) timed on the host on the first `rows` rows of every
+    llama-70b-layer linear, extrapolated linearly to the full layer and
+    labelled as such."""
+    import numpy as np
+    import oracle as O
+    from paper_2510_03275_gb300 import workloads as W
+    cfg = W.config(4)
+    secs = 0.0
+    for lin in cfg.linears:
+        w = W.weights(lin, rows=np.arange(rows))
+        signs = W.hadamard_signs(lin, cfg.block)
+        nb = int(cfg.block * lin.osr)
+        t0 = time.perf_counter()
+        O.encode(w, cfg.block, nb, cfg.quantizer, O.ALPHA_MAXABS, signs)
+        secs += (time.perf_counter() - t0) * lin.n_out / rows
+    return {"oracle_ms_per_layer_extrapolated": round(secs * 1e3, 1), "cores": _cores(),
+            "sample": f"oracle encode (canonical fp32, numpy) on {rows} rows of each of the 7 "
+                      "linears, scaled by rows to the full layer"}
 
 
 def run_reference(args, rank, world):

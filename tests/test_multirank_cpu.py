@@ -81,6 +81,15 @@ def test_profile_hash_ignores_comments_only():
     assert "//x" in bench.code_text('const char* s = "//x";\n')
 
 
+def test_encode_cpu_leg_extrapolates():
+    """The host-side encode timing of the bench: a positive per-layer figure
+    from a row sample (CPU only)."""
+    sys.path.insert(0, ROOT)
+    import bench
+    r = bench.encode_cpu_leg(rows=2)
+    assert r["oracle_ms_per_layer_extrapolated"] > 0 and r["cores"] >= 1 and "2 rows" in r["sample"]
+
+
 def test_reference_arm_under_torchrun_world2():
     env = dict(os.environ, CUDA_VISIBLE_DEVICES="")
     cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node=2",
