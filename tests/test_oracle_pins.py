@@ -294,16 +294,20 @@ def test_error_decreases_with_osr(qz):
     assert errs[-1] < 0.45
 
 
-def test_forward_code_domain_identity():
-    """alpha C G x == x W_hat^T (closed-form adjoint identity, fp64)."""
-    rng = np.random.default_rng(13)
-    B, nb = 128, 320
+@pytest.mark.parametrize("qz", [O.TERNARY, O.BINARY])
+@pytest.mark.parametrize("had", [True, False])
+@pytest.mark.parametrize("B,nb", [(128, 320), (16, 24), (64, 64)])
+def test_forward_code_domain_identity(qz, had, B, nb):
+    """alpha C G x == x W_hat^T (closed-form adjoint identity, fp64), for both
+    quantizers, with and without the rotation, at OSR 2.5, 1.5 and 1."""
+    rng = np.random.default_rng(13 + B + nb + qz + int(had))
     d = np.where(rng.random(B) < 0.5, -1, 1)
-    w = (rng.standard_normal((24, 384)) * 0.02).astype(np.float32)
-    codes, alpha = O.encode(w, B, nb, O.TERNARY, O.ALPHA_MAXABS, d)
-    x = rng.standard_normal((3, 384))
-    y1 = O.forward(x, O.reconstruct(codes, alpha, B, nb, d))
-    y2 = O.forward_code_domain(x, codes, alpha, B, nb, d)
+    K = 3 * B
+    w = (rng.standard_normal((24, K)) * 0.02).astype(np.float32)
+    codes, alpha = O.encode(w, B, nb, qz, O.ALPHA_MAXABS, d, had)
+    x = rng.standard_normal((3, K))
+    y1 = O.forward(x, O.reconstruct(codes, alpha, B, nb, d, had))
+    y2 = O.forward_code_domain(x, codes, alpha, B, nb, d, had)
     assert np.abs(y1 - y2).max() < 1e-10 * np.abs(y1).max()
 
 
