@@ -5,6 +5,7 @@ import re
 from fractions import Fraction
 
 import numpy as np
+import scipy.linalg
 import pytest
 
 import oracle as O
@@ -189,3 +190,34 @@ def test_decode_launch_shapes_fit(sdq, sms):
             assert 1024 + s["b_bytes"] + s["ring"] * s["slot_bytes"] <= s["smem"] <= s["smem_limit"]
             assert s["slot_bytes"] < (1 << 20)
             assert max(-(-s["CB"] // s["sb"]), min(2, s["CB"])) <= 128   # stages per row tile
+
+
+@pytest.mark.parametrize("block,osr", [(128, Fraction(2)), (16, Fraction(5, 2)), (64, Fraction(9, 4))])
+@pytest.mark.parametrize("had", [1, 0])
+def test_poly_table_gives_x_tilde(sdq, block, osr, had):
+    """The decode kernel's order of work, in numpy, with the library's own
+    table: scale x by the table's d_k / sqrt(B), a Walsh-Hadamard transform
+    (Sylvester order), then D^T from the phase rows and shifts, equals the
+    oracle's x_tilde = G x_b (to the bf16 hi + lo precision of the table)."""
+    rng = np.random.default_rng(block + had)
+    signs = np.where(rng.random(block) < 0.5, -1, 1).astype(np.int8)
+    d = sdq.LayerDesc(16, 2 * block, block, osr, 2, had)
+    t, p, q = sdq.sdq_build_poly_table(d, signs)
+    st, nb = 2 * block + 8, d.n_b
+    ent = t[:2 * p * st].reshape(p, st, 2)
+    taps = _bf16(ent[:, :block, 0] & 0xFFFF) + _bf16(ent[:, :block, 1] & 0xFFFF)   # D^T[r][0..B)
+    scale = t[2 * p * st:].view(np.float32).astype(np.float64)
+    x = rng.standard_normal((2, 2 * block)).astype(np.float32).astype(np.float64)
+    want = O.prep_activations(x, block, nb, signs, bool(had))
+    H = scipy.linalg.hadamard(block).astype(np.float64)
+    got = np.zeros_like(want)
+    for m in range(2):
+        for b in range(2):
+            u = x[m, b * block:(b + 1) * block] * scale
+            if had:
+                u = H @ u
+            for j in range(nb):
+                r, mm = j % p, j // p
+                row = np.roll(taps[r], q * mm)          # D^T[j][i] = D^T[r][(i - q m) mod B]
+                got[m, b * nb + j] = row @ u
+    assert np.abs(got - want).max() <= 2.0 ** -14 * np.abs(want).max()
