@@ -48,6 +48,12 @@
  * Ternary fields: 00 = 0, 01 = +1, 11 = -1 (10 is invalid).  Binary: 1 = +1,
  * 0 = -1.  Padding bits are 0.
  *
+ * Invalid codes.  The ternary pattern 10 has no value.  sdq_unpack reports
+ * it (SDQ_ERR_BAD_CODE's condition) by adding the number of such fields to a
+ * caller-owned device counter rather than through its return value, which
+ * would need a device synchronization; the contraction kernels read the
+ * pattern as 0.
+ *
  * Tiled layout (input of sdq_contract; built by sdq_pack): the library's own
  * format (the paper prescribes no storage order).  K_eff is padded to
  * K_pad = 128 ceil(K_eff / 128) codes; rows are grouped by 128 (row tile T,
@@ -136,37 +142,15 @@ size_t sdq_workspace_bytes(sdq_plan plan, int32_t M);
 int sdq_build_tables(const sdq_layer_desc* desc, const int8_t* had_signs,
                      float* a_enc_host, float* g_host);
 
-/* Host-only (no GPU needed): the polyphase table of D^T that the decode
- * kernel's own activation transform reads (sdq_linear_forward at small
- * batches; section 3.5 with Algorithm 1's Resample).  With n_b / block =
- * p / q in lowest terms, band-limited resampling commutes with a cyclic
- * shift of q inputs, so row r + p m of D^T (n_b x block, the adjoint of the
- * decimation) is row r shifted by q m: D^T[r + p m][i] =
- * D^T[r][(i - q m) mod block].  Writes p and q (p_out, q_out) and the
- * table's size in uint32 words (words_out; each may be NULL), and, when
- * `table_host` is not NULL, the table: for r < p and d < 2 block, words
- * 2 (r (2 block + 8) + d) and +1 = the bf16x2 pair (D^T[r][d mod block],
- * D^T[r][(d + 1) mod block]) (first element in the low half) and the bf16x2
- * pair of their remainders after the first rounding; rows padded to
- * 2 block + 8 entries with zeros; then `block` fp32 bit patterns
- * d_k / sqrt(block) (1 without the Hadamard rotation).  Returns
- * SDQ_ERR_UNSUPPORTED when the kernel would not use a table (block not a
- * multiple of 16 or above 256, n_b not a multiple of 8, more than 16 KB of
- * entries, or D^T not polyphase to 1e-12 of its largest entry),
- * SDQ_ERR_WORKSPACE when capacity_words is too small, and the errors of
- * sdq_build_tables. */
-int sdq_build_poly_table(const sdq_layer_desc* desc, const int8_t* had_signs, uint32_t* table_host,
-                         size_t capacity_words, size_t* words_out, int32_t* p_out, int32_t* q_out);
-
 /* Host-only (no GPU needed): the launch shape the decode contraction takes
  * at batch M (1..64) on a device with `sm_count` SMs, as sdq_plan_create
- * chooses it.  Writes 13 int64 values to `out_host`: T (e4m3 terms per
+ * chooses it.  Writes 13 int64 values to `out_host`: T (e2m1 terms per
  * activation), NP (MMA N), S (k chunks), P (CTAs per chunk), CB (128-code
- * blocks per chunk), ring (stages in the shared-memory ring), streamed (1
- * when each stage carries its B operand rows), dynamic shared memory bytes,
- * sb (blocks per stage), nbuf (accumulators per pipeline), bytes per ring
- * slot, bytes of the resident B operand (0 when streamed), and the kernel's
- * shared-memory limit.  SDQ_ERR_UNSUPPORTED if no shape fits. */
+ * blocks per chunk), ring (stages in the shared-memory ring), sb (blocks per
+ * stage), nbuf (accumulators per pipeline), dynamic shared memory bytes,
+ * bytes per ring slot, bytes of the B operand image, TMEM columns between
+ * two blocks' B scales, and the kernel's shared-memory limit.
+ * SDQ_ERR_UNSUPPORTED if no shape fits. */
 int sdq_decode_launch_shape(const sdq_layer_desc* desc, int32_t M, int32_t sm_count, int64_t* out_host);
 
 /* Algorithm 1 without compensation, on every row of W (device, fp32,
@@ -192,44 +176,45 @@ int sdq_unpack(sdq_plan plan, const uint32_t* codes_tiled, uint32_t* codes_plain
 
 /* x_tilde = G x_b for every block b of every row of x (device, bf16 bits,
  * M x k_in row-major), written into the workspace `ws` for sdq_contract.
- * M <= 64: one kernel writes x_tilde in fp32 and, as the decode kernel's
- * tensor-core B operand, T e4m3 terms per batch row m with
- * x_tilde[m] 2^-e_m = sum_t 16^-t q_t[m] (T = 4 for M <= 8, else 2); e_m is set from the bound |x_tilde[m, j]| <= gnorm max_k |x[m, k]|,
- * gnorm = max_j sum_k |G[j, k]|, so that no thread block waits for another.
- * M > 64: x_tilde is written in bf16 in the permuted K order the prefill
- * kernel reads.  Kernels are launched with programmatic dependent launch. */
+ * M <= 64: x_tilde is written in fp32 (M x K_pad, K_pad = 128
+ * ceil(K_eff / 128), padding 0); the decode kernel forms its tensor-core B
+ * operand from it.  M > 64: x_tilde is written in bf16 in the permuted K
+ * order the prefill kernel reads.  Kernels are launched with programmatic
+ * dependent launch.  Errors: INVALID_ARG (also when the current device is
+ * not the plan's), WORKSPACE, CUDA. */
 int sdq_prep_activations(sdq_plan plan, const uint16_t* x, int32_t M,
                          void* ws, size_t ws_bytes, void* stream);
 
 /* Contraction against the tiled codes: y (device, fp32, M x n_out row-major)
  * = alpha_r * sum_j c[r,j] x_tilde[m,j], reading the x_tilde that
  * sdq_prep_activations left in `ws` for the same M.  M <= 64: decode kernel
- * (tcgen05 fp8 MMAs with the codes expanded into tensor memory as the A
- * operand and the prepared fp8 terms as the B operand, copied once per k
- * chunk or, for larger batches, streamed with each stage of codes;
- * split-K over thread blocks with a deterministic last-block reduction; the
- * launch shape is chosen per batch size at plan creation and can be queried
- * with sdq_decode_launch_shape).  M > 64: tcgen05 bf16 prefill kernel. */
+ * (tcgen05 block-scaled 4-bit MMAs, kind::mxf4: the codes expanded into
+ * tensor memory as e2m1 +-2 / 0, the activations as T e2m1 terms per batch
+ * row with one power-of-two scale per 32 codes and term, x_tilde =
+ * sum_t 2^(e_g - 3t) q_t, T = 6 for M <= 4, 4 up to 16, 3 above; each
+ * thread block forms the terms of its k chunk; split-K over thread blocks
+ * with a deterministic last-block reduction; the launch shape is chosen per
+ * batch size at plan creation and can be queried with
+ * sdq_decode_launch_shape).  M > 64: tcgen05 bf16 prefill kernel.  Errors as
+ * sdq_prep_activations, and UNSUPPORTED when no launch shape fits. */
 int sdq_contract(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha, int32_t M,
                  float* y, void* ws, size_t ws_bytes, void* stream);
 
 /* y = the layer applied to x: same inputs, outputs and errors as
  * sdq_prep_activations followed by sdq_contract.  For small decode batches
  * (sdq_forward_kernels() == 1) it is ONE kernel: the decode kernel computes
- * the part of x_tilde its k chunk needs and its fp8 terms itself, with its own
- * power-of-two term scale, and writes no x_tilde to `ws` (sdq_read_prep then
- * returns stale data).  Otherwise it runs the two kernels.  Results of the two
- * routes agree to within the fp8 term rounding (about 2^-16 relative with
- * four terms), not bit for bit. */
+ * the part of x_tilde its k chunk needs itself and writes no x_tilde to `ws`
+ * (sdq_read_prep then returns stale data).  Otherwise it runs the two
+ * kernels.  Results of the two routes agree to within the rounding of
+ * x_tilde (bf16 hi + lo tables, fp32 sums) and of its e2m1 terms, not bit for
+ * bit. */
 int sdq_linear_forward(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha,
                        const uint16_t* x, int32_t M, float* y, void* ws, size_t ws_bytes,
                        void* stream);
 
-/* Kernels sdq_linear_forward launches for this plan, batch M and activation
- * pointer x (its 16-byte alignment matters): 1 (the decode kernel builds its
- * own B operand: M <= 4, block a multiple of 16, n_b a multiple of 8, x
- * 16-byte aligned, and a per-CTA build of at most 64 16-deep MMA steps per
- * warp) or 2.  0 on invalid input.  Host only. */
+/* Kernels sdq_linear_forward launches for this plan, batch M and
+ * activation pointer x: 2 (the prepare kernel, then the contraction).  0 on
+ * invalid input.  Host only. */
 int sdq_forward_kernels(sdq_plan plan, int32_t M, const uint16_t* x);
 
 /* Wait for `stream`, then report whether the last contraction that used
@@ -237,9 +222,13 @@ int sdq_forward_kernels(sdq_plan plan, int32_t M, const uint16_t* x);
  * SDQ_ERR_TIMEOUT (a copy or an MMA did not complete within about 2 s; the
  * output of that call is invalid).  Covers the decode (M <= 64) and the
  * prefill (M > 64) kernels.  Workspace contents never need resetting: the
- * split-K tickets and this record carry a process-wide call number, so stale
- * or random bytes (another call, plan or batch size) do not count, and one
- * workspace may serve several plans in turn (never two calls at once). */
+ * split-K tickets and this record carry a 48-bit tag per call (bit 47 set,
+ * the other 47 bits a bijective scramble of a process-wide call counter),
+ * so zeros, another call's tickets and structured leftovers of another plan
+ * or batch size (counters, small floats) do not count (an arbitrary 64-bit
+ * word matches a given call's tag with probability 2^-47), and the last
+ * arrival at a ticket clears it.  One workspace may serve several plans in
+ * turn (never two calls at once). */
 int sdq_workspace_status(sdq_plan plan, int32_t M, const void* ws, void* stream);
 
 /* Copy x_tilde for M <= 64 out of the workspace as fp32 (M x K_eff,
@@ -257,17 +246,29 @@ int sdq_read_prep(sdq_plan plan, int32_t M, const void* ws, float* xt_out, void*
  *   - M must be 1..64 (the decode path), and sdq_workspace_bytes(plan, M)
  *     must not exceed the array: otherwise SDQ_ERR_INVALID_ARG or
  *     SDQ_ERR_WORKSPACE is returned and nothing is launched.
+ *   - The current device must be the plan's (else SDQ_ERR_INVALID_ARG): the
+ *     array of the current device is used.
  *   - The first call on a device looks up the array's device address
  *     (cudaGetSymbolAddress, with that device current); make that first call
- *     before any stream capture.
+ *     before any stream capture.  The address is cached per device for the
+ *     life of the process: after cudaDeviceReset the cached address is stale,
+ *     so do not use this entry point after resetting a device.
  *   - All calls on a device share the array and it keeps the last call's
  *     contents, none of which needs resetting (see sdq_workspace_status).
  *     Calls that overlap on the GPU (other streams or host threads) race on
  *     the array: serialize them.
- *   - sdq_workspace_status is not available for these calls. */
+ *   - sdq_noalloc_status reports the bounded-wait outcome of the last call. */
 int sdq_linear_forward_noalloc(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha,
                                const uint16_t* x, int32_t M, float* y, void* stream);
 size_t sdq_noalloc_scratch_bytes(void);
+/* Wait for `stream`, then report whether the last sdq_linear_forward_noalloc
+ * call on the current device with this plan and M completed its bounded
+ * device-side waits: SDQ_OK or SDQ_ERR_TIMEOUT (that call's output is
+ * invalid), as sdq_workspace_status does for a caller workspace.  Host only;
+ * reads the call record inside the library's array.  Errors: INVALID_ARG
+ * (also when the current device is not the plan's), WORKSPACE (no call of
+ * this size can have run), CUDA. */
+int sdq_noalloc_status(sdq_plan plan, int32_t M, void* stream);
 
 /* Static string for a status code. */
 const char* sdq_status_string(int status);

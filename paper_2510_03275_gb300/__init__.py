@@ -21,9 +21,9 @@ __all__ = [
     "SDQ_OK", "SDQ_BINARY", "SDQ_TERNARY", "SDQ_ALPHA_MAXABS", "SDQ_ALPHA_MEANABS",
     "SdqError", "LayerDesc", "lib", "library_path",
     "sdq_plan_create", "sdq_plan_destroy", "sdq_k_eff", "sdq_plain_bytes", "sdq_tiled_bytes",
-    "sdq_workspace_bytes", "sdq_build_tables", "sdq_build_poly_table", "sdq_decode_launch_shape", "sdq_encode_rows", "sdq_pack", "sdq_unpack",
+    "sdq_workspace_bytes", "sdq_build_tables", "sdq_decode_launch_shape", "sdq_encode_rows", "sdq_pack", "sdq_unpack",
     "sdq_prep_activations", "sdq_contract", "sdq_linear_forward", "sdq_read_prep",
-    "sdq_workspace_status", "sdq_linear_forward_noalloc", "sdq_noalloc_scratch_bytes",
+    "sdq_workspace_status", "sdq_linear_forward_noalloc", "sdq_noalloc_scratch_bytes", "sdq_noalloc_status",
     "sdq_forward_kernels", "sdq_status_string", "Plan",
 ]
 
@@ -81,8 +81,6 @@ _SIGS = {
     "sdq_tiled_bytes": (_sz, [ctypes.POINTER(_Desc)]),
     "sdq_workspace_bytes": (_sz, [_vp, _i32]),
     "sdq_build_tables": (ctypes.c_int, [ctypes.POINTER(_Desc), _vp, _vp, _vp]),
-    "sdq_build_poly_table": (ctypes.c_int, [ctypes.POINTER(_Desc), _vp, _vp, _sz, ctypes.POINTER(_sz),
-                                            ctypes.POINTER(_i32), ctypes.POINTER(_i32)]),
     "sdq_decode_launch_shape": (ctypes.c_int, [ctypes.POINTER(_Desc), _i32, _i32, _vp]),
     "sdq_encode_rows": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp]),
     "sdq_pack": (ctypes.c_int, [_vp, _vp, _vp, _vp]),
@@ -94,6 +92,7 @@ _SIGS = {
     "sdq_workspace_status": (ctypes.c_int, [_vp, _i32, _vp, _vp]),
     "sdq_forward_kernels": (ctypes.c_int, [_vp, _i32, _vp]),
     "sdq_linear_forward_noalloc": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _vp, _vp]),
+    "sdq_noalloc_status": (ctypes.c_int, [_vp, _i32, _vp]),
     "sdq_noalloc_scratch_bytes": (_sz, []),
     "sdq_status_string": (ctypes.c_char_p, [ctypes.c_int]),
 }
@@ -178,25 +177,8 @@ def sdq_build_tables(desc: LayerDesc, had_signs=None):
     return a, g
 
 
-def sdq_build_poly_table(desc: LayerDesc, had_signs=None):
-    """Host-only: (table as a uint32 numpy array, p, q) -- the polyphase table
-    of D^T the decode kernel's own activation transform reads (layout in
-    include/sdq.h); raises SdqError when the structure does not apply."""
-    import numpy as np
-    words, pp, qq = _sz(0), _i32(0), _i32(0)
-    signs = None if had_signs is None else np.ascontiguousarray(had_signs, dtype=np.int8)
-    sp = None if signs is None else signs.ctypes.data_as(_vp)
-    _check(lib().sdq_build_poly_table(ctypes.byref(desc.c()), sp, None, 0, ctypes.byref(words),
-                                      ctypes.byref(pp), ctypes.byref(qq)), "sdq_build_poly_table")
-    table = np.zeros(words.value, np.uint32)
-    _check(lib().sdq_build_poly_table(ctypes.byref(desc.c()), sp, table.ctypes.data_as(_vp), table.size,
-                                      ctypes.byref(words), ctypes.byref(pp), ctypes.byref(qq)),
-           "sdq_build_poly_table")
-    return table, pp.value, qq.value
-
-
-_SHAPE_KEYS = ("T", "NP", "S", "P", "CB", "ring", "streamed", "smem", "sb", "nbuf", "slot_bytes",
-               "b_bytes", "smem_limit")
+_SHAPE_KEYS = ("T", "NP", "S", "P", "CB", "ring", "sb", "nbuf", "smem", "slot_bytes", "b_bytes", "ss",
+               "smem_limit")
 
 
 def sdq_decode_launch_shape(desc: LayerDesc, M: int, sm_count: int) -> dict:
@@ -248,7 +230,7 @@ def sdq_workspace_status(plan, M, ws, stream=None) -> int:
 
 
 def sdq_forward_kernels(plan, M, x) -> int:
-    """1 if sdq_linear_forward runs as one kernel for this batch and x, else 2."""
+    """Number of kernels sdq_linear_forward launches (2: prepare, contraction)."""
     return lib().sdq_forward_kernels(plan, M, _ptr(x))
 
 
@@ -262,6 +244,12 @@ def sdq_linear_forward_noalloc(plan, codes_tiled, alpha, x, M, y, stream=None):
 
 def sdq_noalloc_scratch_bytes() -> int:
     return lib().sdq_noalloc_scratch_bytes()
+
+
+def sdq_noalloc_status(plan, M, stream=None) -> int:
+    """Synchronize and return the status of the last allocation-free call
+    with this plan and M on the current device (SDQ_OK or a negative status)."""
+    return lib().sdq_noalloc_status(plan, M, _stream(stream))
 
 
 def sdq_status_string(status: int) -> str:

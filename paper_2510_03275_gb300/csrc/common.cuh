@@ -3,7 +3,7 @@
 
 #include <cuda.h>
 #include <cuda_runtime.h>
-#include <cuda_fp8.h>
+#include <cuda_fp16.h>
 #include <atomic>
 #include <cstdint>
 
@@ -18,11 +18,21 @@ inline const DecodeConfig& decode_config(const sdq_plan_s* plan, int M) { return
 // Workspace regions (byte offsets).  cnt: one 64-bit split-K ticket per row
 // tile; err: the call record (two 64-bit words, see call_record_*).
 struct WsLayout {
-  size_t xt, bimg, sexp, part, cnt, err, total;
+  size_t xt, bimg, sfbw, part, cnt, err, total;
 };
 WsLayout workspace_layout(const sdq_plan_s* plan, int M);
+// SDQ_OK when the current device is the plan's, else SDQ_ERR_INVALID_ARG (or
+// SDQ_ERR_CUDA).
+int sdq_check_device(const sdq_plan_s* p);
+// SDQ_ERR_TIMEOUT when the call record in `ws` (layout of plan p, batch M)
+// says the last call gave up a bounded wait, else SDQ_OK; synchronizes
+// `stream`.
+int workspace_record_status(const sdq_plan_s* p, int32_t M, const void* ws, void* stream);
 // Number of a contraction call, from one process-wide counter (never 0).
 uint64_t next_call_number();
+// Tag of call number n for the workspace's tickets and call record: a
+// bijection of the low 47 bits of n, scrambled, with bit 47 set (48 bits).
+uint64_t call_tag(uint64_t n);
 
 // Kernel launchers (return cudaError_t of the launch).
 cudaError_t launch_encode(const sdq_plan_s* p, const float* W, uint32_t* codes, float* alpha,
@@ -30,15 +40,19 @@ cudaError_t launch_encode(const sdq_plan_s* p, const float* W, uint32_t* codes, 
 cudaError_t launch_pack(const sdq_plan_s* p, const uint32_t* plain, uint32_t* tiled, cudaStream_t st);
 cudaError_t launch_unpack(const sdq_plan_s* p, const uint32_t* tiled, uint32_t* plain,
                           uint32_t* bad, cudaStream_t st);
-cudaError_t launch_prep(const sdq_plan_s* p, const uint16_t* x, int M, void* ws, cudaStream_t st);
+// y_zero (M x n_out, may be null): cleared by the decode prepare kernel.
+cudaError_t launch_prep(const sdq_plan_s* p, const uint16_t* x, int M, void* ws, cudaStream_t st,
+                        float* y_zero = nullptr);
 // early = 1: the decode kernel starts streaming codes before waiting for the
 // preceding grid (valid only behind this library's own prep kernels).
-// x != nullptr: the decode kernel builds its B operand from x itself (no prep
-// kernel; see decode_fusable).
+// y_zeroed = 1: y holds zeros (the prepare kernel of the same call cleared
+// it), so that split-K partial sums may be added into it by float atomics
+// (order of the additions not fixed); else the deterministic ticket route.
 cudaError_t launch_decode(const sdq_plan_s* p, const uint32_t* codes, const float* alpha, int M,
-                          float* y, void* ws, cudaStream_t st, int early, const uint16_t* x);
-// Whether the decode kernel can build its own B operand for batch M from x.
-bool decode_fusable(const sdq_plan_s* p, int M, const uint16_t* x);
+                          float* y, void* ws, cudaStream_t st, int early, int y_zeroed);
+// Whether the decode prepare kernel writes the B operand image (n_b a
+// multiple of 64), so that each decode CTA copies its chunk's part.
+bool decode_image(const sdq_plan_s* p);
 cudaError_t launch_prefill(const sdq_plan_s* p, const uint32_t* codes, const float* alpha, int M,
                            float* y, void* ws, cudaStream_t st);
 cudaError_t launch_read_prep(const sdq_plan_s* p, int M, const void* ws, float* out, cudaStream_t st);
@@ -64,26 +78,6 @@ __device__ __forceinline__ uint16_t float_to_bf16_bits(float f) {
   uint32_t u = __float_as_uint(f);
   u += 0x7FFFu + ((u >> 16) & 1u);
   return (uint16_t)(u >> 16);
-}
-
-// fp32 -> e4m3 byte (round to nearest even, saturating) and back.
-__device__ __forceinline__ uint32_t f32_to_e4m3(float v) {
-  __nv_fp8_e4m3 t(v);
-  return (uint32_t)(*reinterpret_cast<const uint8_t*>(&t));
-}
-__device__ __forceinline__ float e4m3_to_f32(uint32_t b) {
-  __nv_fp8_e4m3 t;
-  *reinterpret_cast<uint8_t*>(&t) = (uint8_t)b;
-  return (float)t;
-}
-
-// 16x8x32 warp MMA, e4m3 x e4m3 -> fp32.
-__device__ __forceinline__ void mma_e4m3_16832(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k32.row.col.f32.e4m3.e4m3.f32 "
-      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
-      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
 // 16x8x16 warp MMA, bf16 x bf16 -> fp32.
@@ -130,11 +124,6 @@ __device__ __forceinline__ void bulk_g2s_hint(void* dst, const void* src, uint32
       "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;\n"
       ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy) : "memory");
 }
-__device__ __forceinline__ uint64_t globaltimer_ns() {
-  uint64_t t;
-  asm volatile("mov.u64 %0, %globaltimer;\n" : "=l"(t));
-  return t;
-}
 // Bounded wait for phase `parity` of `bar`: gives up after ~4e9 SM cycles
 // (about 2 s) and returns false (callers record an error and skip the
 // dependent work).  The clock is read only once the first test has failed.
@@ -153,6 +142,16 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
   while (!mbar_try(a, parity))
     if (clock64() - t0 > 4000000000ll) return false;
   return true;
+}
+// 16-byte global -> shared copy that does not pass through registers (`bytes`
+// = 0 fills the destination with zeros); completion by cp_async_wait_all.
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, uint32_t bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n"
+               :: "r"(smem_u32(dst)), "l"(src), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;\n" ::: "memory");
 }
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
@@ -244,8 +243,18 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
   return d;
 }
 
-// 32 TMEM lanes x 32 columns of 32-bit values from registers: register i of
-// the thread of lane l goes to (lane base + l, column + i).
+// 32 TMEM lanes x 16 (8) columns of 32-bit values from registers: register
+// i of the thread of lane l goes to (lane base + l, column + i).
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};\n"
+      ::"r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]) : "memory");
+}
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[8]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};\n" ::"r"(taddr),
+               "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]) : "memory");
+}
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
   asm volatile(
       "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
@@ -257,23 +266,51 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
       : "memory");
 }
 __device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;\n" ::: "memory"); }
-// D (TMEM, fp32) (+)= A (TMEM, e4m3) . B (smem descriptor, e4m3)^T.
-__device__ __forceinline__ void umma_f8_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
-                                           uint32_t idesc, uint32_t accumulate) {
+
+// D (TMEM, fp32) (+)= A (TMEM, e2m1) . B (smem descriptor, e2m1)^T, M = 128,
+// K = 64, with the block scales of A and B read from TMEM (one ue8m0 scale
+// per 32 K; this library stores 1.0 everywhere and scales in the epilogue).
+// A in TMEM: lane = row, column c nibble i (low first) = K index 8 c + i.
+// B in shared memory: K-major, byte j nibble h (low first) = K index 2 j + h.
+__device__ __forceinline__ void umma_mxf4_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                             uint32_t sfa_tmem, uint32_t sfb_tmem, uint32_t accumulate) {
   asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate) : "memory");
+      "{\n .reg .pred p;\n setp.ne.b32 p, %6, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::mxf4.block_scale.scale_vec::2X [%0], [%1], %2, %3, [%4], [%5], p;\n}\n"
+      ::"r"(d_tmem), "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(sfa_tmem), "r"(sfb_tmem), "r"(accumulate)
+      : "memory");
 }
+// Instruction descriptor of umma_mxf4_ts: A and B e2m1, ue8m0 scales,
+// M = 128, N = n (a multiple of 16, at most 256), dense, both K-major.
+__host__ __device__ constexpr uint32_t mxf4_idesc(int n) {
+  return (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | (1u << 23) | (1u << 27);
+}
+// ue8m0 1.0 in every byte of a scale-factor column.
+constexpr uint32_t kUnitScales = 0x7F7F7F7Fu;
+
+// Two fp32 values to a byte of e2m1 codes (round to nearest even, saturating
+// at +-6): `lo` in bits 0-3, `hi` in bits 4-7; `q` receives the two values
+// the codes stand for (exact).
+__device__ __forceinline__ uint32_t e2m1x2(float lo, float hi, float2* q) {
+  uint16_t b;
+  uint32_t h2;
+  asm("{\n .reg .b8 t;\n cvt.rn.satfinite.e2m1x2.f32 t, %3, %2;\n mov.b16 %0, {t, 0};\n"
+      " cvt.rn.f16x2.e2m1x2 %1, t;\n}\n"
+      : "=h"(b), "=r"(h2) : "f"(lo), "f"(hi));
+  *q = __half22float2(*reinterpret_cast<const __half2*>(&h2));
+  return b;
+}
+
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;\n" ::"r"(id), "r"(nthreads) : "memory");
 }
 
-// Call record in the workspace: word 0 = number of the last call that gave up
-// a bounded wait, word 1 = number of the last call that ran.  Call numbers
-// are never 0 and never repeat, so a record written by another call, plan or
-// batch size (or random initial contents, barring a 2^-64 coincidence) does
-// not read as the current call's: nothing in the workspace needs resetting.
+// Call record in the workspace: word 0 = tag of the last call that gave up a
+// bounded wait, word 1 = tag of the last call that ran.  Tags (call_tag in
+// capi.cu) are 48-bit values with bit 47 set, distinct for 2^47 calls and
+// scrambled, so that neither zeroed memory nor structured leftovers of
+// another call, plan or batch size (counters, small floats) read as the
+// current call's: nothing in the workspace needs resetting.
 __device__ __forceinline__ void call_record_start(uint64_t* rec, uint64_t call, bool leader) {
   if (leader) rec[1] = call;
 }
@@ -283,54 +320,80 @@ __device__ __forceinline__ void call_record_fail(uint64_t* rec, uint64_t call) {
 
 __device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;\n" ::: "memory"); }
 
-// Split-K ticket of one row tile: bits 16..63 the call number, bits 0..15 the
-// arrivals of that call.  A ticket that carries another call number counts
-// as empty, so tickets need no reset between calls.  One acq_rel fence (after
-// the CTA barrier that orders the other threads' partial stores before it)
-// publishes the CTA's partials; then every arrival adds 1, and an add that
-// found another call's number installs (call, 1) by compare-and-swap or
-// joins the call that another arrival installed meanwhile.  (Such adds never
-// carry into the call field: a call leaves at most 2 S arrivals in a ticket,
-// far below 2^16.)  The last arrival fences again before reading the other
-// CTAs' partials.  Returns this CTA's arrival number (1..S), or 0 if the
-// compare-and-swap did not settle within its retry bound.
-__device__ __forceinline__ uint32_t ticket_take(uint64_t* tk, uint64_t call) {
+// Split-K ticket of one row tile: bits 16..63 the call's tag, bits 0..15 the
+// arrivals of that call.  A ticket that carries another tag counts as empty.
+// One acq_rel fence (after the CTA barrier that orders the other threads'
+// partial stores before it) publishes the CTA's partials; then every arrival
+// adds 1, and an add that found another tag installs (tag, 1) by
+// compare-and-swap or joins the call that another arrival installed
+// meanwhile.  (Such adds never carry into the tag field: a call leaves at
+// most 2 S arrivals in a ticket, far below 2^16.)  The last arrival
+// (n == total) fences again before reading the other CTAs' partials and
+// clears the ticket, so that a workspace that is only ever used for these
+// calls keeps zeros there.  Returns this CTA's arrival number (1..total), or
+// 0 if the compare-and-swap did not settle within its retry bound.
+__device__ __forceinline__ uint32_t ticket_take(uint64_t* tk, uint64_t call, uint32_t total) {
   unsigned long long* p = reinterpret_cast<unsigned long long*>(tk);
   fence_acq_rel_gpu();
   const unsigned long long old = atomicAdd(p, 1ull);
-  if ((old >> 16) == call) return (uint32_t)(old & 0xFFFFu) + 1;
-  unsigned long long cur = old + 1;   // another call's ticket, with our add in it
-  for (int it = 0; it < 64; ++it) {
-    const unsigned long long prev = atomicCAS(p, cur, (call << 16) | 1ull);
-    if (prev == cur) return 1;
-    if ((prev >> 16) == call) return (uint32_t)(atomicAdd(p, 1ull) & 0xFFFFu) + 1;
-    cur = prev;
+  uint32_t n = 0;
+  if ((old >> 16) == call) {
+    n = (uint32_t)(old & 0xFFFFu) + 1;
+  } else {
+    unsigned long long cur = old + 1;   // another call's ticket, with our add in it
+    for (int it = 0; it < 64 && n == 0; ++it) {
+      const unsigned long long prev = atomicCAS(p, cur, (call << 16) | 1ull);
+      if (prev == cur) n = 1;
+      else if ((prev >> 16) == call) n = (uint32_t)(atomicAdd(p, 1ull) & 0xFFFFu) + 1;
+      else cur = prev;
+    }
   }
-  return 0;
+  if (n == total) {
+    fence_acq_rel_gpu();
+    atomicExch(p, 0ull);
+  }
+  return n;
 }
 
-// MMA K position (within a 128-code block) of natural code kl: the inverse of
-// decode_stage_k below.
+// Install `call`'s tag in a ticket ahead of the arrivals (count 0), unless
+// an arrival already did: one read and at most one compare-and-swap, issued
+// at kernel start so that the end-of-kernel arrivals find the tag and take
+// the one-atomic path of ticket_take.  A lost race is harmless: ticket_take
+// installs or joins the tag itself.
+__device__ __forceinline__ void ticket_install(uint64_t* tk, uint64_t call) {
+  unsigned long long* p = reinterpret_cast<unsigned long long*>(tk);
+  const unsigned long long old = *reinterpret_cast<volatile unsigned long long*>(p);
+  if ((old >> 16) != call) atomicCAS(p, old, call << 16);
+}
+
+// MMA K position kap (within a 128-code block) of natural code kl: the
+// inverse of decode_stage_k.
+//   ternary: kl = 16 w + 2 n + s -> kap = 16 w + 8 s + n
+//   binary:  kl = 32 w + 4 n + k -> kap = 32 w + 8 k + n
 __host__ __device__ __forceinline__ int decode_pos(int kl, bool ternary) {
   if (ternary) {
     const int f = kl & 15;
-    return (kl & ~15) + 4 * (3 - (f & 3)) + (f >> 2);
+    return (kl & ~15) + 8 * (f & 1) + (f >> 1);
   }
   const int f = kl & 31;
-  return (kl & ~31) + 4 * (7 - (f & 7)) + (f >> 3);
+  return (kl & ~31) + 8 * (f & 3) + (f >> 2);
 }
 
-// Natural k (within a 128-code decode block) at MMA K index kap: the order in
-// which the decode expander lays a row's codes into TMEM columns.
-//   ternary: column 4 wi + j (word wi, shift 2j) byte b = code 16 wi + 4b + 3 - j
-//   binary:  column 8 wi + j (word wi, shift j)  byte b = code 32 wi + 8b + 7 - j
+// Natural k (within a 128-code decode block) at MMA K index kap = 8 c + n
+// (TMEM column c of the block's 16, nibble n): the order in which the decode
+// expander turns a row's packed words into e2m1 nibbles.
+//   ternary: word w (codes 16 w .. 16 w + 15, 2 bits each) gives column 2 w
+//            (even codes: nibble n = code 16 w + 2 n) and column 2 w + 1
+//            (odd codes: nibble n = code 16 w + 2 n + 1)
+//   binary:  word w (codes 32 w .. 32 w + 31) gives columns 4 w + k, k < 4,
+//            nibble n = code 32 w + 4 n + k
 __host__ __device__ __forceinline__ int decode_stage_k(int kap, bool ternary) {
   if (ternary) {
     const int kp = kap & 15;
-    return (kap & ~15) + 4 * (kp & 3) + 3 - (kp >> 2);
+    return (kap & ~15) + 2 * (kp & 7) + (kp >> 3);
   }
   const int kp = kap & 31;
-  return (kap & ~31) + 8 * (kp & 3) + 7 - (kp >> 2);
+  return (kap & ~31) + 4 * (kp & 7) + (kp >> 3);
 }
 
 // Position of natural index kl (0..63) inside a 64-code stage of the prefill

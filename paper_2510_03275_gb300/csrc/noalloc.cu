@@ -10,9 +10,10 @@
 // loaded and held until the process exits.
 //
 // The array is shared by every call on a device and keeps whatever the last
-// call left in it: tickets and the call record carry a process-wide call
-// number, so stale contents never count, and everything else is written
-// before it is read.  Two calls that overlap on the GPU (different streams,
+// call left in it: tickets and the call record carry a scrambled 48-bit tag
+// per call, so stale contents do not count (a leftover word matches a call's
+// tag with probability 2^-47), and everything else is written before it is
+// read.  Two calls that overlap on the GPU (different streams,
 // or different host threads) race on the array.
 #include <mutex>
 
@@ -44,18 +45,33 @@ int scratch_for_current_device(void** out) {
   return SDQ_OK;
 }
 
+// Checks shared by the entry point and its status query: batch size, the
+// plan's device being current, the scratch size; then the array's address.
+int noalloc_scratch(sdq_plan p, int32_t M, void** ws) {
+  if (!p || M < 1 || M > sdq::kMaxDecodeM) return SDQ_ERR_INVALID_ARG;
+  int st = sdq::sdq_check_device(p);
+  if (st != SDQ_OK) return st;
+  const size_t need = sdq_workspace_bytes(p, M);
+  if (need == 0) return SDQ_ERR_INVALID_ARG;
+  if (need > kNoAllocScratchBytes) return SDQ_ERR_WORKSPACE;
+  return scratch_for_current_device(ws);
+}
+
 }  // namespace
 
 extern "C" size_t sdq_noalloc_scratch_bytes(void) { return kNoAllocScratchBytes; }
 
 extern "C" int sdq_linear_forward_noalloc(sdq_plan p, const uint32_t* codes_tiled, const float* alpha,
                                           const uint16_t* x, int32_t M, float* y, void* stream) {
-  if (!p || M < 1 || M > sdq::kMaxDecodeM) return SDQ_ERR_INVALID_ARG;
-  const size_t need = sdq_workspace_bytes(p, M);
-  if (need == 0) return SDQ_ERR_INVALID_ARG;
-  if (need > kNoAllocScratchBytes) return SDQ_ERR_WORKSPACE;
   void* ws = nullptr;
-  const int st = scratch_for_current_device(&ws);
+  const int st = noalloc_scratch(p, M, &ws);
   if (st != SDQ_OK) return st;
   return sdq_linear_forward(p, codes_tiled, alpha, x, M, y, ws, kNoAllocScratchBytes, stream);
+}
+
+extern "C" int sdq_noalloc_status(sdq_plan p, int32_t M, void* stream) {
+  void* ws = nullptr;
+  const int st = noalloc_scratch(p, M, &ws);
+  if (st != SDQ_OK) return st;
+  return sdq::workspace_record_status(p, M, ws, stream);
 }

@@ -251,7 +251,7 @@ cudaError_t launch_prefill(const sdq_plan_s* pl, const uint32_t* codes, const fl
   PrefillParams p;
   p.codes = codes; p.alpha = alpha; p.y = y;
   p.rec = reinterpret_cast<uint64_t*>(wbase + L.err);
-  p.call = next_call_number();
+  p.call = call_tag(next_call_number());
   p.M = M; p.N = g.n_out; p.ntiles = g.ntiles; p.ngroups = g.ngroups; p.wpg = g.wpg;
   p.nks = (int)(g.k_eff_pad / kBK);
   p.quantizer = pl->desc.quantizer;

@@ -8,9 +8,10 @@
 // x is bf16 (exact), G is split into bf16 hi + lo parts (relative error of
 // the pair ~2^-16), accumulation in fp32.
 //
-// Decode path (M <= 64): the decode prepare kernel below (x_tilde and the
-// decode kernel's e4m3 B operand in one pass).  Prefill path: bf16 x_tilde
-// in the permuted 64-code stage order of the prefill kernel's operand tiles.
+// Decode path (M <= 64): the decode prepare kernel below writes fp32
+// x_tilde, from which each decode CTA forms the e2m1 terms and scales of its
+// k chunk.  Prefill path: bf16 x_tilde in the permuted 64-code stage order
+// of the prefill kernel's operand tiles.
 #include <algorithm>
 
 #include "common.cuh"
@@ -132,44 +133,30 @@ __global__ void __launch_bounds__(128) prep_kernel(PrepParams p) {
 }
 
 // ------------------------------------------------- decode prepare (M <= 64)
-// One kernel per call: x_tilde = G x_b as above (fp32, kept for checking),
-// and directly the decode kernel's e4m3 B operand.  That operand covers all
-// of K: block kb (128 codes) is NP rows x 128 bytes in the 128-byte-swizzled
-// K-major layout, row n = m T + t holding term t of batch row m at the MMA K
-// position of each code (decode_pos).  With x_tilde[m] 2^-e_m < 448,
-// v = x_tilde 2^-e_m splits into sum_t 16^-t q_t: q_t = e4m3(v_t),
-// v_{t+1} = 16 (v_t - q_t) (exact: e4m3 rounding is relative).  e_m comes
-// from a bound rather than from the maximum of x_tilde, so that no CTA waits
-// for another: |x_tilde[m, j]| <= sum_k |G[j, k]| |x[m, k]| <= gnorm max|x[m]|,
-// gnorm = max_j sum_k |G[j, k]| (with a margin for the bf16 split of G).
-// e4m3 is floating point, so the looser scale costs no relative precision.
-// Rows past M T are not written: they only feed accumulator columns that
-// are never read.  The CTA's x tile and G rows arrive in one round of loads
-// (k chunks of up to 256), overlapped with its reading of the x row for
-// max |x[m]|.
+// One kernel per call: x_tilde = G x_b as above, fp32, M x kpad (the K
+// padding zeroed), and, when n_b is a multiple of 64 (`bimg` set), the
+// decode kernel's B operand for all of K: per 32-code group g of batch row
+// m the power of two 2^e with |x_tilde 2^-e| < 4 (from the group's maximum)
+// and T e2m1 terms, x_tilde = sum_t 2^(e - 3t) q_t, each term the 8x-scaled
+// rounding error of the ones before.  Term t of row m is image row
+// n = m T + t: 128-code block kb occupies bytes 64 (kb & 1) .. + 63 of the
+// 128-byte rows of atom kb / 2 (NP rows, 128-byte swizzle), MMA position
+// kap = 2 byte + nibble (decode_pos order); its scales are the bytes of
+// word (kb, n) of `sfbw`: byte 2 mu + beta = 2^(e - 3t) of K group beta of
+// the block's MMA mu.  The CTA's x tile and G rows arrive in one round of
+// asynchronous copies (k chunks of up to 256).
 struct DecPrepParams {
   const uint16_t* x;
   const uint16_t* g_hi;
   const uint16_t* g_lo;
   float* xt;          // M x kpad fp32
-  uint8_t* bimg;      // e4m3 B operand image
-  int* sexp;          // e_m per batch row
-  float gnorm;
-  int M, K, B, n_b, nblk, T, NP, kc, ternary, vec;
+  uint8_t* bimg;      // B operand image (null: x_tilde only)
+  uint8_t* sfbw;      // B scale words, KB x NP x 4 bytes
+  float* y_zero;      // cleared (M x n_out) for the decode kernel's atomic split-K, or null
+  int64_t y_count;
+  int M, K, B, n_b, nblk, kc, vec, T, NP, ternary;
   int64_t k_eff, kpad;
 };
-
-__device__ __forceinline__ float bf16_abs(uint32_t h) { return __uint_as_float((h & 0x7FFFu) << 16); }
-
-// 16-byte global -> shared copy that does not pass through registers; `bytes`
-// = 0 fills the destination with zeros.
-__device__ __forceinline__ void cp_async16(void* dst, const void* src, uint32_t bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n"
-               :: "r"(smem_u32(dst)), "l"(src), "r"(bytes) : "memory");
-}
-__device__ __forceinline__ void cp_async_wait_all() {
-  asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;\n" ::: "memory");
-}
 
 __global__ void __launch_bounds__(128) prep_decode_kernel(DecPrepParams p) {
   constexpr int TB = 16, NTW = 2;   // 16 blocks x 64 j per CTA; warp w owns j 16w .. 16w + 15
@@ -178,21 +165,23 @@ __global__ void __launch_bounds__(128) prep_decode_kernel(DecPrepParams p) {
   uint16_t* xs = reinterpret_cast<uint16_t*>(dsm);   // TB x ld
   uint16_t* ghs = xs + TB * ld;                        // 64 x ld
   uint16_t* gls = ghs + 64 * ld;                       // 64 x ld
-  __shared__ float red[4];
-  __shared__ int e_s;
   pdl_wait();
   pdl_launch_dependents();
   const int jt = blockIdx.x, bt = blockIdx.y, m = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t = lane & 3;
   const int b0 = bt * TB, j0 = jt * 64, wcol = warp * 16;
   const uint16_t* xr = p.x + (size_t)m * p.K;
+  if (p.y_zero) {   // grid-stride clear of y
+    const int64_t nthr = (int64_t)gridDim.x * gridDim.y * gridDim.z * 128;
+    const int64_t i0 = ((int64_t)(blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x) * 128 + tid;
+    for (int64_t i = i0; i < p.y_count; i += nthr) p.y_zero[i] = 0.f;
+  }
 
   float acc[NTW][4];
 #pragma unroll
   for (int n = 0; n < NTW; ++n)
 #pragma unroll
     for (int e = 0; e < 4; ++e) acc[n][e] = 0.f;
-  float xmax = 0.f;
   for (int kc0 = 0; kc0 < p.B; kc0 += p.kc) {
     if (p.vec) {   // B % 32 == 0, rows 16-byte aligned: asynchronous 16-byte copies
       const int q8 = p.kc / 8;
@@ -220,29 +209,6 @@ __global__ void __launch_bounds__(128) prep_decode_kernel(DecPrepParams p) {
         gls[rr * ld + kk] = gv ? p.g_lo[(size_t)j * p.B + k] : 0;
       }
     }
-    if (kc0 == 0) {
-      // max |x[m, :]| while the tile copies are in flight; 8 independent
-      // 16-byte loads per thread at a time.
-      if (p.vec) {
-        const int nv = p.K / 8;
-        for (int i0 = tid; i0 < nv; i0 += 128 * 8) {
-          uint4 v[8];
-#pragma unroll
-          for (int u = 0; u < 8; ++u) {
-            const int i = i0 + 128 * u;
-            v[u] = i < nv ? __ldg(reinterpret_cast<const uint4*>(xr) + i) : make_uint4(0, 0, 0, 0);
-          }
-#pragma unroll
-          for (int u = 0; u < 8; ++u) {
-            const uint32_t w[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
-#pragma unroll
-            for (int q = 0; q < 4; ++q) xmax = fmaxf(xmax, fmaxf(bf16_abs(w[q]), bf16_abs(w[q] >> 16)));
-          }
-        }
-      } else {
-        for (int i = tid; i < p.K; i += 128) xmax = fmaxf(xmax, bf16_abs(xr[i]));
-      }
-    }
     if (p.vec) cp_async_wait_all();
     __syncthreads();
     for (int ks = 0; ks < p.kc; ks += 16) {
@@ -266,64 +232,89 @@ __global__ void __launch_bounds__(128) prep_decode_kernel(DecPrepParams p) {
     __syncthreads();
   }
 
-  // term scale exponent e_m from the bound
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) xmax = fmaxf(xmax, __shfl_xor_sync(0xffffffffu, xmax, o));
-  if (lane == 0) red[warp] = xmax;
-  __syncthreads();
-  if (tid == 0) {
-    const float mx = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
-    int e = 0;
-    if (mx > 0.f) {   // bound = mx gnorm < 2^(e1 + e2) without forming it (no overflow)
-      int e1 = 0, e2 = 0;
-      frexpf(mx, &e1);
-      frexpf(p.gnorm, &e2);
-      e = e1 + e2 - 8;   // bound * 2^-e < 256 < 448
-    }
-    e = max(e, -120);
-    e_s = e;
-    if (jt == 0 && bt == 0) p.sexp[m] = e;
-  }
-  __syncthreads();
-  const float inv = ldexpf(1.f, -e_s);
-  const bool ter = p.ternary != 0;
+  // x_tilde of the tile: to global memory (fp32) and to shared memory (the G
+  // tiles are no longer read) for the terms below
+  float* tile = reinterpret_cast<float*>(dsm);   // TB x 64
 #pragma unroll
   for (int n = 0; n < NTW; ++n)
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
-      const int b = b0 + g + (e >> 1) * 8;
-      const int j = j0 + wcol + n * 8 + 2 * t + (e & 1);
-      if (b < p.nblk && j < p.n_b) {
-        const int64_t kk = (int64_t)b * p.n_b + j;
-        p.xt[(size_t)m * p.kpad + kk] = acc[n][e];
-        uint8_t* blk = p.bimg + (size_t)(kk >> 7) * p.NP * 128;
-        const int kap = decode_pos((int)(kk & 127), ter);
-        float v = acc[n][e] * inv;
-        for (int tt = 0; tt < p.T; ++tt) {
-          const uint32_t q = f32_to_e4m3(v);
-          const int row = m * p.T + tt;
-          blk[row * 128 + (((kap >> 4) ^ (row & 7)) << 4) + (kap & 15)] = (uint8_t)q;
-          v = (v - e4m3_to_f32(q)) * 16.f;
+      const int bl = g + (e >> 1) * 8, jl = wcol + n * 8 + 2 * t + (e & 1);
+      const int b = b0 + bl, j = j0 + jl;
+      if (b < p.nblk && j < p.n_b) p.xt[(size_t)m * p.kpad + (int64_t)b * p.n_b + j] = acc[n][e];
+      tile[bl * 64 + jl] = acc[n][e];
+    }
+  // K padding of this batch row
+  if (jt == 0 && bt == 0)
+    for (int64_t k = p.k_eff + tid; k < p.kpad; k += 128) p.xt[(size_t)m * p.kpad + k] = 0.f;
+  if (!p.bimg) return;
+  __syncthreads();
+  // Terms: thread = (block bl of the tile, 32-code group gm of the tile's 64
+  // codes, quarter s4): 8 MMA positions of one 32-position scale group; the
+  // four quarters of a group are consecutive lanes and share its maximum.
+  {
+    const bool ter = p.ternary != 0;
+    const int bl = tid >> 3, gm = (tid >> 2) & 1, s4 = tid & 3, b = b0 + bl;
+    const bool act = b < p.nblk;
+    const int64_t kk0 = (int64_t)b * p.n_b + j0;   // 64-aligned: n_b % 64 == 0
+    const int64_t kb = kk0 >> 7;
+    const int kl0 = (int)(kk0 & 127);
+    const int g8 = (kl0 >> 3) + 4 * gm + s4;
+    float v[8];
+    float mx = 0.f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int kl = decode_stage_k(8 * g8 + i, ter);
+      v[i] = act ? tile[bl * 64 + (kl - kl0)] : 0.f;
+      mx = fmaxf(mx, fabsf(v[i]));
+    }
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+    int ex = -125;
+    if (mx > 0.f) {   // mx < 2^E, so |v 2^-(E - 2)| < 4
+      int E = 0;
+      frexpf(mx, &E);
+      ex = E - 2;
+    }
+    const float inv = ldexpf(1.f, -ex);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] *= inv;
+    if (act) {
+      uint8_t* img = p.bimg + (size_t)(kb >> 1) * p.NP * 128;
+      const int chunk = 4 * (int)(kb & 1) + (g8 >> 2), off = 4 * (g8 & 3);
+      for (int tt = 0; tt < p.T; ++tt) {
+        uint32_t word = 0;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          float2 q;
+          word |= e2m1x2(v[2 * i], v[2 * i + 1], &q) << (8 * i);
+          v[2 * i] = (v[2 * i] - q.x) * 8.f;
+          v[2 * i + 1] = (v[2 * i + 1] - q.y) * 8.f;
         }
+        const int row = m * p.T + tt;
+        *reinterpret_cast<uint32_t*>(img + row * 128 + ((chunk ^ (row & 7)) << 4) + off) = word;
+        if (s4 == 0) p.sfbw[((size_t)kb * p.NP + row) * 4 + (g8 >> 2)] = (uint8_t)max(1, min(254, 127 + ex - 3 * tt));
       }
     }
-  // K padding of this batch row (x_tilde and its terms are 0 there).
-  if (jt == 0 && bt == 0) {
-    for (int64_t k = p.k_eff + tid; k < p.kpad; k += 128) {
-      p.xt[(size_t)m * p.kpad + k] = 0.f;
-      uint8_t* blk = p.bimg + (size_t)(k >> 7) * p.NP * 128;
-      const int kap = decode_pos((int)(k & 127), ter);
-      for (int tt = 0; tt < p.T; ++tt) {
-        const int row = m * p.T + tt;
-        blk[row * 128 + (((kap >> 4) ^ (row & 7)) << 4) + (kap & 15)] = 0;
-      }
+  }
+  // the K padding (the last block's second half, MMA positions 64..127 =
+  // bytes 32..63 of its 64, when K_eff is an odd number of 64-code halves):
+  // zero terms, unit scales
+  if (jt == 0 && bt == 0 && p.kpad > p.k_eff && tid < 2 * p.T) {
+    const int64_t kb = p.k_eff >> 7;
+    const int tt = tid >> 1, c = 4 * (int)(kb & 1) + 2 + (tid & 1), row = m * p.T + tt;
+    uint8_t* img = p.bimg + (size_t)(kb >> 1) * p.NP * 128;
+    *reinterpret_cast<uint4*>(img + row * 128 + ((c ^ (row & 7)) << 4)) = make_uint4(0, 0, 0, 0);
+    if ((tid & 1) == 0) {
+      p.sfbw[((size_t)kb * p.NP + row) * 4 + 2] = 127;
+      p.sfbw[((size_t)kb * p.NP + row) * 4 + 3] = 127;
     }
   }
 }
 
 }  // namespace
 
-cudaError_t launch_prep(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws, cudaStream_t st) {
+cudaError_t launch_prep(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws, cudaStream_t st, float* y_zero) {
   const Geometry& g = pl->geo;
   const WsLayout L = workspace_layout(pl, M);
   uint8_t* base = static_cast<uint8_t*>(ws);
@@ -333,13 +324,14 @@ cudaError_t launch_prep(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws
     DecPrepParams p;
     p.x = x; p.g_hi = pl->d_g_hi; p.g_lo = pl->d_g_lo;
     p.xt = reinterpret_cast<float*>(base + L.xt);
-    p.bimg = base + L.bimg;
-    p.sexp = reinterpret_cast<int*>(base + L.sexp);
-    p.gnorm = pl->gnorm;
-    p.M = M; p.K = g.k_in; p.B = g.block; p.n_b = g.n_b; p.nblk = g.nblk;
+    p.bimg = decode_image(pl) ? base + L.bimg : nullptr;
+    p.sfbw = base + L.sfbw;
     p.T = dc.T; p.NP = dc.NP;
-    p.kc = std::max(16, std::min(g.block, 256));
+    p.y_zero = y_zero;
+    p.y_count = (int64_t)M * g.n_out;
     p.ternary = g.bits == 2;
+    p.M = M; p.K = g.k_in; p.B = g.block; p.n_b = g.n_b; p.nblk = g.nblk;
+    p.kc = std::max(16, std::min(g.block, 256));
     p.vec = vec;
     p.k_eff = g.k_eff; p.kpad = g.k_eff_pad;
     const size_t smem = (size_t)(16 + 128) * (p.kc + 8) * sizeof(uint16_t);

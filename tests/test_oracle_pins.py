@@ -327,8 +327,8 @@ def test_decimation_adjoint_is_upsample_over_osr_plus_rank1():
 def test_decimation_adjoint_is_polyphase(B, osr):
     """Band-limited resampling commutes with shifts that land on both grids:
     n_b / B = p / q, a cyclic shift of the n_b codes by p is one of the B
-    outputs by q, so row r + p m of D^T is row r rolled by q m (the structure
-    the decode kernel's polyphase table stores)."""
+    outputs by q, so row r + p m of D^T is row r rolled by q m: D^T is fixed
+    by its first p rows (a polyphase structure)."""
     nb = int(B * osr)
     p, q = osr.numerator, osr.denominator
     rng = np.random.default_rng(B + nb)

@@ -2,15 +2,18 @@
 
 Codes, alpha and packed layouts must be bit-exact.  Layer outputs must be
 within max |y - y_ref| / max |y_ref| <= 1e-2 of the oracle's fp64 forward on
-the same codes (the accuracy bar for layer outputs); the fp8 activation
-expansion is expected to do far better (about 2^-16 per element with four
-terms, M <= 8, and 2^-8 with two), which is also asserted.
+the same codes (the accuracy bar for layer outputs), and every element
+within the bound of the path's own arithmetic (tests/errbound.py: T e2m1
+terms per 32-code group on the decode path, one bf16 rounding of x_tilde on
+the prefill path, fp32 accumulation on both); the element-wise error
+max |d| / max(|y_ref|, 1e-3 max |y_ref|) is reported beside it.
 """
 from fractions import Fraction
 
 import numpy as np
 import pytest
 
+import errbound as EB
 import oracle as O
 from paper_2510_03275_gb300 import workloads as W
 
@@ -229,30 +232,41 @@ def test_prep_matches_oracle(sdq, torch_cuda):
         assert err < 2e-5, err
 
 
+def _terms(sdq, d, m):
+    import torch
+    if m > 64:
+        return None   # the prefill path: x_tilde in bf16
+    return sdq.sdq_decode_launch_shape(d, m, torch.cuda.get_device_properties(0).multi_processor_count)["T"]
+
+
 def _check_forward(plan, d, signs, codes, alpha, tiled, sdq, torch, m, seed, rows=None):
-    """codes: all rows, or (with ``rows``) just the sampled rows."""
+    """codes: all rows, or (with ``rows``) just the sampled rows.  Asserts
+    every element within its bound; returns max |d| / max |y_ref|."""
     bits, x = _x(torch, m, d.k_in, seed)
     ws = plan.alloc_workspace(m)
     y = plan.forward(tiled, torch.from_numpy(alpha).cuda(), x, ws=ws)
     assert sdq.sdq_workspace_status(plan.handle, m, ws) == 0
     a = alpha if rows is None else alpha[rows]
-    yr = O.forward_code_domain(W.bf16_to_float(bits), codes, a, d.block, d.n_b, signs)
+    xf = W.bf16_to_float(bits)
+    yr = O.forward_code_domain(xf, codes, a, d.block, d.n_b, signs)
     yg = y.cpu().numpy()
     if rows is not None:
         yg = yg[:, rows]
+    EB.check(yg, yr, EB.forward_bound(xf, codes, a, d.block, d.n_b, signs, T=_terms(sdq, d, m)),
+             f"M={m} n={d.n_out} k={d.k_in} B={d.block} OSR={d.osr}")
     return np.abs(yg - yr).max() / np.abs(yr).max()
 
 
 @pytest.mark.parametrize("q", [O.TERNARY, O.BINARY])
 @pytest.mark.parametrize("m", [1, 2, 3, 4, 5, 8, 16, 17, 33, 64])
 @pytest.mark.parametrize("shape", [(33, 384, 128, Fraction(5, 2)), (256, 512, 512, 2),
-                                   (100, 1024, 128, Fraction(3, 2)), (17, 20, 4, Fraction(5, 2))])
+                                   (100, 1024, 128, Fraction(3, 2)), (17, 20, 4, Fraction(5, 2)),
+                                   (150, 640, 128, 3), (260, 1536, 128, 3)])
 def test_forward_decode_small(sdq, torch_cuda, q, m, shape):
     n, k, b, osr = shape
     lay = _setup_layer(sdq, torch_cuda, n, k, b, osr, q, seed=n + k + m)
     err = _check_forward(*lay, sdq, torch_cuda, m, seed=m)
-    bound = 1e-3 if m <= 8 else 8e-3   # four e4m3 terms up to M = 8, two above
-    assert err <= min(TOL, bound), err
+    assert err <= TOL, err
 
 
 def test_forward_encoded_single_and_opt125m(sdq, torch_cuda):
@@ -288,7 +302,89 @@ def test_forward_full_size_sampled(sdq, torch_cuda, ci, name, m):
     lay = _setup_layer(sdq, torch, lin.n_out, lin.k_in, cfg.block, lin.osr, cfg.quantizer,
                        seed=lin.seed, rows=rows)
     err = _check_forward(*lay, sdq, torch, m, seed=m + 11, rows=rows)
-    assert err <= min(TOL, 1e-3 if m <= 8 else 8e-3), err
+    assert err <= TOL, err
+
+
+@pytest.mark.parametrize("name", ["q", "k", "v", "o", "fc1", "fc2"])
+@pytest.mark.parametrize("m", [1, 16])
+def test_forward_opt125m_all_linears(sdq, torch_cuda, name, m):
+    """OPT-125M's six linears (binary codes, OSR 2.5) at M = 1 and 16, every
+    output row checked."""
+    cfg = W.config(1)
+    lin = [l for l in cfg.linears if l.name == name][0]
+    lay = _setup_layer(sdq, torch_cuda, lin.n_out, lin.k_in, cfg.block, lin.osr, cfg.quantizer, seed=lin.seed)
+    err = _check_forward(*lay, sdq, torch_cuda, m, seed=m + 3)
+    assert err <= TOL, err
+
+
+@pytest.mark.parametrize("name", ["l2.gate", "l3.down", "l0.q"])
+def test_forward_llama13b_multiosr_decode(sdq, torch_cuda, name):
+    """LLaMA-13B stack under the MultiOSR map, batch-8 decode at full size
+    (l2.gate at OSR 3, l3.down at OSR 1.5); 48 sampled rows."""
+    from paper_2510_03275_gb300.multiosr import allocate
+    torch = torch_cuda
+    cfg = W.config(3, multiosr=allocate)
+    lin = [l for l in cfg.linears if l.name == name][0]
+    if name == "l2.gate":
+        assert lin.osr == 3
+    if name == "l3.down":
+        assert lin.osr == Fraction(3, 2)
+    rows = np.sort(np.random.default_rng(lin.seed + 8).choice(lin.n_out, 48, replace=False))
+    lay = _setup_layer(sdq, torch, lin.n_out, lin.k_in, cfg.block, lin.osr, cfg.quantizer,
+                       seed=lin.seed, rows=rows)
+    err = _check_forward(*lay, sdq, torch, 8, seed=19, rows=rows)
+    assert err <= TOL, err
+
+
+def _device_codes(torch, plan, d, q, seed):
+    """Random valid plain codes for every row of a full-size layer, drawn on
+    the device (torch's seeded generator; ternary fields 00 / 01 / 11 with
+    probabilities 1/2, 1/4, 1/4, padding fields zero)."""
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed)
+    nw = sdq_plain_words(plan, d)
+    w = torch.randint(-2 ** 31, 2 ** 31 - 1, (d.n_out, nw), generator=g, device="cuda", dtype=torch.int64)
+    w = w.to(torch.int32)
+    if q == O.TERNARY:   # field 10 -> 00: clear the high bit where the low bit is 0
+        hi_clear = torch.bitwise_and(torch.bitwise_left_shift(torch.bitwise_not(w), 1), -0x55555556)
+        w = torch.bitwise_and(w, torch.bitwise_not(hi_clear))
+    keff = plan.k_eff
+    per = 32 // q
+    full = keff // per
+    if full < nw:
+        rem = keff - full * per
+        if rem:
+            w[:, full] = torch.bitwise_and(w[:, full], (1 << (q * rem)) - 1)
+            w[:, full + 1:] = 0
+        else:
+            w[:, full:] = 0
+    return w.reshape(-1)
+
+
+def sdq_plain_words(plan, d):
+    return O.plain_words_per_row(plan.k_eff, d.quantizer)
+
+
+@pytest.mark.parametrize("name,m", [("gate", 1), ("down", 16), ("q", 64)])
+def test_forward_full_size_every_row_coded(sdq, torch_cuda, name, m):
+    """LLaMA-70B linears with random codes in every row (drawn on the
+    device); 64 sampled rows read back, unpacked by the oracle and checked."""
+    torch = torch_cuda
+    cfg = W.config(4)
+    lin = [l for l in cfg.linears if l.name == name][0]
+    d = _desc(sdq, lin.n_out, lin.k_in, cfg.block, lin.osr, cfg.quantizer)
+    rng = np.random.default_rng(lin.seed)
+    signs = np.where(rng.random(cfg.block) < 0.5, -1, 1).astype(np.int8)
+    plan = sdq.Plan(d, signs)
+    plain = _device_codes(torch, plan, d, cfg.quantizer, seed=lin.seed)
+    tiled = plan.pack(plain)
+    alpha = (rng.random(lin.n_out) * 0.05 + 0.01).astype(np.float32)
+    rows = np.sort(rng.choice(lin.n_out, 64, replace=False))
+    wpr = sdq_plain_words(plan, d)
+    sub = plain.view(lin.n_out, wpr)[torch.as_tensor(rows, device="cuda")].cpu().numpy().view(np.uint32)
+    codes = O.unpack_plain(sub, cfg.quantizer, plan.k_eff)
+    err = _check_forward(plan, d, signs, codes, alpha, tiled, sdq, torch, m, seed=m + 23, rows=rows)
+    assert err <= TOL, err
 
 
 def test_workspace_too_small_rejected(sdq, torch_cuda):
@@ -306,7 +402,7 @@ def test_workspace_too_small_rejected(sdq, torch_cuda):
 # ---------------------------------------------------------------- prefill
 @pytest.mark.parametrize("q", [O.TERNARY, O.BINARY])
 @pytest.mark.parametrize("m,shape", [(128, (256, 512, 128, 2)), (200, (300, 384, 128, Fraction(5, 2))),
-                                     (65, (17, 20, 4, Fraction(5, 2))), (130, (256, 512, 512, 2)),
+                                     (65, (17, 20, 4, Fraction(5, 2))), (130, (256, 512, 512, 2)), (130, (150, 640, 128, 3)),
                                      (384, (520, 768, 128, Fraction(3, 2)))])
 def test_forward_prefill_small(sdq, torch_cuda, q, m, shape):
     """tcgen05 prefill path (M > 64) against the oracle; x_tilde enters the
@@ -315,7 +411,6 @@ def test_forward_prefill_small(sdq, torch_cuda, q, m, shape):
     lay = _setup_layer(sdq, torch_cuda, n, k, b, osr, q, seed=n + k + m)
     err = _check_forward(*lay, sdq, torch_cuda, m, seed=m)
     assert err <= TOL, err
-    assert err <= 8e-3, err
 
 
 @pytest.mark.parametrize("ci,name,m", [(4, "q", 4096), (4, "gate", 4096), (4, "down", 4096),
@@ -330,4 +425,4 @@ def test_forward_prefill_full_size_sampled(sdq, torch_cuda, ci, name, m):
     lay = _setup_layer(sdq, torch, lin.n_out, lin.k_in, cfg.block, lin.osr, cfg.quantizer,
                        seed=lin.seed, rows=rows)
     err = _check_forward(*lay, sdq, torch, m, seed=m + 5, rows=rows)
-    assert err <= min(TOL, 8e-3), err
+    assert err <= TOL, err
