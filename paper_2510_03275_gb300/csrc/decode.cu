@@ -22,38 +22,50 @@
 //             each CTA copies its k chunk's part; otherwise the CTA forms its
 //             part from the prepared fp32 x_tilde
 //   scales    A: 1.0 everywhere; B: 2^(e - 3t) for term row m T + t and
-//             32-code group g, one set of TMEM columns per 128-code block
+//             32-code group g, one set of TMEM columns per 128-code block of
+//             a stage, written by the expanders beside the stage's codes
 //             (scale id 0 for its first MMA, 2 for its second)
 //   D (TMEM)  fp32, 128 lanes x NP columns
 // so that y[m, r] = alpha_r / 2 * sum_t D[r, m T + t].
 //
-// A stage is up to sb blocks of 128 codes (2 sb MMAs): every mbarrier wait
-// of an MMA-issuing thread costs about as much as several MMAs, so the CTA
-// runs two independent pipelines e = 0, 1 on alternate stages (i = e mod 2),
-// each with its own producer thread, two expander sets, MMA issuer, two
-// TMEM slots and accumulator; the epilogue adds the two accumulators.  Set
-// t of pipeline e owns TMEM slot 2e + t and expands the pipeline's stages
-// j = t (mod 2): every mbarrier has one producer and one consumer that both
-// walk its phases in order.
+// Issuing one of these MMAs occupies the issuing thread for about 130 cycles
+// whatever N is, while MMAs issued from different warps proceed side by
+// side; so the stages (sb <= 4 blocks of 128 codes each, 2 sb MMAs: large
+// stages, since every stage costs each thread it passes through a few
+// hundred cycles of waits and signals) of a row tile
+// are dealt round-robin to `npipe` (1, 2 or 4) MMA pipelines, each with its
+// own issuing warp and accumulator, and the epilogue adds the pipelines'
+// accumulators.  Stage i of the CTA uses
+//   ring slot i mod ring      (codes in shared memory; ring a multiple of 4)
+//   producer i mod 4          (one thread issuing its bulk copies)
+//   expander set i mod 4      (4 warps, one per TMEM lane quadrant)
+//   TMEM A slot i mod ns      (ns = 4 or 8 slots of 16 sb columns: with 4,
+//                             each expander set refills its one slot once
+//                             the MMAs of its previous stage are done, the
+//                             codes already in registers)
+//   pipeline i mod npipe
+// so that every mbarrier has one producer and one consumer that both walk its
+// phases in order.
 //
-// CTA (k chunk s, row set p) of one SM, 24 warps:
-//   warps 0, 1    lane 0 of warp e streams pipeline e's stages (one 128-row
-//                 tile x up to sb * 128 codes = contiguous slabs of the tiled
-//                 layout) into its shared-memory ring slots with bulk
-//                 copies; warp 0 also owns the TMEM allocation
-//   warps 2, 3    lane 0 of warp 2 + e issues pipeline e's MMAs, commits to
-//                 the stage's TMEM slot and, after its last stage of a row
-//                 tile, to its accumulator
-//   warps 4..19   first the B operand and its scales, then the expanders:
-//                 set x = 2e + t (warps 4 + 4x .. 7 + 4x, one per TMEM lane
-//                 quadrant) expands stages i = e + 2t (mod 4) into TMEM slot x
-//   warps 20..23  epilogue: read and add the accumulators, sum the terms,
-//                 scale and store y; with split-K (S > 1) either add into y
-//                 with float atomics (y cleared by the prepare kernel of the
-//                 same call: sdq_linear_forward) or store a partial, and after
-//                 the main loop take the tiles' tickets; the CTA with a tile's
-//                 last ticket sums its S partials in a fixed order
-//                 (deterministic: sdq_contract)
+// CTA (k chunk s, row set p) of one SM, 28 warps:
+//   warps 0..3    lane 0 of warp e issues pipeline e's MMAs (e < npipe),
+//                 commits to the stage's TMEM slot and, after its last stage
+//                 of a row tile, to its accumulator; warp 0 also owns the
+//                 TMEM allocation
+//   warps 4..7    epilogue: read and add the pipelines' accumulators, sum the
+//                 terms, scale and store y; with split-K (S > 1) either add
+//                 into y with float atomics (y cleared by the prepare kernel
+//                 of the same call: sdq_linear_forward) or store a partial,
+//                 and after the main loop take the tiles' tickets; the CTA
+//                 with a tile's last ticket sums its S partials in a fixed
+//                 order (deterministic: sdq_contract)
+//   warps 8..23   first the B operand and its scales, then the expanders:
+//                 set x (warps 8 + 4x .. 11 + 4x) expands stages i = x mod 4
+//   warps 24..27  lane 0 of warp 24 + x streams stages i = x mod 4 (one
+//                 128-row tile x sb * 128 codes = contiguous slabs of the
+//                 tiled layout) into the ring with bulk copies: a thread
+//                 starts a bulk copy only every ~600 cycles, four side by
+//                 side keep an SM's share of HBM busy
 // With `early` set the producers start the code stream before waiting for
 // the preceding grid (codes are never written by the prep kernels).
 // Every mbarrier wait is bounded (about 2 s); a timeout writes the call's
@@ -70,23 +82,26 @@ namespace {
 
 constexpr int kBlk = 128;                        // codes per block (2 MMAs of K = 64)
 constexpr int kAColsPerBlk = kBlk / 8;           // TMEM columns of a block's e2m1 codes
-constexpr int kProducers = 2;                    // warps 0, 1
-constexpr int kIssuerWarp0 = 2;                  // warps 2, 3
-constexpr int kSlots = 2;                        // TMEM A slots (and expander sets) per pipeline
-constexpr int kMaxSb = 4;                        // at most 4 blocks per stage
-constexpr int kExpWarp0 = 4;                     // warps 4..19
-constexpr int kExpSets = 2 * kSlots;
-constexpr int kEpiWarp0 = kExpWarp0 + 4 * kExpSets;   // warps 20..23
-constexpr int kThreads = 32 * (kEpiWarp0 + 4);   // 768
-constexpr int kMaxRing = 24;
+constexpr int kASlots = 8;                       // TMEM A slots at most: stage i -> slot i mod ns (4 or 8)
+constexpr int kExpSets = 4;                      // expander sets: stage i -> set i mod 4
+constexpr int kMaxPipes = 4;                     // MMA pipelines: stage i -> i mod npipe
+constexpr int kMaxSb = 4;                        // blocks per stage (ns slots x 16 sb columns)
+constexpr int kEpiWarp0 = kMaxPipes;             // warps 4..7
+constexpr int kExpWarp0 = kEpiWarp0 + 4;         // warps 8..23
+constexpr int kProducerWarp0 = kExpWarp0 + 4 * kExpSets; // warps 24..27
+constexpr int kThreads = 32 * (kProducerWarp0 + kExpSets); // 896
+constexpr int kMaxRing = 32;
 constexpr int kMaxSpu = 128;                     // stages per row tile (config search bound)
-constexpr int kSmemMax = 224 * 1024;
+constexpr int kSmemMax = 222 * 1024;
 constexpr int kSmemMin = 120 * 1024;             // > half an SM: one CTA per SM
 constexpr int kBuildThreads = 32 * 4 * kExpSets; // the expander warps load the B operand
 constexpr int kRedWords = 64;                    // split-K sums summed CTA-wide: first 2048 tiles
 constexpr int kSfaCols = 4;                      // A scales: column 32 q + lane r holds row r's
-static_assert(kMaxRing <= 32 && 2 * kSlots + 7 <= 16 && kRedWords == 64 && kMaxSpu < 160,
-              "the prologue's per-warp set-up assumes these bounds");
+constexpr int kAlphaAhead = 4;                   // epilogue: alpha loads this many row tiles ahead
+constexpr int kRingBytes = 160 * 1024;           // code bytes in flight per CTA (target)
+static_assert(kMaxRing <= 32 && kASlots == 8 && 2 * kMaxPipes + 1 + kMaxPipes <= 32 && kRedWords == 64 &&
+                  kMaxSpu < 160 && kMaxRing % kExpSets == 0,
+              "the prologue's per-warp set-up and the stage maps assume these bounds");
 
 struct DecodeParams {
   const uint32_t* codes;
@@ -101,7 +116,7 @@ struct DecodeParams {
   uint64_t call;         // call tag
   int bsrc;              // B operand from: 1 prepared x_tilde, 2 prepared image
   int64_t k_eff, kpad;
-  int M, T, NP, S, P, CB, KB, ring, sb, nbuf, dbase, sfa, sfb, ss;
+  int M, T, NP, S, P, CB, KB, ring, sb, nbuf, npipe, ns, ns_log2, dbase, sfa, sfs, ss;
   int n_out, ntiles, ngroups, ternary, early;
   int atomic_y;          // split-K by float atomic adds into y (zeroed by the prepare kernel)
   uint32_t blk_bytes, slot_bytes, b_bytes, sfb_bytes;
@@ -136,7 +151,7 @@ __device__ __forceinline__ int stage_block(int j, int ncb, int spu) { return j *
 // the CTA's image (two 128-code blocks per 128-byte row, 128-byte swizzle);
 // the scale bytes 2^(e - 3t) to `sfbs`, one 32-bit word per (block, term
 // row): byte 2 mu + beta = scale of K group beta of the block's MMA mu.
-__device__ void write_terms(const DecodeParams& p, uint8_t* bop, uint8_t* sfbs, int kb0, int ncb, int et) {
+__device__ __noinline__ void write_terms(const DecodeParams& p, uint8_t* bop, uint8_t* sfbs, int kb0, int ncb, int et) {
   const bool ter = p.ternary != 0;
   const int ntask = p.M * ncb * 16;
   const int64_t lim = min((int64_t)ncb * kBlk, p.k_eff - (int64_t)kb0 * kBlk);   // chunk codes below K_eff
@@ -188,41 +203,33 @@ __device__ void write_terms(const DecodeParams& p, uint8_t* bop, uint8_t* sfbs, 
   }
 }
 
-// The scale factors into TMEM, columns from sfa on: A's (1.0) in the first
-// kSfaCols, then per block bl the set of ss columns of B's: term row n at
-// column n / 32 of the set, lane n mod 32 of every lane quadrant (each
-// quadrant of the MMA reads its own copy).  32 columns per tcgen05.st (the
-// column count is rounded up to 32 in the TMEM plan); the four builder warps
-// of a lane quadrant share the stores.
-__device__ void store_scales(const DecodeParams& p, uint32_t tmem, const uint8_t* sfbs, int ncb, int warp, int lane) {
-  const int q = warp & 3, x = (warp - kExpWarp0) >> 2;
-  const uint32_t lq = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)p.sfa;
-  const int ncs = (p.NP + 31) / 32, MT = p.M * p.T, ncol = kSfaCols + ncb * p.ss;
-  const uint32_t* w = reinterpret_cast<const uint32_t*>(sfbs);
-  for (int c0 = 32 * x; c0 < ncol; c0 += 128) {
-    uint32_t v[32];
+// n 16-byte words global -> shared by the kBuildThreads builder threads,
+// four loads in flight per thread.
+__device__ __forceinline__ void copy_lsu(uint4* dst, const uint4* src, int n, int et) {
+  for (int t0 = et; t0 < n; t0 += 4 * kBuildThreads) {
+    uint4 v[4];
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      const int cc = c0 + i - kSfaCols;
-      uint32_t val = kUnitScales;
-      if (cc >= 0 && cc < ncb * p.ss) {
-        const int bl = cc / p.ss, j = cc - bl * p.ss, n = 32 * j + lane;
-        if (j < ncs && n < MT) val = w[bl * p.NP + n];
-      }
-      v[i] = val;
-    }
-    tmem_st32(lq + (uint32_t)c0, v);
+    for (int k = 0; k < 4; ++k)
+      if (t0 + k * kBuildThreads < n) v[k] = __ldcg(src + t0 + k * kBuildThreads);
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (t0 + k * kBuildThreads < n) dst[t0 + k * kBuildThreads] = v[k];
   }
 }
 
+// kTernary: 2-bit ternary codes, else 1-bit binary (one instantiation each,
+// so that the expander's loop carries only its own code path).
+template <bool kTernary>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t c_full[kMaxRing], c_empty[kMaxRing];
-  __shared__ __align__(8) uint64_t a_full[2 * kSlots], a_empty[2 * kSlots];
-  __shared__ __align__(8) uint64_t acc_full[2][2], acc_empty[2][2], b_full, b_copy, mma_done[2];
+  __shared__ __align__(8) uint64_t a_full[kASlots], a_empty[kASlots];
+  __shared__ __align__(8) uint64_t acc_full[kMaxPipes][2], acc_empty[kMaxPipes][2], b_full;
+  __shared__ __align__(8) uint64_t mma_done[kMaxPipes];
   __shared__ uint32_t tmem_base;
   __shared__ uint32_t red_bits[kRedWords];  // tiles whose split-K sum this CTA owes (all threads sum)
   __shared__ int sblk[kMaxSpu + 1];         // first block of stage j of a tile
+  __shared__ float s_alpha[kAlphaAhead][kTileRows];   // epilogue: alpha of the next row tiles
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int sidx = blockIdx.x % p.S, prow = blockIdx.x / p.S;
@@ -234,6 +241,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   // unit u is tile prow + ((u + rot) mod nunits) P.
   const int rot = (int)(((int64_t)sidx * ((nunits + p.S - 1) / p.S)) % max(nunits, 1));
   const int nstages = nunits * spu;
+  const int np = p.npipe;
   const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
   uint8_t* base = smem_raw + (sbase - smem_u32(smem_raw));
   uint8_t* bop = base;                                          // B image: b_bytes
@@ -241,30 +249,32 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   uint8_t* ring = sfbs + p.sfb_bytes;                           // ring x slot_bytes
 
   // Set-up spread over warps 1.. (warp 0 allocates TMEM meanwhile).
-  if (warp == 1 && lane < p.ring) {
-    mbar_init(&c_full[lane], 1);
-    mbar_init(&c_empty[lane], 4);   // one arrival per expander warp of the slot's set
+  if (warp == 1) {
+    if (lane < p.ring) {
+      mbar_init(&c_full[lane], 1);
+      mbar_init(&c_empty[lane], 4);   // one arrival per expander warp of the slot's set
+    }
   } else if (warp == 2) {
-    if (lane < 2 * kSlots) {
+    if (lane < kASlots) {
       mbar_init(&a_full[lane], 4);
       mbar_init(&a_empty[lane], 1);
-    } else if (lane < 2 * kSlots + 4) {
-      const int e = (lane - 2 * kSlots) >> 1, b = lane & 1;
-      mbar_init(&acc_full[e][b], 1);
-      mbar_init(&acc_empty[e][b], 128);
-    } else if (lane == 2 * kSlots + 4) {
-      mbar_init(&b_full, 1);
-      mbar_init(&b_copy, 1);
-    } else if (lane == 2 * kSlots + 5 || lane == 2 * kSlots + 6) {
-      mbar_init(&mma_done[lane - 2 * kSlots - 5], 1);
     }
-  } else if (warp >= 3 && warp < 3 + (kMaxSpu + 32) / 32) {
-    const int j = tid - 96;
+  } else if (warp == 3) {
+    if (lane < 2 * kMaxPipes) {
+      mbar_init(&acc_full[lane >> 1][lane & 1], 1);
+      mbar_init(&acc_empty[lane >> 1][lane & 1], 128);
+    } else if (lane == 2 * kMaxPipes) {
+      mbar_init(&b_full, 1);
+    } else if (lane < 2 * kMaxPipes + 1 + kMaxPipes) {
+      mbar_init(&mma_done[lane - 2 * kMaxPipes - 1], 1);
+    }
+  } else if (warp >= kExpWarp0 && warp < kExpWarp0 + (kMaxSpu + 32) / 32) {
+    const int j = tid - 32 * kExpWarp0;
     if (j <= spu) sblk[j] = stage_block(j, ncb, spu);
-  } else if (warp >= 8 && warp < 10) {
-    red_bits[tid - 256] = 0u;
+  } else if (warp >= kExpWarp0 + 6 && warp < kExpWarp0 + 8) {
+    red_bits[tid - 32 * (kExpWarp0 + 6)] = 0u;
   }
-  if (warp == 1 || warp == 2) fence_mbar_init();
+  if (warp >= 1 && warp <= 3) fence_mbar_init();
   if (warp == 0) {
     __syncwarp();
     tmem_alloc(&tmem_base, 512);
@@ -274,25 +284,24 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   __syncthreads();
   tc_fence_after();
   pdl_launch_dependents();
-  // (the builders wait inside their build; the producers, with `early`, after
-  // their first stages)
-  const bool builder = warp >= kExpWarp0 && warp < kEpiWarp0;
-  if (!builder && (warp >= kProducers || !p.early)) pdl_wait();
+  // (the builders wait inside their build; the producers, with `early`,
+  // after their stages)
+  const bool builder = warp >= kExpWarp0 && warp < kProducerWarp0;
+  const bool epilogue = warp >= kEpiWarp0 && warp < kExpWarp0;
+  if (!builder && !epilogue && (warp < kProducerWarp0 || !p.early)) pdl_wait();
   const uint32_t tmem = tmem_base;
   bool ok = true;
 
-  if (warp < kProducers) {
+  if (warp >= kProducerWarp0) {
     if (lane == 0) {
-      // Producer of pipeline `warp`: stages i = warp (mod 2), ring slots
-      // i mod ring (ring is even).  Stage (unit u, j) is the slabs
-      // (tile, 2 b) .. (tile, 2 b' - 1) of its blocks [b, b'), adjacent in the
-      // tiled layout.
-      int last_i = -1;
-      int u = 0, j = warp;
+      // Producer x: stages i = x (mod 4), stage i = (unit u, j) being the
+      // slabs (tile, 2 b) .. (tile, 2 b' - 1) of its blocks [b, b'), adjacent
+      // in the tiled layout, into ring slot i mod ring (round r = i / ring).
+      const int x = warp - kProducerWarp0;
+      int last_i = -1, u = 0, j = x, slot = x, r = 0;
       while (j >= spu) { j -= spu; ++u; }
       const uint64_t pol = l2_policy_evict_first();   // codes are read once per call
-      for (int i = warp; i < nstages && ok; i += kProducers) {
-        const int slot = i % p.ring, r = i / p.ring;
+      for (int i = x; i < nstages && ok; i += kExpSets) {
         if (r > 0) ok = mbar_wait(&c_empty[slot], (r - 1) & 1);
         if (!ok) break;
         const int b0 = sblk[j], b1 = sblk[j + 1];
@@ -303,20 +312,21 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         mbar_expect_tx(&c_full[slot], bytes);
         bulk_g2s_hint(ring + (size_t)slot * p.slot_bytes, src, bytes, &c_full[slot], pol);
         last_i = i;
-        j += kProducers;
+        j += kExpSets;
         while (j >= spu) { j -= spu; ++u; }
+        slot += kExpSets;
+        if (slot >= p.ring) { slot -= p.ring; ++r; }
       }
       if (p.early) pdl_wait();
       // Every copy this thread issued has landed before the CTA may exit.
-      for (int i = last_i; i >= 0 && i > last_i - p.ring; i -= kProducers)
+      for (int i = last_i; i >= 0 && i > last_i - p.ring; i -= kExpSets)
         if (!mbar_wait(&c_full[i % p.ring], (i / p.ring) & 1)) ok = false;
     }
-  } else if (warp < kExpWarp0) {
-    if (lane == 0) {
-      // MMA issuer of pipeline e: stages i = e (mod 2), the pipeline's jj-th
-      // stage (jj = i / 2) in TMEM slot 2e + (jj mod 2), into its own
-      // accumulator.
-      const int e = warp - kIssuerWarp0;
+  } else if (warp < kMaxPipes) {
+    if (lane == 0 && warp < np) {
+      // MMA issuer of pipeline e: stages i = e (mod np) in order, stage i's
+      // codes in TMEM slot i mod 8, into the pipeline's accumulator.
+      const int e = warp;
       ok = mbar_wait(&b_full, 0);
       tc_fence_after();
       const uint32_t idesc0 = mxf4_idesc(p.NP), idesc1 = idesc0 | (2u << 4);   // B scale bytes 0-1 / 2-3
@@ -324,13 +334,13 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       // kept incremental (a single thread's scalar latency is on the path).
       const uint64_t bd0 = sw128_desc(sbase);
       const uint64_t astep = (uint64_t)((p.NP * 128) >> 4);   // descriptor units per image row pair
-      const uint32_t sfa = tmem + (uint32_t)p.sfa, sfb0 = tmem + (uint32_t)p.sfb;
+      const uint32_t sfa = tmem + (uint32_t)p.sfa, sfs = tmem + (uint32_t)p.sfs;
+      const uint32_t sslot = (uint32_t)(p.sb * p.ss);   // B scale columns per TMEM slot
       const uint32_t aslot = (uint32_t)(kAColsPerBlk * p.sb);
-      int k = 0, buf = 0, u = 0, j = e;
-      while (j >= spu) { j -= spu; ++u; }
+      int k = 0, buf = 0, u = e / spu, j = e - (e / spu) * spu, last = -1;
       bool first = true;
       uint32_t dt = 0;
-      for (int i = e, jj = 0; i < nstages && ok; i += 2, ++jj) {
+      for (int i = e; i < nstages && ok; i += np) {
         if (first) {
           buf = p.nbuf == 2 ? (k & 1) : 0;
           if (k >= p.nbuf) {
@@ -339,22 +349,23 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
           }
           dt = tmem + (uint32_t)(p.dbase + (e * p.nbuf + buf) * p.NP);
         }
-        const int a = kSlots * e + (jj & 1);
-        ok = mbar_wait(&a_full[a], (jj >> 1) & 1);
+        const int s = i & (p.ns - 1);
+        ok = mbar_wait(&a_full[s], (i >> p.ns_log2) & 1);
         if (!ok) break;
         tc_fence_after();
         const int b0 = sblk[j], nb = sblk[j + 1] - b0;
-        uint32_t at = tmem + (uint32_t)a * aslot;
-        for (int bb = 0; bb < nb; ++bb, at += kAColsPerBlk) {
+        uint32_t at = tmem + (uint32_t)s * aslot;
+        uint32_t sfb = sfs + (uint32_t)s * sslot;
+        for (int bb = 0; bb < nb; ++bb, at += kAColsPerBlk, sfb += (uint32_t)p.ss) {
           const int bl = b0 + bb, kb = kb0 + bl;
           const uint64_t bd = bd0 + (uint64_t)((kb >> 1) - (kb0 >> 1)) * astep + 4u * (uint32_t)(kb & 1);
-          const uint32_t sfb = sfb0 + (uint32_t)(bl * p.ss);
           umma_mxf4_ts(dt, at, bd, idesc0, sfa, sfb, (first && bb == 0) ? 0u : 1u);
           umma_mxf4_ts(dt, at + 8, bd + 2, idesc1, sfa, sfb, 1u);
         }
-        umma_commit(&a_empty[a]);
+        umma_commit(&a_empty[s]);
+        last = i;
         const int u0 = u;
-        j += 2;
+        j += np;
         while (j >= spu) { j -= spu; ++u; }
         first = u != u0;
         if (first) {   // this pipeline's last stage of the tile
@@ -366,53 +377,55 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       if (!mbar_wait(&mma_done[e], 0)) ok = false;
       // ... and the last commit to each of this pipeline's TMEM slots has
       // arrived (those phases have no other waiter).
-      const int njs = (nstages - e + 1) / 2;   // stages of this pipeline
-      for (int jj = max(0, njs - kSlots); jj < njs; ++jj)
-        if (!mbar_wait(&a_empty[kSlots * e + jj % kSlots], (jj / kSlots) & 1)) ok = false;
+      for (int i = last; i >= 0 && i > last - p.ns; i -= np)
+        if (!mbar_wait(&a_empty[i & (p.ns - 1)], (i >> p.ns_log2) & 1)) ok = false;
     }
-  } else if (warp < kEpiWarp0) {
+  } else if (warp >= kExpWarp0) {
     // ------------------------------------------------ builders, then expanders
     const int et = tid - 32 * kExpWarp0;
+    pdl_wait();
     if (p.bsrc == 2) {
-      // the prepared image rows of the chunk's blocks and their scale words
-      pdl_wait();
-      if (et == 0) {
-        const int a0 = kb0 >> 1, a1 = (kb0 + ncb - 1) >> 1;
-        const uint32_t ib = (uint32_t)(a1 - a0 + 1) * p.NP * 128, sb = (uint32_t)ncb * p.NP * 4;
-        mbar_expect_tx(&b_copy, ib + sb);
-        bulk_g2s(bop, p.bimg + (size_t)a0 * p.NP * 128, ib, &b_copy);
-        bulk_g2s(sfbs, p.sfbw + (size_t)kb0 * p.NP * 4, sb, &b_copy);
-      }
-      ok = mbar_wait(&b_copy, 0);
-      if (!ok) mbar_wait(&b_copy, 0);   // a copy still in flight must land before the CTA exits
+      // The prepared image rows of the chunk's blocks and their scale words,
+      // with plain 16-byte loads (L2 hits: the prepare kernel just wrote
+      // them).  A bulk copy here would queue behind the code stream the
+      // producers have started on the same SM, microseconds of HBM traffic.
+      const int a0 = kb0 >> 1, a1 = (kb0 + ncb - 1) >> 1;
+      copy_lsu(reinterpret_cast<uint4*>(bop), reinterpret_cast<const uint4*>(p.bimg + (size_t)a0 * p.NP * 128),
+               (a1 - a0 + 1) * p.NP * 8, et);
+      copy_lsu(reinterpret_cast<uint4*>(sfbs), reinterpret_cast<const uint4*>(p.sfbw + (size_t)kb0 * p.NP * 4),
+               ncb * p.NP / 4, et);
     } else {
-      pdl_wait();
       write_terms(p, bop, sfbs, kb0, ncb, et);
-      fence_proxy_async_smem();   // generic-proxy stores -> the MMAs' async-proxy reads
     }
-    named_bar_sync(3, kBuildThreads);
-    store_scales(p, tmem, sfbs, ncb, warp, lane);
-    tmem_st_wait();
+    fence_proxy_async_smem();   // generic-proxy stores -> the MMAs' async-proxy reads
+    // A's scales, 1.0 for every row and K group: kSfaCols columns from sfa
+    // (the B scales go with each stage, below)
+    if (warp < kExpWarp0 + 4) {
+      const uint32_t one[4] = {kUnitScales, kUnitScales, kUnitScales, kUnitScales};
+      tmem_st4(tmem + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)p.sfa, one);
+      tmem_st_wait();
+    }
     tc_fence_before();
     named_bar_sync(3, kBuildThreads);
-    if (et == 0) mbar_arrive(&b_full);
+    if (et == 0) mbar_arrive(&b_full);   // (every issuer waits on its one phase)
 
-    // Set x = 2e + t expands stages i = e + 2t (mod 4) in order: TMEM slot
-    // x, ring slots i mod ring (ring is a multiple of 4).
+    // Set x expands stages i = x (mod 4) in order: ring slot i mod ring,
+    // TMEM slot i mod ns (its codes, then its B scales).
     const int x = (warp - kExpWarp0) >> 2, q = warp & 3, r = 32 * q + lane;
-    const int ex = x / kSlots, tx = x - ex * kSlots;
+    const int MT = p.M * p.T;
     const uint32_t lane_addr = tmem + ((uint32_t)(32 * q) << 16);
+    const uint32_t aslot = (uint32_t)(kAColsPerBlk * p.sb);
     const uint32_t slab = p.blk_bytes / 2;
-    int u = 0, j = ex + 2 * tx;
+    int u = 0, j = x, slot = x, rnd = 0;
     while (j >= spu) { j -= spu; ++u; }
-    for (int i = ex + 2 * tx; i < nstages && ok; i += 2 * kSlots) {
-      const int slot = i % p.ring, jj = i >> 1, a = x;
-      ok = warp_wait(&c_full[slot], (i / p.ring) & 1);
+    for (int i = x; i < nstages && ok; i += kExpSets) {
+      const int s = i & (p.ns - 1);
+      ok = warp_wait(&c_full[slot], rnd & 1);
       if (!ok) break;
       // Codes into registers first, so that the ring slot goes back to the
       // producer before this set waits for its TMEM slot.
-      const int nb = sblk[j + 1] - sblk[j];
-      j += 2 * kSlots;
+      const int sb0 = sblk[j], nb = sblk[j + 1] - sb0;
+      j += kExpSets;
       while (j >= spu) { j -= spu; ++u; }
       const uint8_t* cs = ring + (size_t)slot * p.slot_bytes;
       uint32_t w[kMaxSb][8];
@@ -420,7 +433,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       for (int bb = 0; bb < kMaxSb; ++bb) {
         if (bb < nb) {
           const uint8_t* cb = cs + bb * p.blk_bytes;
-          if (p.ternary) {
+          if constexpr (kTernary) {
             const uint4 g0 = *reinterpret_cast<const uint4*>(cb + r * 16);
             const uint4 g1 = *reinterpret_cast<const uint4*>(cb + slab + r * 16);
             w[bb][0] = g0.x; w[bb][1] = g0.y; w[bb][2] = g0.z; w[bb][3] = g0.w;
@@ -434,8 +447,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&c_empty[slot]);
-      if (jj >= kSlots) {
-        ok = warp_wait(&a_empty[a], ((jj / kSlots) - 1) & 1);
+      slot += kExpSets;
+      if (slot >= p.ring) { slot -= p.ring; ++rnd; }
+      if (i >= p.ns) {
+        ok = warp_wait(&a_empty[s], ((i >> p.ns_log2) - 1) & 1);
         if (!ok) break;
         tc_fence_after();
       }
@@ -444,7 +459,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         if (bb < nb) {
           // e2m1 nibble [sign, code bit 0, 0, 0]: +-2.0 or 0 (decode_stage_k order)
           uint32_t v[16];
-          if (p.ternary) {
+          if constexpr (kTernary) {
 #pragma unroll
             for (int wi = 0; wi < 8; ++wi) {
               v[2 * wi] = (w[bb][wi] << 2) & 0xCCCCCCCCu;   // even codes
@@ -456,64 +471,105 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
 #pragma unroll
               for (int k = 0; k < 4; ++k) v[4 * wi + k] = ((w[bb][wi] << (3 - k)) & 0x88888888u) | 0x44444444u;
           }
-          tmem_st16(lane_addr + (uint32_t)(a * kAColsPerBlk * p.sb + kAColsPerBlk * bb), v);
+          tmem_st16(lane_addr + (uint32_t)s * aslot + (uint32_t)(kAColsPerBlk * bb), v);
+          // the block's B scales: term row n = 32 c + lane at column c of the
+          // block's set, this warp's lane quadrant (every quadrant a copy)
+          const uint32_t* sw = reinterpret_cast<const uint32_t*>(sfbs) + (size_t)(sb0 + bb) * p.NP;
+          const uint32_t sc = lane_addr + (uint32_t)p.sfs + (uint32_t)(s * p.sb * p.ss + bb * p.ss);
+          for (int c = 0; 32 * c < p.NP; ++c) {
+            const int n = 32 * c + lane;
+            tmem_st1(sc + (uint32_t)c, n < MT ? sw[n] : kUnitScales);
+          }
         }
       }
       tmem_st_wait();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&a_full[a]);
+      if (lane == 0) mbar_arrive(&a_full[s]);
     }
   } else {
     // ------------------------------------------------------------- epilogue
     const int q = warp & 3, r = 32 * q + lane, et = tid - 32 * kEpiWarp0;
     const int NR = p.ntiles * kTileRows;
     const int MT = p.M * p.T;
+    // alpha of this thread's row, fetched kAlphaAhead row tiles ahead into
+    // a shared-memory ring by cp.async (one group per tile): a global load
+    // issued while the code stream runs waits behind it for microseconds,
+    // and a register it targets would stall the first instruction to touch
+    // it.
+    auto alpha_fetch = [&](int u) {
+      if (u < nunits) {
+        const int ut = u + rot < nunits ? u + rot : u + rot - nunits;
+        const int row = (prow + ut * p.P) * kTileRows + r;
+        if (row < p.n_out) cp_async4(&s_alpha[u % kAlphaAhead][et], p.alpha + row);
+      }
+      cp_async_commit();
+    };
+#pragma unroll
+    for (int k = 0; k < kAlphaAhead; ++k) alpha_fetch(k);
+    pdl_wait();   // y and the workspace belong to the preceding grid until then
     call_record_start(p.rec, p.call, blockIdx.x == 0 && et == 0);
     // the k-chunk-0 CTA of each row set puts this call's tag into the row
     // set's tickets while the main loop runs
     if (p.S > 1 && !p.atomic_y && sidx == 0 && et < 32)
       for (int u = et; u < nunits; u += 32) ticket_install(p.cnt + prow + u * p.P, p.call);
-    int kc[2] = {0, 0};
+    int kc[kMaxPipes] = {0, 0, 0, 0};
+    const uint32_t lq = tmem + ((uint32_t)(32 * q) << 16);
     for (int u = 0; u < nunits && ok; ++u) {
-      // issuers with stages in this tile: both, unless the tile is one stage
-      const bool in0 = spu >= 2 || ((u * spu) & 1) == 0;
-      const bool in1 = spu >= 2 || ((u * spu) & 1) == 1;
-      const int bf0 = kc[0] % p.nbuf, bf1 = kc[1] % p.nbuf;
+      // pipelines with stages in this tile: all, unless it has fewer stages
+      uint32_t in = 0;
+      if (spu >= np) {
+        in = (1u << np) - 1u;
+      } else {
+        for (int t = 0; t < spu; ++t) in |= 1u << ((u * spu + t) % np);
+      }
       bool w = true;
-      if (in0) w = mbar_wait(&acc_full[0][bf0], (kc[0] / p.nbuf) & 1);
-      if (in1 && w) w = mbar_wait(&acc_full[1][bf1], (kc[1] / p.nbuf) & 1);
+#pragma unroll
+      for (int e = 0; e < kMaxPipes; ++e)
+        if (((in >> e) & 1u) && w) w = mbar_wait(&acc_full[e][kc[e] % p.nbuf], (kc[e] / p.nbuf) & 1);
       ok = group_and(2, 128, w);
       if (!ok) break;
       tc_fence_after();
       const int ut = u + rot < nunits ? u + rot : u + rot - nunits;   // unit of this tile
       const int row = (prow + ut * p.P) * kTileRows + r;
       const bool live = row < p.n_out;
-      const float sa = live ? 0.5f * __ldg(p.alpha + row) : 0.f;
-      const uint32_t lq = tmem + ((uint32_t)(32 * q) << 16);
-      const uint32_t d0 = lq + (uint32_t)(p.dbase + bf0 * p.NP);
-      const uint32_t d1 = lq + (uint32_t)(p.dbase + (p.nbuf + bf1) * p.NP);
+      cp_async_wait_group<kAlphaAhead - 1>();   // tile u's group has landed
+      const float sa = live ? 0.5f * s_alpha[u % kAlphaAhead][et] : 0.f;
+      alpha_fetch(u + kAlphaAhead);
       int m = 0, t = 0;
       float acc = 0.f;
       for (int c0 = 0; c0 < MT; c0 += 16) {
-        uint32_t r0[16], r1[16];
-        if (in0) tmem_ld16(d0 + (uint32_t)c0, r0);
-        if (in1) tmem_ld16(d1 + (uint32_t)c0, r1);
-        tmem_ld_wait();
+        float sum[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) sum[i] = 0.f;
+#pragma unroll
+        for (int e = 0; e < kMaxPipes; ++e) {
+          if ((in >> e) & 1u) {
+            uint32_t rr[16];
+            tmem_ld16(lq + (uint32_t)(p.dbase + (e * p.nbuf + kc[e] % p.nbuf) * p.NP + c0), rr);
+            tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 16; ++i) sum[i] += __uint_as_float(rr[i]);
+          }
+        }
         if (c0 + 16 >= MT) {
           tc_fence_before();
-          if (in0) mbar_arrive(&acc_empty[0][bf0]);
-          if (in1) mbar_arrive(&acc_empty[1][bf1]);
-        }
 #pragma unroll
+          for (int e = 0; e < kMaxPipes; ++e)
+            if ((in >> e) & 1u) mbar_arrive(&acc_empty[e][kc[e] % p.nbuf]);
+        }
+        // (not unrolled: this code runs once per tile, and unrolled it is
+        // cold instruction memory every time, each miss an L2 round trip
+        // while the code stream loads it)
+#pragma unroll 1
         for (int i = 0; i < 16; ++i) {
           if (c0 + i < MT) {
-            acc += (in0 ? __uint_as_float(r0[i]) : 0.f) + (in1 ? __uint_as_float(r1[i]) : 0.f);
+            acc += sum[i];
             if (++t == p.T) {   // the terms of batch row m, already scaled by their B scales
               if (p.S == 1) {
                 if (live) p.y[(size_t)m * p.n_out + row] = sa * acc;
               } else if (p.atomic_y) {
-                if (live) atomicAdd(p.y + (size_t)m * p.n_out + row, sa * acc);
+                if (live) red_add_f32(p.y + (size_t)m * p.n_out + row, sa * acc);
               } else {
                 p.part[((size_t)sidx * p.M + m) * NR + row] = acc;
               }
@@ -522,8 +578,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
           }
         }
       }
-      kc[0] += in0;
-      kc[1] += in1;
+#pragma unroll
+      for (int e = 0; e < kMaxPipes; ++e) kc[e] += (in >> e) & 1u;
     }
   }
   if (!ok) call_record_fail(p.rec, p.call);
@@ -584,7 +640,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
     }
   }
   if (warp == 0) {
-    __syncwarp();   // warp-collective: lane 0 ran the producer loop alone
+    __syncwarp();   // warp-collective: lane 0 ran the issuer loop alone
     tc_fence_after();
     tmem_dealloc(tmem, 512);
   }
@@ -592,84 +648,102 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
 
 }  // namespace
 
-// Launch shape for batch M: the (S, P) grid of at most one CTA per SM (more
-// only where nothing else fits) that minimises a simple time model: the larger of the MMA time of the busiest
-// CTA and the HBM time of codes plus split-K partials (the bytes in flight
-// capped by the CTAs' code rings), plus the split-K tail (one fence, one
-// ticket, the final sums).  TMEM holds, from column 0: four A slots of sb
-// blocks (16 sb columns each), the A scales (4 columns), one set of
-// ss = 4 ceil(ceil(NP / 32) / 4) B scale columns per block of the chunk, and
-// at the top the accumulators (2 pipelines x nbuf x NP columns).
+// Launch shape for batch M: the pipelines, TMEM slots, accumulators, stage
+// size and (S, P) grid of at most one CTA per SM (more only where nothing
+// else fits) that minimise a time model fitted to per-stage timestamps of
+// the kernel: per CTA the stage rate of its MMA pipelines (about 150 cycles
+// per MMA and 550 per stage on an issuing thread, the pipelines side by
+// side) and of its 4 expander sets (a set waits for the MMAs of its
+// previous stage when it owns one TMEM slot), against the HBM time of the
+// codes (the bytes in flight capped by the CTAs' code rings, at a loaded
+// latency), plus the prologue (B operand and scales) and the split-K tail.
+// TMEM holds, from column 0: ns A slots of sb blocks (16 sb columns each),
+// the A scales (4 columns), per slot the B scales of its sb blocks (a set of
+// ss = 4 ceil(ceil(NP / 32) / 4) columns per block: scale columns start on a
+// multiple of 4), and at the top the accumulators (npipe x nbuf x NP
+// columns).
 DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
   const Geometry& g = pl->geo;
   DecodeConfig best{};
   best.M = M;
   best.T = decode_terms(M);
   best.NP = (M * best.T + 15) / 16 * 16;
-  best.nbuf = best.NP <= 64 ? 2 : 1;
-  best.dbase = 512 - 2 * best.nbuf * best.NP;
   best.ss = 4 * (((best.NP + 31) / 32 + 3) / 4);
   const int KB = (int)(g.k_eff_pad / kBlk);
   const int sms = std::max(1, pl->sm_count);
   const int blk_bytes = kTileRows * kBlk * g.bits / 8;
-  // M = 1 constants fitted to measured launches: each split-K tile costs
-  // its epilogue (partial stores, a release fence and a ticket round trip
-  // while the code stream loads HBM) beyond its MMAs, and the ring's copies
-  // see a longer loaded latency.
-  const double clk = 1.9e9, bw = 6.5e12;
-  const double latency = M == 1 ? 3.0e-6 : 2.2e-6;             // loaded HBM latency
-  const double t_tile = M == 1 ? 0.5e-6 : 0.0;                 // per split-K tile
-  const double t_blk = 2.0 * std::max(32.0, best.NP * 0.3) / clk;   // two MMAs, two issuers
+  const double clk = 1.9e9, bw = 6.0e12, latency = 2.5e-6;   // loaded HBM latency (bulk copies)
+  const double c_mma = 150.0 + 0.5 * best.NP, c_stage = 550.0;   // issuing thread, cycles
+  const double c_xblk = 200.0, c_xstage = 600.0;                 // expander set, cycles
   const double code_bytes = (double)g.ntiles * kTileRows * g.k_eff_pad * g.bits / 8;
   double best_t = 1e30;
-  // k chunks beyond the SM count (CTAs in several waves) only where the
-  // chunk's B operand and scales would not fit otherwise (large batches on
-  // small parts)
-  for (int S = 1; S <= KB && (S <= sms || best.S == 0); ++S) {
-    const int CB = (KB + S - 1) / S;
-    if ((S - 1) * CB >= KB) continue;                      // no empty chunk
-    const int sfcols = (kSfaCols + CB * best.ss + 31) / 32 * 32;   // scale columns, stored 32 at a time
-    const int sb = std::min(kMaxSb, (best.dbase - sfcols) / 64);
-    if (sb < 1) continue;                                  // TMEM
-    const int b_bytes = (CB / 2 + 1) * best.NP * 128;       // image rows of the chunk's blocks
-    const int sfb_bytes = (CB * best.NP * 4 + 15) / 16 * 16;  // its B scale words
-    const int slot_bytes = sb * blk_bytes;
-    int ring = std::min(kMaxRing, (kSmemMax - 2048 - b_bytes - sfb_bytes) / slot_bytes);
-    ring -= ring % kExpSets;          // each ring slot belongs to one expander set
-    if (ring < kExpSets) continue;
-    const int spu = std::max((CB + sb - 1) / sb, std::min(2, CB));
-    if (spu > kMaxSpu) continue;
-    // the B operand of the chunk, built before the first MMA: a latency
-    // floor plus the e2m1 terms of CB 128-code blocks per batch row
-    const double t_build = 2.0e-6 + CB * M * best.T * 4.0e-9;
-    for (int P = 1; P <= std::min(g.ntiles, std::max(1, sms / S)); ++P) {
-      const int grid = S * P;
-      const int waves = (grid + sms - 1) / sms;
-      const int units = (g.ntiles + P - 1) / P;
-      const double inflight = (double)grid * ring * slot_bytes;   // code bytes in flight
-      const double bw_eff = std::min(bw, inflight / latency);
-      const double part_bytes = S > 1 ? 8.0 * S * M * g.ntiles * kTileRows : 0.0;
-      // split-K: the CTA that sums a tile reads S partials for each of its
-      // 128 M (m, row) pairs, in rounds of 16 loads (~1.2 us a round).  M = 1:
-      // summed per tile by the epilogue while MMAs go on (within the fixed
-      // split-K tail below).  Else M x 128 / 768 pairs per thread of the whole
-      // CTA after the main loop, about units / S tiles per CTA (rotated tile
-      // orders).
-      const bool now = M == 1;
-      const int rounds = (kTileRows * M + kThreads - 1) / kThreads * ((S + 15) / 16);
-      const double red = S <= 1 || now ? 0.0 : (double)((units + S - 1) / S) * rounds * 1.2e-6;
-      const double tail = S > 1 ? 2.5e-6 + red : 0.0;
-      const double t_cta = units * (CB * t_blk + spu * 90.0 / clk + 300.0 / clk + (S > 1 ? t_tile : 0.0));
-      const double t = std::max(waves * t_cta, (code_bytes + part_bytes) / bw_eff) + tail + t_build;
-      if (t < best_t * 0.999) {
-        best_t = t;
-        best.S = S; best.P = P; best.CB = CB; best.ring = ring; best.sb = sb;
-        best.smem = std::max<size_t>(kSmemMin, 1024 + (size_t)b_bytes + sfb_bytes + (size_t)ring * slot_bytes);
+  const int pipes[3] = {4, 2, 1};
+  for (int pi = 0; pi < 3; ++pi) {
+    const int np = pipes[pi];
+    for (int ns = 4; ns <= kASlots; ns *= 2)
+      for (int nbuf = 2; nbuf >= 1; --nbuf) {
+        const int dbase = 512 - np * nbuf * best.NP;
+        // k chunks beyond the SM count (CTAs in several waves) only where the
+        // chunk's B operand and scales would not fit otherwise (large batches
+        // on small parts)
+        // TMEM slot: 16 sb code columns and sb ss B scale columns; then A's scales
+        const int sb = std::min(kMaxSb, (dbase - kSfaCols) / (ns * (kAColsPerBlk + best.ss)));
+        if (sb < 1) continue;                                    // TMEM
+        for (int S = 1; S <= KB && (S <= sms || best.S == 0); ++S) {
+          const int CB = (KB + S - 1) / S;
+          if ((S - 1) * CB >= KB) continue;                      // no empty chunk
+          const int b_bytes = (CB / 2 + 1) * best.NP * 128;       // image rows of the chunk's blocks
+          const int sfb_bytes = (CB * best.NP * 4 + 15) / 16 * 16;  // its B scale words
+          const int slot_bytes = sb * blk_bytes;
+          // code bytes in flight per CTA: about the SM's share of HBM
+          // bandwidth at the loaded latency, at least two stages per set
+          int ring = std::min(kMaxRing, (kSmemMax - 2048 - b_bytes - sfb_bytes) / slot_bytes);
+          ring = std::min(ring, std::max(2 * kExpSets, (kRingBytes + slot_bytes - 1) / slot_bytes + kExpSets - 1));
+          ring -= ring % kExpSets;          // each ring slot belongs to one expander set
+          if (ring < kExpSets) continue;
+          const int spu = std::max((CB + sb - 1) / sb, std::min(2, CB));
+          if (spu > kMaxSpu) continue;
+          const double issue = 2.0 * sb * c_mma + c_stage;        // cycles per stage, one pipeline
+          const double expand = c_xstage + c_xblk * sb;           // cycles per stage, one set
+          const double set_cyc = ns == 4 ? std::max(expand, issue * 4.0 / np + 300.0) : std::max(expand, issue * 2.0 / np);
+          const double rate = std::min(np / issue, kExpSets / set_cyc);   // stages per cycle per CTA
+          // the prologue: a latency floor, the B operand (image copy or terms
+          // formed in the CTA) and the scale columns
+          const double t_build = 2.5e-6 + CB * M * best.T * 2.0e-9;
+          for (int P = 1; P <= std::min(g.ntiles, std::max(1, sms / S)); ++P) {
+            const int grid = S * P;
+            const int waves = (grid + sms - 1) / sms;
+            const int units = (g.ntiles + P - 1) / P;
+            // per row tile: its stages on the pipelines, or the epilogue of a
+            // tile (accumulator reads, the split-K adds; overlapped with the
+            // next nbuf - 1 tiles' MMAs), whichever is longer; the last
+            // tile's epilogue is exposed
+            const double t_tile = spu / rate / clk;
+            const double t_epi = 1.5e-6 + 0.02e-6 * M;
+            const double t_cta = units * std::max(t_tile, nbuf == 2 ? t_epi : t_tile + t_epi) + t_epi;
+            const double inflight = (double)grid * ring * slot_bytes;   // code bytes in flight
+            const double bw_eff = std::min(bw, inflight / latency);
+            const double part_bytes = S > 1 ? 8.0 * S * M * g.ntiles * kTileRows : 0.0;
+            // split-K tail: the CTA that sums a tile reads S partials for each of
+            // its 128 M (m, row) pairs, in rounds of 16 loads (~1.2 us a round),
+            // about units / S tiles per CTA (rotated tile orders); with float
+            // atomics only the adds themselves
+            const int rounds = (kTileRows * M + kThreads - 1) / kThreads * ((S + 15) / 16);
+            const double red = S <= 1 ? 0.0 : (double)((units + S - 1) / S) * rounds * 1.2e-6;
+            const double tail = 1.0e-6 + (S > 1 ? red : 0.0);
+            const double t = std::max(waves * t_cta, (code_bytes + part_bytes) / bw_eff) + tail + t_build;
+            if (t < best_t * 0.999) {
+              best_t = t;
+              best.S = S; best.P = P; best.CB = CB; best.ring = ring; best.sb = sb;
+              best.npipe = np; best.ns = ns; best.nbuf = nbuf; best.dbase = dbase;
+              best.smem = std::max<size_t>(kSmemMin, 1024 + (size_t)b_bytes + sfb_bytes + (size_t)ring * slot_bytes);
+            }
+          }
+        }
       }
-    }
   }
-  best.sfa = 64 * best.sb;
-  best.sfb = best.sfa + kSfaCols;
+  best.sfa = best.ns * kAColsPerBlk * best.sb;
+  best.sfs = best.sfa + kSfaCols;
   return best;
 }
 
@@ -687,9 +761,9 @@ extern "C" int sdq_decode_launch_shape(const sdq_layer_desc* desc, int32_t M, in
   const DecodeConfig dc = decode_config_search(&pl, M);
   if (dc.S < 1) return SDQ_ERR_UNSUPPORTED;
   const int64_t blk = (int64_t)kTileRows * kBlk * pl.geo.bits / 8;
-  const int64_t v[13] = {dc.T, dc.NP, dc.S, dc.P, dc.CB, dc.ring, dc.sb, dc.nbuf, (int64_t)dc.smem,
-                         dc.sb * blk, (int64_t)(dc.CB / 2 + 1) * dc.NP * 128, dc.ss, kSmemMax + 1024};
-  for (int i = 0; i < 13; ++i) out[i] = v[i];
+  const int64_t v[15] = {dc.T, dc.NP, dc.S, dc.P, dc.CB, dc.ring, dc.sb, dc.nbuf, (int64_t)dc.smem,
+                         dc.sb * blk, (int64_t)(dc.CB / 2 + 1) * dc.NP * 128, dc.ss, kSmemMax + 1024, dc.npipe, dc.ns};
+  for (int i = 0; i < 15; ++i) out[i] = v[i];
   return SDQ_OK;
 }
 
@@ -718,7 +792,8 @@ cudaError_t launch_decode(const sdq_plan_s* pl, const uint32_t* codes, const flo
   p.k_eff = g.k_eff; p.kpad = g.k_eff_pad;
   p.M = M; p.T = dc.T; p.NP = dc.NP; p.S = dc.S; p.P = dc.P; p.CB = dc.CB;
   p.KB = (int)(g.k_eff_pad / kBlk); p.ring = dc.ring;
-  p.sb = dc.sb; p.nbuf = dc.nbuf; p.dbase = dc.dbase; p.sfa = dc.sfa; p.sfb = dc.sfb; p.ss = dc.ss;
+  p.sb = dc.sb; p.nbuf = dc.nbuf; p.npipe = dc.npipe; p.ns = dc.ns; p.ns_log2 = dc.ns == 8 ? 3 : 2;
+  p.dbase = dc.dbase; p.sfa = dc.sfa; p.sfs = dc.sfs; p.ss = dc.ss;
   p.n_out = g.n_out; p.ntiles = g.ntiles; p.ngroups = g.ngroups; p.ternary = g.bits == 2;
   p.early = early;
   p.atomic_y = y_zeroed && dc.S > 1;
@@ -727,9 +802,12 @@ cudaError_t launch_decode(const sdq_plan_s* pl, const uint32_t* codes, const flo
   p.b_bytes = (uint32_t)((dc.CB / 2 + 1) * dc.NP * 128);
   p.sfb_bytes = (uint32_t)((dc.CB * dc.NP * 4 + 15) / 16 * 16);
   static std::atomic<int> smem_set[64];   // per device: limit raised to kSmemMax + 1 KB
-  cudaError_t e = smem_limit_once(decode_kernel, kSmemMax + 1024, pl->device, smem_set);
+  static std::atomic<int> smem_set_b[64];
+  cudaError_t e = p.ternary ? smem_limit_once(decode_kernel<true>, kSmemMax + 1024, pl->device, smem_set)
+                            : smem_limit_once(decode_kernel<false>, kSmemMax + 1024, pl->device, smem_set_b);
   if (e != cudaSuccess) return e;
-  return launch_pdl(decode_kernel, dim3(dc.S * dc.P), dim3(kThreads), dc.smem, st, p);
+  return p.ternary ? launch_pdl(decode_kernel<true>, dim3(dc.S * dc.P), dim3(kThreads), dc.smem, st, p)
+                   : launch_pdl(decode_kernel<false>, dim3(dc.S * dc.P), dim3(kThreads), dc.smem, st, p);
 }
 
 }  // namespace sdq

@@ -45,7 +45,7 @@ constexpr int kMaxDecodeM = 64;
 inline int decode_terms(int M) { return M <= 4 ? 6 : (M <= 16 ? 4 : 3); }
 
 // Launch shape of the decode kernel for one batch size (chosen at plan time).
-// Grid = S * P CTAs, one per SM: CTA (s, p) contracts k chunk s (CB blocks
+// Grid = S * P CTAs, one per SM (more in waves only where nothing else fits): CTA (s, p) contracts k chunk s (CB blocks
 // of 128 codes) against row tiles p, p + P, p + 2P, ...
 struct DecodeConfig {
   int M, T, NP;           // batch, e2m1 terms per activation, MMA N (M*T rounded up to 16)
@@ -53,9 +53,11 @@ struct DecodeConfig {
   int ring;               // code stages in the shared-memory ring
   int sb;                 // 128-code blocks per stage
   int nbuf;               // accumulators per pipeline
+  int npipe;              // MMA pipelines (issuing warps, each with its accumulators)
+  int ns;                 // TMEM A slots (4 or 8)
   int dbase;              // TMEM column of the first accumulator
-  int sfa, sfb, ss;       // TMEM columns of the A scales, of the first block's
-                          // B scales, and between two blocks' B scales
+  int sfa, sfs, ss;       // TMEM columns of the A scales, of TMEM slot 0's B
+                          // scales, and between two blocks' B scales
   size_t smem;            // dynamic shared memory of the decode kernel
 };
 

@@ -120,11 +120,12 @@ def test_decode_launch_shapes_fit(sdq, sms):
     """Every decode launch shape the plan would choose keeps the kernel's
     invariants: at most one CTA per SM (or one per k chunk, where a chunk's
     B operand would not fit otherwise), k chunks covering K with none empty,
-    a ring of 4..24 stages in multiples of 4, TMEM columns within 512 (four
-    A slots of 16 sb columns, 4 A-scale columns and one 4-aligned set of
-    B-scale columns per block, stored 32 columns at a time, the
-    accumulators), the B image, its scale words and the ring within the
-    shared-memory limit, and the e2m1 term count of the batch size."""
+    a ring of 4..32 stages in multiples of 4 (one expander set per ring
+    slot), 1, 2 or 4 MMA pipelines, TMEM columns within 512 (4 or 8 slots of
+    16 sb code columns and sb 4-aligned sets of B-scale columns, 4 A-scale
+    columns, npipe x nbuf accumulators), the B
+    image, its scale words and the ring within the shared-memory limit, and
+    the e2m1 term count of the batch size."""
     for n, k, b, osr, qz in _launch_shapes():
         d = sdq.LayerDesc(n, k, b, osr, qz, 1, 0)
         kb = -(-sdq.sdq_k_eff(d) // 128)
@@ -135,11 +136,11 @@ def test_decode_launch_shapes_fit(sdq, sms):
             assert s["T"] == t and s["NP"] == -(-(m * t) // 16) * 16
             assert 1 <= s["S"] and 1 <= s["P"] and (s["S"] * s["P"] <= sms or s["P"] == 1)
             assert (s["S"] - 1) * s["CB"] < kb <= s["S"] * s["CB"]
-            assert 4 <= s["ring"] <= 24 and s["ring"] % 4 == 0
-            assert s["nbuf"] == (2 if s["NP"] <= 64 else 1)
+            assert 4 <= s["ring"] <= 32 and s["ring"] % 4 == 0
+            assert s["npipe"] in (1, 2, 4) and s["nbuf"] in (1, 2) and s["ns"] in (4, 8)
             assert s["ss"] == 4 * (-(-(-(-s["NP"] // 32)) // 4))
             assert 1 <= s["sb"] <= 4
-            assert 64 * s["sb"] + -(-(4 + s["CB"] * s["ss"]) // 32) * 32 + 2 * s["nbuf"] * s["NP"] <= 512
+            assert s["ns"] * s["sb"] * (16 + s["ss"]) + 4 + s["npipe"] * s["nbuf"] * s["NP"] <= 512
             assert s["slot_bytes"] == s["sb"] * blk
             assert s["b_bytes"] == (s["CB"] // 2 + 1) * s["NP"] * 128
             sfb = -(-(s["CB"] * s["NP"] * 4) // 16) * 16   # the chunk's B scale words
