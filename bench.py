@@ -213,6 +213,161 @@ def alg_bytes(lay, M):
     return lin.n_out * k_eff * 2 // 8 + 4 * lin.n_out + 2 * M * lin.k_in + 4 * M * lin.n_out
 
 
+def random_plan(P, torch, n, k, block, osr, quantizer, seed):
+    """A plan and random valid codes in the tiled layout, drawn on the device
+    (timing legs: the contraction's work does not depend on the code values;
+    ternary fields 10 are mapped to 00)."""
+    from fractions import Fraction
+    desc = P.LayerDesc(n, k, block, Fraction(osr), quantizer)
+    plan = P.Plan(desc)
+    nw = P.sdq_tiled_bytes(desc) // 4
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed)
+    w = torch.randint(-2 ** 31, 2 ** 31 - 1, (nw,), generator=g, device="cuda", dtype=torch.int64).to(torch.int32)
+    if quantizer == P.SDQ_TERNARY:
+        w &= ~(((~w) << 1) & -0x55555556)
+    alpha = torch.full((n,), 0.02, dtype=torch.float32, device="cuda")
+    return {"plan": plan, "tiled": w, "alpha": alpha, "code_bytes": P.sdq_tiled_bytes(desc), "n": n, "k": k}
+
+
+def graph_step_ms(torch, stream, calls, reps=50, warm=5):
+    """Mean time of one replay of a CUDA graph of `calls` (callables taking
+    the stream), events on the replay stream."""
+    with torch.cuda.stream(stream):
+        for _ in range(2):
+            for c in calls:
+                c(stream)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for c in calls:
+            c(stream)
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        for _ in range(warm):
+            g.replay()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            g.replay()
+        b.record(stream)
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / reps
+
+
+def fwd_call(P, lay, x, y, ws, M):
+    return lambda st: P.sdq_linear_forward(lay["plan"].handle, lay["tiled"], lay["alpha"], x, M, y, ws, st)
+
+
+def step_leg(P, torch, stream, lays, M, reps=50):
+    """Decode step over `lays` (one sdq_linear_forward per linear, graph-replayed):
+    weight GB/s over the step."""
+    calls, keep = [], []
+    for lay in lays:
+        x = torch.randn(M, lay["k"], device="cuda").to(torch.bfloat16)
+        y = torch.empty(M, lay["n"], dtype=torch.float32, device="cuda")
+        ws = lay["plan"].alloc_workspace(M)
+        keep += [x, y, ws]
+        calls.append(fwd_call(P, lay, x, y, ws, M))
+    ms = graph_step_ms(torch, stream, calls, reps)
+    tot = sum(l["code_bytes"] for l in lays)
+    return {"GBps": round(tot / (ms * 1e-3) / 1e9, 1), "us_per_step": round(ms * 1e3, 2),
+            "code_bytes_per_step": tot, "calls": len(lays)}
+
+
+def extra_configs_leg(P, W, torch, stream, hbm):
+    """The other workloads, with random device codes: OPT-125M per-linear
+    latency (L2 flushed before each call) at M = 1 and 16; the LLaMA-7B layer
+    step at M = 1, 4, 16, 64; the LLaMA-13B 4-layer stack under the MultiOSR
+    map: M = 8 decode step and M = 2048 prefill (contraction alone and with its
+    prepare kernel)."""
+    import numpy as np
+    from paper_2510_03275_gb300.multiosr import allocate
+    out = {}
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    # OPT-125M
+    cfg = W.config(1)
+    lat = {}
+    for lin in cfg.linears:
+        lay = random_plan(P, torch, lin.n_out, lin.k_in, cfg.block, lin.osr, cfg.quantizer, lin.seed)
+        for M in (1, 16):
+            x = torch.randn(M, lin.k_in, device="cuda").to(torch.bfloat16)
+            y = torch.empty(M, lin.n_out, dtype=torch.float32, device="cuda")
+            ws = lay["plan"].alloc_workspace(M)
+            for _ in range(3):
+                P.sdq_linear_forward(lay["plan"].handle, lay["tiled"], lay["alpha"], x, M, y, ws, stream)
+            ts = []
+            for i in range(15):
+                with torch.cuda.stream(stream):
+                    flush.fill_(i)
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                P.sdq_linear_forward(lay["plan"].handle, lay["tiled"], lay["alpha"], x, M, y, ws, stream)
+                b.record(stream)
+                torch.cuda.synchronize()
+                ts.append(a.elapsed_time(b) * 1e3)
+            ts.sort()
+            us = ts[len(ts) // 2]
+            lat.setdefault(str(M), {})[lin.name] = {"us": round(us, 2),
+                                                    "GBps_l2_flushed": round(lay["code_bytes"] / us / 1e3, 1)}
+    out["opt125m"] = {"what": "per-linear latency of one sdq_linear_forward (prepare + contraction), L2 "
+                              "flushed before each call, median of 15; binary codes, OSR 5/2",
+                      "by_batch": lat}
+    # LLaMA-7B
+    cfg = W.config(2)
+    lays = [random_plan(P, torch, l.n_out, l.k_in, cfg.block, l.osr, cfg.quantizer, l.seed) for l in cfg.linears]
+    sweep = {}
+    for M in (1, 4, 16, 64):
+        r = step_leg(P, torch, stream, lays, M, reps=30)
+        r["frac_of_hbm"] = round(r["GBps"] / hbm, 4)
+        sweep[str(M)] = r
+    out["llama7b_layer"] = {"what": "decode step (7 linears, graph-replayed), weight GB/s per batch size",
+                            "by_batch": sweep}
+    del lays
+    # LLaMA-13B 4-layer stack, MultiOSR
+    cfg = W.config(3, multiosr=allocate)
+    lays = [random_plan(P, torch, l.n_out, l.k_in, cfg.block, l.osr, cfg.quantizer, l.seed) for l in cfg.linears]
+    dec = step_leg(P, torch, stream, lays, 8, reps=10)
+    dec["frac_of_hbm"] = round(dec["GBps"] / hbm, 4)
+    M = 2048
+    ms_k5, ms_all, flops = 0.0, 0.0, 0
+    for lay, lin in zip(lays, cfg.linears):
+        x = torch.randn(M, lin.k_in, device="cuda").to(torch.bfloat16)
+        y = torch.empty(M, lin.n_out, dtype=torch.float32, device="cuda")
+        ws = lay["plan"].alloc_workspace(M)
+        P.sdq_prep_activations(lay["plan"].handle, x, M, ws, stream)
+        P.sdq_contract(lay["plan"].handle, lay["tiled"], lay["alpha"], M, y, ws, stream)
+        ms_k5 += graph_step_ms(torch, stream, [lambda st, lay=lay, y=y, ws=ws: P.sdq_contract(
+            lay["plan"].handle, lay["tiled"], lay["alpha"], M, y, ws, st)], reps=5, warm=2)
+        ms_all += graph_step_ms(torch, stream, [fwd_call(P, lay, x, y, ws, M)], reps=5, warm=2)
+        flops += 2 * M * lin.n_out * lay["plan"].k_eff
+        del x, y, ws
+    out["llama13b_4layers_multiosr"] = {
+        "osr": sorted({str(l.osr) for l in cfg.linears}),
+        "decode_m8": dec,
+        "prefill_m2048": {"tflops_contraction": round(flops / (ms_k5 * 1e-3) / 1e12, 1),
+                          "tflops_with_prepare": round(flops / (ms_all * 1e-3) / 1e12, 1),
+                          "ms_contraction": round(ms_k5, 3), "ms_with_prepare": round(ms_all, 3),
+                          "flops": flops}}
+    del lays, flush
+    torch.cuda.empty_cache()
+    return out
+
+
+def fused_groups_leg(P, torch, stream, hbm, M=1):
+    """The LLaMA-70B layer with q/k/v and gate/up each stored as one matrix
+    (rows concatenated: they read the same input), 4 calls per step; random
+    device codes."""
+    shapes = [("qkv", 10240, 8192), ("o", 8192, 8192), ("gate_up", 57344, 8192), ("down", 8192, 28672)]
+    lays = [random_plan(P, torch, n, k, 128, 2, P.SDQ_TERNARY, 1234 + i) for i, (_, n, k) in enumerate(shapes)]
+    r = step_leg(P, torch, stream, lays, M, reps=50)
+    r["frac_of_hbm"] = round(r["GBps"] / hbm, 4)
+    r["groups"] = [f"{nm} {n}x{k}" for nm, n, k in shapes]
+    del lays
+    torch.cuda.empty_cache()
+    return r
+
+
 def run_sdq(args, rank, world, dist):
     import numpy as np
     import torch
@@ -364,7 +519,7 @@ def run_sdq(args, rank, world, dist):
         "metric": METRIC, "value": round(value, 1), "unit": "GB/s",
         "n_gpus": world, "steps": args.steps, "warmup": max(3, args.warmup),
         "ms_per_step": round(ms_step, 5), "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "u2-codes/e4m3-mma/f32-acc", "data": "synthetic",
+        "vs_baseline": None, "dtype": "u2-codes/e2m1-mma(mxf4)/f32-acc", "data": "synthetic",
         "config": {"workload": "llama70b-layer decode: q/o 8192x8192, k/v 1024x8192, "
                                "gate/up 28672x8192, down 8192x28672; OSR 2 ternary B=128"
                                + (f" [only {args.linears}]" if args.linears else ""),
@@ -381,15 +536,20 @@ def run_sdq(args, rank, world, dist):
         "gpu_launches": sum(lay["kernels"] for lay in layers) * args.steps,
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
                      "unit": "GB/s", "frac": round(achieved / hbm, 4), "traffic": traffic,
-                     "kernel": "decode_kernel (" + ("one-kernel sdq_linear_forward"
-                                                    if all(l["kernels"] == 1 for l in layers)
-                                                    else "sdq_contract") + f", M={M})",
+                     "kernel": f"decode_kernel, per launch (sdq_contract after its prepare kernel, M={M})",
                      "peak_source": peak_src,
                      "nominal_8tbs_frac": round(achieved / 8000.0, 4), "per_linear": per_lin},
+        "roofline_per_step": {"bound": "hbm", "achieved": round(value, 1), "peak": hbm, "unit": "GB/s",
+                              "frac": round(value / hbm, 4),
+                              "what": "code bytes of the step / step time: both kernels of every call "
+                                      "and the gaps between them"},
         "encode": {"ms_per_layer": round(enc_ms, 3), "what": "sdq_encode_rows + sdq_pack, 7 linears"},
     }
+    if rank == 0:
+        out["fused_groups"] = fused_groups_leg(P, torch, stream, hbm, M)
     if not args.no_extras and rank == 0:
         out["decode_sweep"] = decode_sweep(P, W, torch, layers, stream, hbm, tf_burst, peak_src)
+        out["other_configs"] = extra_configs_leg(P, W, torch, stream, hbm)
         out["prefill"] = prefill_leg(P, W, torch, layers, stream, tf_burst, tf_sus, peak_src)
         out["cpu_baseline"] = cpu_baseline_leg()
         try:
@@ -448,7 +608,7 @@ def decode_sweep(P, W, torch, layers, stream, hbm_gbs, tf_bf16, peak_src):
 def prefill_leg(P, W, torch, layers, stream, tf_burst, tf_sus, peak_src):
     import numpy as np
     M = 4096
-    flops, ms = 0, 0.0
+    flops, ms, ms_p = 0, 0.0, 0.0
     try:
         for lay in layers:
             lin = lay["lin"]
@@ -457,15 +617,22 @@ def prefill_leg(P, W, torch, layers, stream, tf_burst, tf_sus, peak_src):
             ws = lay["plan"].alloc_workspace(M)
             P.sdq_prep_activations(lay["plan"].handle, x, M, ws, stream)
             P.sdq_contract(lay["plan"].handle, lay["tiled"], lay["alpha"], M, y, ws, stream)
-            evs = []
+            evs, evp = [], []
             for _ in range(5):
                 a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
                 a.record(stream)
                 P.sdq_contract(lay["plan"].handle, lay["tiled"], lay["alpha"], M, y, ws, stream)
                 b.record(stream)
                 evs.append((a, b))
+            for _ in range(5):
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                P.sdq_linear_forward(lay["plan"].handle, lay["tiled"], lay["alpha"], x, M, y, ws, stream)
+                b.record(stream)
+                evp.append((a, b))
             torch.cuda.synchronize()
             ms += sum(a.elapsed_time(b) for a, b in evs) / len(evs)
+            ms_p += sum(a.elapsed_time(b) for a, b in evp) / len(evp)
             flops += 2 * M * lin.n_out * lay["plan"].k_eff
             del x, y, ws
     except P.SdqError as e:
@@ -473,6 +640,10 @@ def prefill_leg(P, W, torch, layers, stream, tf_burst, tf_sus, peak_src):
     tflops = flops / (ms * 1e-3) / 1e12
     return {"value": round(tflops, 1), "unit": "TFLOP/s", "M": M, "ms_per_layer": round(ms, 3),
             "flops_per_layer": flops,
+            "with_prepare": {"value": round(flops / (ms_p * 1e-3) / 1e12, 1), "unit": "TFLOP/s",
+                             "ms_per_layer": round(ms_p, 3),
+                             "what": "sdq_linear_forward: the prepare kernel (x_tilde in bf16) and the "
+                                     "contraction"},
             "roofline": {"bound": "tensor", "achieved": round(tflops, 1), "peak": tf_burst,
                          "unit": "TFLOP/s", "frac": round(tflops / tf_burst, 4),
                          "peak_source": peak_src + " bf16 burst"}}

@@ -66,8 +66,9 @@
 //                 tiled layout) into the ring with bulk copies: a thread
 //                 starts a bulk copy only every ~600 cycles, four side by
 //                 side keep an SM's share of HBM busy
-// With `early` set the producers start the code stream before waiting for
-// the preceding grid (codes are never written by the prep kernels).
+// With `early` set the producers start the code stream (one stage each)
+// before waiting for the preceding grid (codes are never written by the
+// prep kernels).
 // Every mbarrier wait is bounded (about 2 s); a timeout writes the call's
 // tag into the workspace's call record and the CTA drains its copies and
 // MMAs before freeing TMEM.
@@ -99,6 +100,7 @@ constexpr int kRedWords = 64;                    // split-K sums summed CTA-wide
 constexpr int kSfaCols = 4;                      // A scales: column 32 q + lane r holds row r's
 constexpr int kAlphaAhead = 4;                   // epilogue: alpha loads this many row tiles ahead
 constexpr int kRingBytes = 160 * 1024;           // code bytes in flight per CTA (target)
+constexpr int kEarlyStages = 1;                  // stages per producer issued before the preceding grid completes
 static_assert(kMaxRing <= 32 && kASlots == 8 && 2 * kMaxPipes + 1 + kMaxPipes <= 32 && kRedWords == 64 &&
                   kMaxSpu < 160 && kMaxRing % kExpSets == 0,
               "the prologue's per-warp set-up and the stage maps assume these bounds");
@@ -301,7 +303,12 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       int last_i = -1, u = 0, j = x, slot = x, r = 0;
       while (j >= spu) { j -= spu; ++u; }
       const uint64_t pol = l2_policy_evict_first();   // codes are read once per call
+      bool waited = !p.early;
       for (int i = x; i < nstages && ok; i += kExpSets) {
+        // with `early`, kEarlyStages stages ahead of the preceding grid: more
+        // would queue ahead of the loads that grid and this CTA's prologue
+        // make once it completes
+        if (!waited && i >= x + kExpSets * kEarlyStages) { pdl_wait(); waited = true; }
         if (r > 0) ok = mbar_wait(&c_empty[slot], (r - 1) & 1);
         if (!ok) break;
         const int b0 = sblk[j], b1 = sblk[j + 1];
@@ -317,7 +324,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         slot += kExpSets;
         if (slot >= p.ring) { slot -= p.ring; ++r; }
       }
-      if (p.early) pdl_wait();
+      if (!waited) pdl_wait();
       // Every copy this thread issued has landed before the CTA may exit.
       for (int i = last_i; i >= 0 && i > last_i - p.ring; i -= kExpSets)
         if (!mbar_wait(&c_full[i % p.ring], (i / p.ring) & 1)) ok = false;
@@ -672,10 +679,11 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
   const int KB = (int)(g.k_eff_pad / kBlk);
   const int sms = std::max(1, pl->sm_count);
   const int blk_bytes = kTileRows * kBlk * g.bits / 8;
-  const double clk = 1.9e9, bw = 6.0e12, latency = 2.5e-6;   // loaded HBM latency (bulk copies)
+  const double clk = 1.9e9;
+  const double hbm = 6.0e12, cta_bw = 30e9;                    // bytes/s: HBM, one CTA's copy ring
+  const double t_tail = 2.0e-6, ring_latency = 4.0e-6;   // a ring slot's round trip under load
   const double c_mma = 150.0 + 0.5 * best.NP, c_stage = 550.0;   // issuing thread, cycles
   const double c_xblk = 200.0, c_xstage = 600.0;                 // expander set, cycles
-  const double code_bytes = (double)g.ntiles * kTileRows * g.k_eff_pad * g.bits / 8;
   double best_t = 1e30;
   const int pipes[3] = {4, 2, 1};
   for (int pi = 0; pi < 3; ++pi) {
@@ -706,32 +714,26 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
           const double issue = 2.0 * sb * c_mma + c_stage;        // cycles per stage, one pipeline
           const double expand = c_xstage + c_xblk * sb;           // cycles per stage, one set
           const double set_cyc = ns == 4 ? std::max(expand, issue * 4.0 / np + 300.0) : std::max(expand, issue * 2.0 / np);
-          const double rate = std::min(np / issue, kExpSets / set_cyc);   // stages per cycle per CTA
-          // the prologue: a latency floor, the B operand (image copy or terms
-          // formed in the CTA) and the scale columns
-          const double t_build = 2.5e-6 + CB * M * best.T * 2.0e-9;
+          const double mma_rate = std::min(np / issue, kExpSets / set_cyc) * clk;   // stages per second per CTA
+          // the prologue: the wait for the prepare kernel, the B operand (image
+          // copy or terms formed in the CTA)
+          const double t_build = 2.0e-6 + (b_bytes + sfb_bytes) / 25e9 + CB * M * best.T * 2.0e-9;
           for (int P = 1; P <= std::min(g.ntiles, std::max(1, sms / S)); ++P) {
             const int grid = S * P;
             const int waves = (grid + sms - 1) / sms;
             const int units = (g.ntiles + P - 1) / P;
-            // per row tile: its stages on the pipelines, or the epilogue of a
-            // tile (accumulator reads, the split-K adds; overlapped with the
-            // next nbuf - 1 tiles' MMAs), whichever is longer; the last
-            // tile's epilogue is exposed
-            const double t_tile = spu / rate / clk;
-            const double t_epi = 1.5e-6 + 0.02e-6 * M;
-            const double t_cta = units * std::max(t_tile, nbuf == 2 ? t_epi : t_tile + t_epi) + t_epi;
-            const double inflight = (double)grid * ring * slot_bytes;   // code bytes in flight
-            const double bw_eff = std::min(bw, inflight / latency);
-            const double part_bytes = S > 1 ? 8.0 * S * M * g.ntiles * kTileRows : 0.0;
-            // split-K tail: the CTA that sums a tile reads S partials for each of
-            // its 128 M (m, row) pairs, in rounds of 16 loads (~1.2 us a round),
-            // about units / S tiles per CTA (rotated tile orders); with float
-            // atomics only the adds themselves
-            const int rounds = (kTileRows * M + kThreads - 1) / kThreads * ((S + 15) / 16);
-            const double red = S <= 1 ? 0.0 : (double)((units + S - 1) / S) * rounds * 1.2e-6;
-            const double tail = 1.0e-6 + (S > 1 ? red : 0.0);
-            const double t = std::max(waves * t_cta, (code_bytes + part_bytes) / bw_eff) + tail + t_build;
+            // A CTA streams its units row tiles (CB blocks each) at the
+            // lowest of: the measured per-CTA ceiling of the copy ring, its
+            // share of HBM bandwidth, and the rate its MMA pipelines and
+            // expander sets sustain; every row tile adds a cost that grows
+            // with the k chunks adding into the same rows of y (accumulator
+            // hand-off, epilogue, split-K contention: fitted to measured
+            // calls), every call a prologue and a tail.
+            const double tile_bytes = (double)CB * blk_bytes;
+            const double rate = std::min({cta_bw, hbm / std::min(grid, sms), mma_rate * slot_bytes,
+                                          (double)ring * slot_bytes / ring_latency});
+            const double t_cta = units * (tile_bytes / rate + 0.8e-6 + 0.15e-6 * S);
+            const double t = waves * t_cta + t_build + t_tail;
             if (t < best_t * 0.999) {
               best_t = t;
               best.S = S; best.P = P; best.CB = CB; best.ring = ring; best.sb = sb;

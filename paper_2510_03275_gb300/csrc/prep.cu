@@ -165,12 +165,27 @@ __global__ void __launch_bounds__(128) prep_decode_kernel(DecPrepParams p) {
   uint16_t* xs = reinterpret_cast<uint16_t*>(dsm);   // TB x ld
   uint16_t* ghs = xs + TB * ld;                        // 64 x ld
   uint16_t* gls = ghs + 64 * ld;                       // 64 x ld
-  pdl_wait();
+  // The decode kernel may start right away: it waits for this grid to
+  // complete before it reads anything this grid writes (y, the workspace).
   pdl_launch_dependents();
   const int jt = blockIdx.x, bt = blockIdx.y, m = blockIdx.z;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, t = lane & 3;
   const int b0 = bt * TB, j0 = jt * 64, wcol = warp * 16;
   const uint16_t* xr = p.x + (size_t)m * p.K;
+  // G's rows for the first k chunk before waiting for the preceding grid: the
+  // plan's tables are never written by the stream
+  auto load_g = [&](int kc0) {
+    const int q8 = p.kc / 8;
+    for (int i = tid; i < 64 * q8; i += 128) {
+      const int rr = i / q8, q = i - rr * q8, j = j0 + rr;
+      const bool v = j < p.n_b;
+      const size_t off = v ? (size_t)j * p.B + kc0 + 8 * q : 0;
+      cp_async16(ghs + rr * ld + 8 * q, p.g_hi + off, v ? 16u : 0u);
+      cp_async16(gls + rr * ld + 8 * q, p.g_lo + off, v ? 16u : 0u);
+    }
+  };
+  if (p.vec) load_g(0);
+  pdl_wait();
   if (p.y_zero) {   // grid-stride clear of y
     const int64_t nthr = (int64_t)gridDim.x * gridDim.y * gridDim.z * 128;
     const int64_t i0 = ((int64_t)(blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x) * 128 + tid;
@@ -190,13 +205,7 @@ __global__ void __launch_bounds__(128) prep_decode_kernel(DecPrepParams p) {
         const bool v = b < p.nblk;
         cp_async16(xs + rr * ld + 8 * q, v ? xr + (size_t)b * p.B + kc0 + 8 * q : xr, v ? 16u : 0u);
       }
-      for (int i = tid; i < 64 * q8; i += 128) {
-        const int rr = i / q8, q = i - rr * q8, j = j0 + rr;
-        const bool v = j < p.n_b;
-        const size_t off = v ? (size_t)j * p.B + kc0 + 8 * q : 0;
-        cp_async16(ghs + rr * ld + 8 * q, p.g_hi + off, v ? 16u : 0u);
-        cp_async16(gls + rr * ld + 8 * q, p.g_lo + off, v ? 16u : 0u);
-      }
+      if (kc0 > 0) load_g(kc0);
     } else {
       for (int i = tid; i < TB * p.kc; i += 128) {
         const int rr = i / p.kc, kk = i - rr * p.kc, k = kc0 + kk, b = b0 + rr;
