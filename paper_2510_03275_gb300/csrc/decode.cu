@@ -118,7 +118,7 @@ struct DecodeParams {
   uint64_t call;         // call tag
   int bsrc;              // B operand from: 1 prepared x_tilde, 2 prepared image
   int64_t k_eff, kpad;
-  int M, T, NP, S, P, CB, KB, ring, sb, nbuf, npipe, ns, ns_log2, dbase, sfa, sfs, ss;
+  int M, T, NP, S, P, CB, KB, ring, sb, nbuf, npipe, ns, ns_log2, dbase, sfa, sfs, ss, sss;
   int n_out, ntiles, ngroups, ternary, early;
   int atomic_y;          // split-K by float atomic adds into y (zeroed by the prepare kernel)
   uint32_t blk_bytes, slot_bytes, b_bytes, sfb_bytes;
@@ -342,7 +342,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       const uint64_t bd0 = sw128_desc(sbase);
       const uint64_t astep = (uint64_t)((p.NP * 128) >> 4);   // descriptor units per image row pair
       const uint32_t sfa = tmem + (uint32_t)p.sfa, sfs = tmem + (uint32_t)p.sfs;
-      const uint32_t sslot = (uint32_t)(p.sb * p.ss);   // B scale columns per TMEM slot
+      const uint32_t sslot = (uint32_t)p.sss;   // B scale columns per TMEM slot
       const uint32_t aslot = (uint32_t)(kAColsPerBlk * p.sb);
       int k = 0, buf = 0, u = e / spu, j = e - (e / spu) * spu, last = -1;
       bool first = true;
@@ -461,31 +461,70 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         if (!ok) break;
         tc_fence_after();
       }
+      // Few, wide TMEM stores: a tcgen05.st costs its warp a few hundred
+      // cycles here whatever its width.  The codes first, two blocks per
+      // store ...
 #pragma unroll
-      for (int bb = 0; bb < kMaxSb; ++bb) {
-        if (bb < nb) {
+      for (int bp = 0; bp < kMaxSb; bp += 2) {
+        if (bp < nb) {
           // e2m1 nibble [sign, code bit 0, 0, 0]: +-2.0 or 0 (decode_stage_k order)
-          uint32_t v[16];
-          if constexpr (kTernary) {
+          uint32_t v[32];
 #pragma unroll
-            for (int wi = 0; wi < 8; ++wi) {
-              v[2 * wi] = (w[bb][wi] << 2) & 0xCCCCCCCCu;   // even codes
-              v[2 * wi + 1] = w[bb][wi] & 0xCCCCCCCCu;      // odd codes
+          for (int h = 0; h < 2; ++h) {
+            const int bb = bp + h;
+            if constexpr (kTernary) {
+#pragma unroll
+              for (int wi = 0; wi < 8; ++wi) {
+                v[16 * h + 2 * wi] = (w[bb][wi] << 2) & 0xCCCCCCCCu;   // even codes
+                v[16 * h + 2 * wi + 1] = w[bb][wi] & 0xCCCCCCCCu;      // odd codes
+              }
+            } else {   // words hold the inverted bits: 1 = -1
+#pragma unroll
+              for (int wi = 0; wi < 4; ++wi)
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+                  v[16 * h + 4 * wi + k] = ((w[bb][wi] << (3 - k)) & 0x88888888u) | 0x44444444u;
             }
-          } else {   // words hold the inverted bits: 1 = -1
-#pragma unroll
-            for (int wi = 0; wi < 4; ++wi)
-#pragma unroll
-              for (int k = 0; k < 4; ++k) v[4 * wi + k] = ((w[bb][wi] << (3 - k)) & 0x88888888u) | 0x44444444u;
           }
-          tmem_st16(lane_addr + (uint32_t)s * aslot + (uint32_t)(kAColsPerBlk * bb), v);
-          // the block's B scales: term row n = 32 c + lane at column c of the
-          // block's set, this warp's lane quadrant (every quadrant a copy)
+          const uint32_t ad = lane_addr + (uint32_t)s * aslot + (uint32_t)(kAColsPerBlk * bp);
+          if (bp + 1 < nb) {
+            tmem_st32(ad, v);
+          } else {
+            uint32_t v16[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) v16[i] = v[i];
+            tmem_st16(ad, v16);
+          }
+        }
+      }
+      // ... then the stage's B scales (one store for the slot when a block's
+      // set is 4 columns)
+      const uint32_t sc = lane_addr + (uint32_t)p.sfs + (uint32_t)(s * p.sss);
+      if (p.ss == 4) {
+        // column 4 bb + c: term row n = 32 c + lane of block bb; the slot's
+        // scale area is sss = 4, 8 or 16 columns, one store of that width
+        uint32_t sv[4 * kMaxSb];
+#pragma unroll
+        for (int cc = 0; cc < 4 * kMaxSb; ++cc) {
+          const int bb = cc >> 2, n = 32 * (cc & 3) + lane;
+          sv[cc] = (bb < nb && n < MT) ? reinterpret_cast<const uint32_t*>(sfbs)[(sb0 + bb) * p.NP + n]
+                                       : kUnitScales;
+        }
+        if (p.sss == 16) {
+          tmem_st16(sc, sv);
+        } else if (p.sss == 8) {
+          const uint32_t s8[8] = {sv[0], sv[1], sv[2], sv[3], sv[4], sv[5], sv[6], sv[7]};
+          tmem_st8(sc, s8);
+        } else {
+          const uint32_t s4[4] = {sv[0], sv[1], sv[2], sv[3]};
+          tmem_st4(sc, s4);
+        }
+      } else {
+        for (int bb = 0; bb < nb; ++bb) {
           const uint32_t* sw = reinterpret_cast<const uint32_t*>(sfbs) + (size_t)(sb0 + bb) * p.NP;
-          const uint32_t sc = lane_addr + (uint32_t)p.sfs + (uint32_t)(s * p.sb * p.ss + bb * p.ss);
           for (int c = 0; 32 * c < p.NP; ++c) {
             const int n = 32 * c + lane;
-            tmem_st1(sc + (uint32_t)c, n < MT ? sw[n] : kUnitScales);
+            tmem_st1(sc + (uint32_t)(bb * p.ss + c), n < MT ? sw[n] : kUnitScales);
           }
         }
       }
@@ -694,8 +733,14 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
         // k chunks beyond the SM count (CTAs in several waves) only where the
         // chunk's B operand and scales would not fit otherwise (large batches
         // on small parts)
-        // TMEM slot: 16 sb code columns and sb ss B scale columns; then A's scales
-        const int sb = std::min(kMaxSb, (dbase - kSfaCols) / (ns * (kAColsPerBlk + best.ss)));
+        // TMEM slot: 16 sb code columns and its B scale columns (sb sets of
+        // ss; with ss = 4 rounded up to 4, 8 or 16, the width of the one
+        // store that writes them); then A's scales
+        int sb = kMaxSb, sss = 0;
+        for (; sb >= 1; --sb) {
+          sss = best.ss == 4 ? (sb == 1 ? 4 : (sb == 2 ? 8 : 16)) : sb * best.ss;
+          if (ns * (kAColsPerBlk * sb + sss) + kSfaCols <= dbase) break;
+        }
         if (sb < 1) continue;                                    // TMEM
         for (int S = 1; S <= KB && (S <= sms || best.S == 0); ++S) {
           const int CB = (KB + S - 1) / S;
@@ -737,7 +782,7 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
             if (t < best_t * 0.999) {
               best_t = t;
               best.S = S; best.P = P; best.CB = CB; best.ring = ring; best.sb = sb;
-              best.npipe = np; best.ns = ns; best.nbuf = nbuf; best.dbase = dbase;
+              best.npipe = np; best.ns = ns; best.nbuf = nbuf; best.dbase = dbase; best.sss = sss;
               best.smem = std::max<size_t>(kSmemMin, 1024 + (size_t)b_bytes + sfb_bytes + (size_t)ring * slot_bytes);
             }
           }
@@ -795,7 +840,7 @@ cudaError_t launch_decode(const sdq_plan_s* pl, const uint32_t* codes, const flo
   p.M = M; p.T = dc.T; p.NP = dc.NP; p.S = dc.S; p.P = dc.P; p.CB = dc.CB;
   p.KB = (int)(g.k_eff_pad / kBlk); p.ring = dc.ring;
   p.sb = dc.sb; p.nbuf = dc.nbuf; p.npipe = dc.npipe; p.ns = dc.ns; p.ns_log2 = dc.ns == 8 ? 3 : 2;
-  p.dbase = dc.dbase; p.sfa = dc.sfa; p.sfs = dc.sfs; p.ss = dc.ss;
+  p.dbase = dc.dbase; p.sfa = dc.sfa; p.sfs = dc.sfs; p.ss = dc.ss; p.sss = dc.sss;
   p.n_out = g.n_out; p.ntiles = g.ntiles; p.ngroups = g.ngroups; p.ternary = g.bits == 2;
   p.early = early;
   p.atomic_y = y_zeroed && dc.S > 1;

@@ -56,8 +56,9 @@ struct DecodeConfig {
   int npipe;              // MMA pipelines (issuing warps, each with its accumulators)
   int ns;                 // TMEM A slots (4 or 8)
   int dbase;              // TMEM column of the first accumulator
-  int sfa, sfs, ss;       // TMEM columns of the A scales, of TMEM slot 0's B
-                          // scales, and between two blocks' B scales
+  int sfa, sfs, ss, sss;  // TMEM columns of the A scales, of TMEM slot 0's B
+                          // scales, between two blocks' B scales, and between
+                          // two slots' B scales
   size_t smem;            // dynamic shared memory of the decode kernel
 };
 

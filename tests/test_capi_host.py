@@ -122,7 +122,8 @@ def test_decode_launch_shapes_fit(sdq, sms):
     B operand would not fit otherwise), k chunks covering K with none empty,
     a ring of 4..32 stages in multiples of 4 (one expander set per ring
     slot), 1, 2 or 4 MMA pipelines, TMEM columns within 512 (4 or 8 slots of
-    16 sb code columns and sb 4-aligned sets of B-scale columns, 4 A-scale
+    16 sb code columns and their B-scale columns: sb 4-aligned sets, with
+    4-column sets rounded up to one 4, 8 or 16-column store, 4 A-scale
     columns, npipe x nbuf accumulators), the B
     image, its scale words and the ring within the shared-memory limit, and
     the e2m1 term count of the batch size."""
@@ -140,7 +141,8 @@ def test_decode_launch_shapes_fit(sdq, sms):
             assert s["npipe"] in (1, 2, 4) and s["nbuf"] in (1, 2) and s["ns"] in (4, 8)
             assert s["ss"] == 4 * (-(-(-(-s["NP"] // 32)) // 4))
             assert 1 <= s["sb"] <= 4
-            assert s["ns"] * s["sb"] * (16 + s["ss"]) + 4 + s["npipe"] * s["nbuf"] * s["NP"] <= 512
+            sss = ({1: 4, 2: 8}.get(s["sb"], 16) if s["ss"] == 4 else s["sb"] * s["ss"])
+            assert s["ns"] * (16 * s["sb"] + sss) + 4 + s["npipe"] * s["nbuf"] * s["NP"] <= 512
             assert s["slot_bytes"] == s["sb"] * blk
             assert s["b_bytes"] == (s["CB"] // 2 + 1) * s["NP"] * 128
             sfb = -(-(s["CB"] * s["NP"] * 4) // 16) * 16   # the chunk's B scale words
