@@ -191,23 +191,34 @@ int sdq_prep_activations(sdq_plan plan, const uint16_t* x, int32_t M,
  * (tcgen05 block-scaled 4-bit MMAs, kind::mxf4: the codes expanded into
  * tensor memory as e2m1 +-2 / 0, the activations as T e2m1 terms per batch
  * row with one power-of-two scale per 32 codes and term, x_tilde =
- * sum_t 2^(e_g - 3t) q_t, T = 6 for M <= 4, 4 up to 16, 3 above; each
- * thread block forms the terms of its k chunk; split-K over thread blocks
- * with a deterministic last-block reduction; the launch shape is chosen per
- * batch size at plan creation and can be queried with
+ * sum_t 2^(e_g - 3t) q_t, T = 6 for M <= 4, 4 up to 16, 3 above; the prepare
+ * kernel writes these terms for all of K when n_b is a multiple of 64, else
+ * each thread block forms those of its k chunk from x_tilde; split-K over
+ * thread blocks with a deterministic last-block reduction: results are
+ * bit-for-bit reproducible for a given plan, M and device; the launch shape
+ * is chosen per batch size at plan creation and can be queried with
  * sdq_decode_launch_shape).  M > 64: tcgen05 bf16 prefill kernel.  Errors as
  * sdq_prep_activations, and UNSUPPORTED when no launch shape fits. */
 int sdq_contract(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha, int32_t M,
                  float* y, void* ws, size_t ws_bytes, void* stream);
 
+/* y += the contraction above (M <= 64 only; UNSUPPORTED above): every
+ * thread block adds its k chunk's share into y with float reductions, so y
+ * must hold valid values (e.g. a residual stream the layer's output is added
+ * to, or zeros).  The order of the additions is not fixed: results may
+ * differ from run to run in the last bits.  Same inputs and errors as
+ * sdq_contract otherwise. */
+int sdq_contract_add(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha, int32_t M,
+                     float* y, void* ws, size_t ws_bytes, void* stream);
+
 /* y = the layer applied to x: same inputs, outputs and errors as
- * sdq_prep_activations followed by sdq_contract.  For small decode batches
- * (sdq_forward_kernels() == 1) it is ONE kernel: the decode kernel computes
- * the part of x_tilde its k chunk needs itself and writes no x_tilde to `ws`
- * (sdq_read_prep then returns stale data).  Otherwise it runs the two
- * kernels.  Results of the two routes agree to within the rounding of
- * x_tilde (bf16 hi + lo tables, fp32 sums) and of its e2m1 terms, not bit for
- * bit. */
+ * sdq_prep_activations followed by sdq_contract, as two kernels.  For decode
+ * batches (M <= 64) whose launch shape splits K over thread blocks, the
+ * prepare kernel also clears y and the contraction adds its k chunks' shares
+ * into it with float reductions (as sdq_contract_add): results agree with
+ * sdq_contract to within the order of those additions, not bit for bit.
+ * The contraction may start streaming the codes before the prepare kernel
+ * completes (it reads nothing the prepare kernel writes until then). */
 int sdq_linear_forward(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha,
                        const uint16_t* x, int32_t M, float* y, void* ws, size_t ws_bytes,
                        void* stream);

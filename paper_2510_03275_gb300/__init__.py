@@ -22,7 +22,7 @@ __all__ = [
     "SdqError", "LayerDesc", "lib", "library_path",
     "sdq_plan_create", "sdq_plan_destroy", "sdq_k_eff", "sdq_plain_bytes", "sdq_tiled_bytes",
     "sdq_workspace_bytes", "sdq_build_tables", "sdq_decode_launch_shape", "sdq_encode_rows", "sdq_pack", "sdq_unpack",
-    "sdq_prep_activations", "sdq_contract", "sdq_linear_forward", "sdq_read_prep",
+    "sdq_prep_activations", "sdq_contract", "sdq_contract_add", "sdq_linear_forward", "sdq_read_prep",
     "sdq_workspace_status", "sdq_linear_forward_noalloc", "sdq_noalloc_scratch_bytes", "sdq_noalloc_status",
     "sdq_forward_kernels", "sdq_status_string", "Plan",
 ]
@@ -87,6 +87,7 @@ _SIGS = {
     "sdq_unpack": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp]),
     "sdq_prep_activations": (ctypes.c_int, [_vp, _vp, _i32, _vp, _sz, _vp]),
     "sdq_contract": (ctypes.c_int, [_vp, _vp, _vp, _i32, _vp, _vp, _sz, _vp]),
+    "sdq_contract_add": (ctypes.c_int, [_vp, _vp, _vp, _i32, _vp, _vp, _sz, _vp]),
     "sdq_linear_forward": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _vp, _vp, _sz, _vp]),
     "sdq_read_prep": (ctypes.c_int, [_vp, _i32, _vp, _vp, _vp]),
     "sdq_workspace_status": (ctypes.c_int, [_vp, _i32, _vp, _vp]),
@@ -212,6 +213,12 @@ def sdq_prep_activations(plan, x, M, ws, stream=None):
 def sdq_contract(plan, codes_tiled, alpha, M, y, ws, stream=None):
     _check(lib().sdq_contract(plan, _ptr(codes_tiled), _ptr(alpha), M, _ptr(y), _ptr(ws),
                               ws.numel() * ws.element_size(), _stream(stream)), "sdq_contract")
+
+
+def sdq_contract_add(plan, codes_tiled, alpha, M, y, ws, stream=None):
+    """y += the contraction (M <= 64; float reductions, order not fixed)."""
+    _check(lib().sdq_contract_add(plan, _ptr(codes_tiled), _ptr(alpha), M, _ptr(y), _ptr(ws),
+                                  ws.numel() * ws.element_size(), _stream(stream)), "sdq_contract_add")
 
 
 def sdq_linear_forward(plan, codes_tiled, alpha, x, M, y, ws, stream=None):

@@ -194,12 +194,12 @@ extern "C" int sdq_prep_activations(sdq_plan p, const uint16_t* x, int32_t M, vo
 }
 
 static int contract(sdq_plan p, const uint32_t* codes_tiled, const float* alpha, int32_t M, float* y,
-                    void* ws, size_t ws_bytes, void* stream, int early, int y_zeroed) {
+                    void* ws, size_t ws_bytes, void* stream, int early, int y_mode) {
   int st = check_ws(p, M, ws, ws_bytes);
   if (st != SDQ_OK) return st;
   if (!codes_tiled || !alpha || !y || !aligned16(codes_tiled) || !aligned16(y)) return SDQ_ERR_INVALID_ARG;
   cudaError_t e = M <= kMaxDecodeM
-                      ? launch_decode(p, codes_tiled, alpha, M, y, ws, (cudaStream_t)stream, early, y_zeroed)
+                      ? launch_decode(p, codes_tiled, alpha, M, y, ws, (cudaStream_t)stream, early, y_mode)
                       : launch_prefill(p, codes_tiled, alpha, M, y, ws, (cudaStream_t)stream);
   if (e == cudaErrorNotSupported) return SDQ_ERR_UNSUPPORTED;
   return cuda_status(e);
@@ -207,14 +207,19 @@ static int contract(sdq_plan p, const uint32_t* codes_tiled, const float* alpha,
 
 extern "C" int sdq_contract(sdq_plan p, const uint32_t* codes_tiled, const float* alpha, int32_t M,
                             float* y, void* ws, size_t ws_bytes, void* stream) {
-  return contract(p, codes_tiled, alpha, M, y, ws, ws_bytes, stream, 0, 0);
+  return contract(p, codes_tiled, alpha, M, y, ws, ws_bytes, stream, 0, kYStore);
 }
 
-// Small decode batches: one kernel that builds its own B operand from x.
-// Otherwise the prepare kernel, then the contraction; behind its own prepare
-// kernel the decode kernel may start reading the codes before the preceding
-// grid finishes: that grid waited for everything before it in the stream, and
-// it does not write the codes.
+extern "C" int sdq_contract_add(sdq_plan p, const uint32_t* codes_tiled, const float* alpha, int32_t M,
+                                float* y, void* ws, size_t ws_bytes, void* stream) {
+  if (M > kMaxDecodeM) return p && M >= 1 ? SDQ_ERR_UNSUPPORTED : SDQ_ERR_INVALID_ARG;
+  return contract(p, codes_tiled, alpha, M, y, ws, ws_bytes, stream, 0, kYAdd);
+}
+
+// The prepare kernel, then the contraction; behind its own prepare kernel the
+// decode kernel may start reading the codes before the preceding grid
+// finishes: that grid waited for everything before it in the stream, and it
+// does not write the codes.
 extern "C" int sdq_linear_forward(sdq_plan p, const uint32_t* codes_tiled, const float* alpha,
                                   const uint16_t* x, int32_t M, float* y, void* ws, size_t ws_bytes,
                                   void* stream) {
@@ -226,7 +231,7 @@ extern "C" int sdq_linear_forward(sdq_plan p, const uint32_t* codes_tiled, const
   if (!x || !aligned16(x) || !y || !aligned16(y)) return SDQ_ERR_INVALID_ARG;
   st = cuda_status(launch_prep(p, x, M, ws, (cudaStream_t)stream, zero_y ? y : nullptr));
   if (st != SDQ_OK) return st;
-  return contract(p, codes_tiled, alpha, M, y, ws, ws_bytes, stream, 1, zero_y ? 1 : 0);
+  return contract(p, codes_tiled, alpha, M, y, ws, ws_bytes, stream, 1, zero_y ? kYZeroed : kYStore);
 }
 
 extern "C" int sdq_forward_kernels(sdq_plan p, int32_t M, const uint16_t* x) {

@@ -45,11 +45,14 @@ cudaError_t launch_prep(const sdq_plan_s* p, const uint16_t* x, int M, void* ws,
                         float* y_zero = nullptr);
 // early = 1: the decode kernel starts streaming codes before waiting for the
 // preceding grid (valid only behind this library's own prep kernels).
-// y_zeroed = 1: y holds zeros (the prepare kernel of the same call cleared
-// it), so that split-K partial sums may be added into it by float atomics
-// (order of the additions not fixed); else the deterministic ticket route.
+// y_mode: kYStore: y = the result (split-K by the deterministic ticket
+// route); kYZeroed: y holds zeros (the prepare kernel of the same call
+// cleared it), so that split-K partial sums are added into it by float
+// reductions (order of the additions not fixed); kYAdd: y += the result, by
+// float reductions whatever the split.
+constexpr int kYStore = 0, kYZeroed = 1, kYAdd = 2;
 cudaError_t launch_decode(const sdq_plan_s* p, const uint32_t* codes, const float* alpha, int M,
-                          float* y, void* ws, cudaStream_t st, int early, int y_zeroed);
+                          float* y, void* ws, cudaStream_t st, int early, int y_mode);
 // Whether the decode prepare kernel writes the B operand image (n_b a
 // multiple of 64), so that each decode CTA copies its chunk's part.
 bool decode_image(const sdq_plan_s* p);

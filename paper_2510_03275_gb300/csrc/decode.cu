@@ -120,7 +120,7 @@ struct DecodeParams {
   int64_t k_eff, kpad;
   int M, T, NP, S, P, CB, KB, ring, sb, nbuf, npipe, ns, ns_log2, dbase, sfa, sfs, ss, sss;
   int n_out, ntiles, ngroups, ternary, early;
-  int atomic_y;          // split-K by float atomic adds into y (zeroed by the prepare kernel)
+  int atomic_y;          // add into y with float reductions (y zeroed by the prepare kernel, or y += result)
   uint32_t blk_bytes, slot_bytes, b_bytes, sfb_bytes;
 };
 
@@ -612,10 +612,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
           if (c0 + i < MT) {
             acc += sum[i];
             if (++t == p.T) {   // the terms of batch row m, already scaled by their B scales
-              if (p.S == 1) {
-                if (live) p.y[(size_t)m * p.n_out + row] = sa * acc;
-              } else if (p.atomic_y) {
+              if (p.atomic_y) {
                 if (live) red_add_f32(p.y + (size_t)m * p.n_out + row, sa * acc);
+              } else if (p.S == 1) {
+                if (live) p.y[(size_t)m * p.n_out + row] = sa * acc;
               } else {
                 p.part[((size_t)sidx * p.M + m) * NR + row] = acc;
               }
@@ -820,7 +820,7 @@ bool decode_image(const sdq_plan_s* pl) { return pl->geo.n_b % 64 == 0; }
 
 
 cudaError_t launch_decode(const sdq_plan_s* pl, const uint32_t* codes, const float* alpha, int M,
-                          float* y, void* ws, cudaStream_t st, int early, int y_zeroed) {
+                          float* y, void* ws, cudaStream_t st, int early, int y_mode) {
   const Geometry& g = pl->geo;
   const DecodeConfig& dc = decode_config(pl, M);
   if (dc.S < 1) return cudaErrorNotSupported;   // no launch shape fits
@@ -843,7 +843,7 @@ cudaError_t launch_decode(const sdq_plan_s* pl, const uint32_t* codes, const flo
   p.dbase = dc.dbase; p.sfa = dc.sfa; p.sfs = dc.sfs; p.ss = dc.ss; p.sss = dc.sss;
   p.n_out = g.n_out; p.ntiles = g.ntiles; p.ngroups = g.ngroups; p.ternary = g.bits == 2;
   p.early = early;
-  p.atomic_y = y_zeroed && dc.S > 1;
+  p.atomic_y = y_mode == kYAdd || (y_mode == kYZeroed && dc.S > 1);
   p.blk_bytes = (uint32_t)(kTileRows * kBlk * g.bits / 8);
   p.slot_bytes = p.sb * p.blk_bytes;
   p.b_bytes = (uint32_t)((dc.CB / 2 + 1) * dc.NP * 128);

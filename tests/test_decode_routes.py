@@ -179,3 +179,41 @@ def test_llama70b_decode_kernels(sdq, torch_cuda, name):
     x = torch.zeros((16, lin.k_in), dtype=torch.bfloat16, device="cuda")
     for m in (1, 8, 16):
         assert sdq.sdq_forward_kernels(plan.handle, m, x) == 2
+
+
+@pytest.mark.parametrize("m", [1, 4, 16, 64])
+@pytest.mark.parametrize("shape", [(300, 2048, 128, 2), (129, 272, 16, Fraction(5, 2)), (1000, 4096, 128, 2)])
+def test_contract_add_accumulates(sdq, torch_cuda, m, shape):
+    """sdq_contract_add adds the layer's output into y (a residual stream):
+    y0 + W_hat x within the bound, twice in a row gives y0 + 2 W_hat x, and
+    batches above the decode range are refused."""
+    torch = torch_cuda
+    n, k, b, osr = shape
+    plan, d, signs, codes, alpha, tiled = _layer(sdq, torch, n, k, b, osr, O.TERNARY, seed=n + 3 * m)
+    bits, x = _x(torch, m, k, seed=7 * m + 3)
+    al = torch.from_numpy(alpha).cuda()
+    ws = plan.alloc_workspace(m)
+    sdq.sdq_prep_activations(plan.handle, x, m, ws)
+    y0 = np.random.default_rng(m + n).standard_normal((m, n)).astype(np.float32)
+    y = torch.from_numpy(y0).cuda()
+    sdq.sdq_contract_add(plan.handle, tiled, al, m, y, ws)
+    assert sdq.sdq_workspace_status(plan.handle, m, ws) == 0
+    xf = W.bf16_to_float(bits)
+    yr = O.forward_code_domain(xf, codes, alpha, b, d.n_b, signs)
+    bound = EB.forward_bound(xf, codes, alpha, b, d.n_b, signs, T=_terms(sdq, d, m))
+    # the float adds into y0 round at |y0| (ulp 2^-23 of its magnitude)
+    slack = 2.0 ** -22 * (np.abs(y0) + np.abs(yr))
+    assert np.all(np.abs(y.cpu().numpy() - y0 - yr) <= bound + slack)
+    sdq.sdq_contract_add(plan.handle, tiled, al, m, y, ws)
+    assert np.all(np.abs(y.cpu().numpy() - y0 - 2 * yr) <= 2 * bound + 2 * slack)
+
+
+def test_contract_add_refuses_prefill_batches(sdq, torch_cuda):
+    torch = torch_cuda
+    plan, d, signs, codes, alpha, tiled = _layer(sdq, torch, 256, 512, 128, 2, O.TERNARY, seed=1)
+    m = 128
+    ws = plan.alloc_workspace(m)
+    y = torch.zeros((m, 256), dtype=torch.float32, device="cuda")
+    with pytest.raises(sdq.SdqError) as e:
+        sdq.sdq_contract_add(plan.handle, tiled, torch.from_numpy(alpha).cuda(), m, y, ws)
+    assert e.value.status == -2   # SDQ_ERR_UNSUPPORTED
