@@ -74,6 +74,7 @@
 // MMAs before freeing TMEM.
 #include <algorithm>
 #include <cmath>
+#include <type_traits>
 
 #include "common.cuh"
 
@@ -582,10 +583,29 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       cp_async_wait_group<kAlphaAhead - 1>();   // tile u's group has landed
       const float sa = live ? 0.5f * s_alpha[u % kAlphaAhead][et] : 0.f;
       alpha_fetch(u + kAlphaAhead);
-      int m = 0, t = 0;
-      float acc = 0.f;
-      for (int c0 = 0; c0 < MT; c0 += 16) {
-        float sum[16];
+      // y (or the partial) of batch row m from the sum of its T terms
+      // where and how this tile's results are written (one address rule and
+      // one kind of write per tile)
+      const bool partial = p.S > 1 && !p.atomic_y;
+      float* eb = partial ? p.part + (size_t)sidx * p.M * NR + row : p.y + row;
+      uint32_t est = partial ? (uint32_t)NR : (uint32_t)p.n_out;
+      float esc = partial ? 1.f : sa;
+      int emode = !(partial || live) ? 0 : (p.atomic_y ? 1 : 2);   // none, float add, store
+      int Mv = p.M;
+      // (computed here, once: without this the compiler re-derives them from
+      // the kernel parameters inside the loops below)
+      asm volatile("" : "+l"(eb), "+r"(est), "+f"(esc), "+r"(emode), "+r"(Mv));
+      auto emit = [&](int m, float acc) {
+        if (m < Mv) {
+          float* a = eb + (size_t)m * est;
+          if (emode == 1) red_add_f32(a, esc * acc);
+          else if (emode == 2) *a = esc * acc;
+        }
+      };
+      // columns c0 .. c0 + 15 of the pipelines' accumulators, added (whole
+      // x16 loads stay inside the NP columns, a multiple of 16); the
+      // accumulators go back to the MMAs after the tile's last load
+      auto load16 = [&](int c0, float (&sum)[16]) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) sum[i] = 0.f;
 #pragma unroll
@@ -604,25 +624,54 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
           for (int e = 0; e < kMaxPipes; ++e)
             if ((in >> e) & 1u) mbar_arrive(&acc_empty[e][kc[e] % p.nbuf]);
         }
-        // (not unrolled: this code runs once per tile, and unrolled it is
-        // cold instruction memory every time, each miss an L2 round trip
-        // while the code stream loads it)
+      };
+      if (MT <= 16) {
+        // one or two batch rows: a short loop (not unrolled: it runs once per
+        // long tile, and unrolled code is cold instruction memory every time,
+        // each miss an L2 round trip while the code stream loads it)
+        float sum[16];
+        load16(0, sum);
+        int m = 0, t = 0;
+        float acc = 0.f;
 #pragma unroll 1
-        for (int i = 0; i < 16; ++i) {
-          if (c0 + i < MT) {
-            acc += sum[i];
-            if (++t == p.T) {   // the terms of batch row m, already scaled by their B scales
-              if (p.atomic_y) {
-                if (live) red_add_f32(p.y + (size_t)m * p.n_out + row, sa * acc);
-              } else if (p.S == 1) {
-                if (live) p.y[(size_t)m * p.n_out + row] = sa * acc;
-              } else {
-                p.part[((size_t)sidx * p.M + m) * NR + row] = acc;
+        for (int i = 0; i < MT; ++i) {
+          acc += sum[i];
+          if (++t == p.T) { emit(m, acc); acc = 0.f; t = 0; ++m; }
+        }
+      } else {
+        // many batch rows: 16 kSub columns hold whole rows, so where each
+        // row's terms end is known at compile time and the sums stay in
+        // registers (a loop over a register array indexed at run time puts
+        // it in local memory: about 200 cycles a column)
+        auto terms = [&](auto tc) {
+          constexpr int T = decltype(tc)::value;
+          constexpr int kSub = T == 4 ? 1 : 3;
+          int m = 0;
+          float acc = 0.f;
+#pragma unroll 1
+          for (int c0 = 0; c0 < MT; c0 += 16 * kSub) {
+#pragma unroll
+            for (int sub = 0; sub < kSub; ++sub) {
+              const int cs = c0 + 16 * sub;
+              if (cs < MT) {
+                float sum[16];
+                load16(cs, sum);
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                  acc += sum[i];
+                  if ((16 * sub + i) % T == T - 1) {
+                    emit(m, acc);
+                    acc = 0.f;
+                    ++m;
+                  }
+                }
               }
-              acc = 0.f; t = 0; ++m;
             }
           }
-        }
+        };
+        if (p.T == 3) terms(std::integral_constant<int, 3>());
+        else if (p.T == 4) terms(std::integral_constant<int, 4>());
+        else terms(std::integral_constant<int, 6>());
       }
 #pragma unroll
       for (int e = 0; e < kMaxPipes; ++e) kc[e] += (in >> e) & 1u;
@@ -725,6 +774,11 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
   const double c_xblk = 200.0, c_xstage = 600.0;                 // expander set, cycles
   double best_t = 1e30;
   const int pipes[3] = {4, 2, 1};
+  const int MT = M * best.T;
+  double t_epi[3];
+  for (int pi = 0; pi < 3; ++pi)
+    t_epi[pi] = MT <= 16 ? 0.0   // (one or two batch rows: within the fitted per-tile cost below)
+                         : ((MT + 15) / 16) * (385.0 * pipes[pi] + 650.0) / clk;
   for (int pi = 0; pi < 3; ++pi) {
     const int np = pipes[pi];
     for (int ns = 4; ns <= kASlots; ns *= 2)
@@ -777,7 +831,12 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
             const double tile_bytes = (double)CB * blk_bytes;
             const double rate = std::min({cta_bw, hbm / std::min(grid, sms), mma_rate * slot_bytes,
                                           (double)ring * slot_bytes / ring_latency});
-            const double t_cta = units * (tile_bytes / rate + 0.8e-6 + 0.15e-6 * S);
+            // the tile's epilogue (accumulator loads per pipeline and the
+            // terms' sums and writes per 16 columns, measured per tile) runs
+            // beside the next tile's MMAs with two accumulators, else between
+            const double t_stream = tile_bytes / rate;
+            const double t_tile = nbuf == 2 ? std::max(t_stream, t_epi[pi]) : t_stream + t_epi[pi];
+            const double t_cta = units * (t_tile + 0.8e-6 + 0.15e-6 * S);
             const double t = waves * t_cta + t_build + t_tail;
             if (t < best_t * 0.999) {
               best_t = t;
