@@ -206,18 +206,10 @@ __device__ __noinline__ void write_terms(const DecodeParams& p, uint8_t* bop, ui
   }
 }
 
-// n 16-byte words global -> shared by the kBuildThreads builder threads,
-// four loads in flight per thread.
+// n 16-byte words global -> shared by the kBuildThreads builder threads as
+// cp.async copies, all in flight at once (completion: cp_async_wait_all).
 __device__ __forceinline__ void copy_lsu(uint4* dst, const uint4* src, int n, int et) {
-  for (int t0 = et; t0 < n; t0 += 4 * kBuildThreads) {
-    uint4 v[4];
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-      if (t0 + k * kBuildThreads < n) v[k] = __ldcg(src + t0 + k * kBuildThreads);
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-      if (t0 + k * kBuildThreads < n) dst[t0 + k * kBuildThreads] = v[k];
-  }
+  for (int t = et; t < n; t += kBuildThreads) cp_async16(dst + t, src + t, 16);
 }
 
 // kTernary: 2-bit ternary codes, else 1-bit binary (one instantiation each,
@@ -394,14 +386,16 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
     pdl_wait();
     if (p.bsrc == 2) {
       // The prepared image rows of the chunk's blocks and their scale words,
-      // with plain 16-byte loads (L2 hits: the prepare kernel just wrote
-      // them).  A bulk copy here would queue behind the code stream the
-      // producers have started on the same SM, microseconds of HBM traffic.
+      // with 16-byte cp.async copies, all in flight at once (L2 hits: the
+      // prepare kernel just wrote them).  A bulk copy here would queue behind
+      // the code stream the producers have started on the same SM,
+      // microseconds of HBM traffic.
       const int a0 = kb0 >> 1, a1 = (kb0 + ncb - 1) >> 1;
       copy_lsu(reinterpret_cast<uint4*>(bop), reinterpret_cast<const uint4*>(p.bimg + (size_t)a0 * p.NP * 128),
                (a1 - a0 + 1) * p.NP * 8, et);
       copy_lsu(reinterpret_cast<uint4*>(sfbs), reinterpret_cast<const uint4*>(p.sfbw + (size_t)kb0 * p.NP * 4),
                ncb * p.NP / 4, et);
+      cp_async_wait_all();
     } else {
       write_terms(p, bop, sfbs, kb0, ncb, et);
     }
@@ -625,10 +619,32 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
             if ((in >> e) & 1u) mbar_arrive(&acc_empty[e][kc[e] % p.nbuf]);
         }
       };
-      if (MT <= 16) {
-        // one or two batch rows: a short loop (not unrolled: it runs once per
-        // long tile, and unrolled code is cold instruction memory every time,
-        // each miss an L2 round trip while the code stream loads it)
+      if (MT <= 8) {
+        // one batch row: 8 columns of two pipelines' accumulators in flight
+        // per wait (the last tile's epilogue is the call's tail)
+        float acc = 0.f;
+#pragma unroll
+        for (int e0 = 0; e0 < kMaxPipes; e0 += 2) {
+          const bool h0 = (in >> e0) & 1u, h1 = (in >> (e0 + 1)) & 1u;
+          uint32_t r0[8], r1[8];
+          if (h0) tmem_ld8(lq + (uint32_t)(p.dbase + (e0 * p.nbuf + kc[e0] % p.nbuf) * p.NP), r0);
+          if (h1) tmem_ld8(lq + (uint32_t)(p.dbase + ((e0 + 1) * p.nbuf + kc[e0 + 1] % p.nbuf) * p.NP), r1);
+          if (h0 || h1) tmem_ld_wait();
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            if (h0 && i < MT) acc += __uint_as_float(r0[i]);
+            if (h1 && i < MT) acc += __uint_as_float(r1[i]);
+          }
+        }
+        tc_fence_before();
+#pragma unroll
+        for (int e = 0; e < kMaxPipes; ++e)
+          if ((in >> e) & 1u) mbar_arrive(&acc_empty[e][kc[e] % p.nbuf]);
+        emit(0, acc);
+      } else if (MT <= 16) {
+        // two batch rows: a short loop (not unrolled: it runs once per long
+        // tile, and unrolled code is cold instruction memory every time, each
+        // miss an L2 round trip while the code stream loads it)
         float sum[16];
         load16(0, sum);
         int m = 0, t = 0;
