@@ -43,6 +43,10 @@ cudaError_t launch_unpack(const sdq_plan_s* p, const uint32_t* tiled, uint32_t* 
 // y_zero (M x n_out, may be null): cleared by the decode prepare kernel.
 cudaError_t launch_prep(const sdq_plan_s* p, const uint16_t* x, int M, void* ws, cudaStream_t st,
                         float* y_zero = nullptr);
+// Prefill prepare (M > 64) on the tensor cores where the layer allows it;
+// *used = false (nothing launched) otherwise.
+cudaError_t launch_prep_tc(const sdq_plan_s* p, const uint16_t* x, int M, void* ws, cudaStream_t st,
+                           bool* used);
 // early = 1: the decode kernel starts streaming codes before waiting for the
 // preceding grid (valid only behind this library's own prep kernels).
 // y_mode: kYStore: y = the result (split-K by the deterministic ticket
@@ -81,6 +85,13 @@ __device__ __forceinline__ uint16_t float_to_bf16_bits(float f) {
   uint32_t u = __float_as_uint(f);
   u += 0x7FFFu + ((u >> 16) & 1u);
   return (uint16_t)(u >> 16);
+}
+
+// Two fp32 -> bf16 (round to nearest even), lo in bits 0-15, hi in 16-31.
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;\n" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
 }
 
 // 16x8x16 warp MMA, bf16 x bf16 -> fp32.

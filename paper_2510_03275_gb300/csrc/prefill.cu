@@ -27,6 +27,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <mutex>
 
 #include "common.cuh"
@@ -230,6 +231,190 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
+// ------------------------------------------ prefill prepare, tensor cores
+// x_tilde = G x_b for every block b (section 3.5), as one GEMM: x viewed as
+// R = M nblk rows of B = 128 inputs (row r = block r mod nblk of batch row
+// r / nblk), x_tilde rows = x rows . G^T (128 x n_b), on tcgen05.mma
+// kind::f16 (M = 128 rows, N = n_b, K = 16 per instruction) with G split
+// into bf16 hi and lo parts accumulated into the same fp32 accumulator (the
+// pair carries G to ~2^-16; x is bf16, exact).  Persistent CTAs, one per SM,
+// over tiles of 128 rows:
+//   warp 0     TMEM allocation (two accumulators of n_b columns); lane 0
+//              loads G hi / lo once, then the x tiles into a 2-slot ring
+//              (TMA, 128-byte swizzle: the canonical K-major operand layout)
+//   warp 1     lane 0 issues each tile's 16 MMAs into accumulator t mod 2
+//   warps 2-9  epilogue, two warps per TMEM lane quadrant (half of the n_b
+//              columns each): bf16 x_tilde (round to nearest even) in the
+//              prefill operand order (prefill_pos64) with 16-byte stores;
+//              the K padding of every batch row set to zero
+// Bounded waits as in the contraction kernels.
+constexpr int kPtEpiWarps = 8;
+constexpr int kPtThreads = 64 + 32 * kPtEpiWarps;
+constexpr int kPtRows = 128;
+constexpr int kPtXTile = kPtRows * 128 * 2;   // 32 KB: 128 rows x 128 bf16 (two 64-wide K chunks)
+
+struct PrepTcParams {
+  uint16_t* xtb;
+  uint64_t* rec;
+  uint64_t call;
+  int64_t R, k_eff, kpad;
+  int M, nblk, n_b, ntile, ternary;
+};
+
+__global__ void __launch_bounds__(kPtThreads, 1)
+    prep_tc_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap ghmap,
+                   const __grid_constant__ CUtensorMap glmap, PrepTcParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t g_full, x_full[2], x_empty[2], acc_full[2], acc_empty[2];
+  __shared__ uint32_t tmem_base;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
+  uint8_t* base = smem_raw + (sbase - smem_u32(smem_raw));
+  const uint32_t gchunk = (uint32_t)p.n_b * 128u;   // one 64-wide K chunk of G^T: n_b rows x 128 B
+  uint8_t* gh = base;                               // 2 chunks
+  uint8_t* gl = base + 2 * gchunk;                  // 2 chunks
+  uint8_t* xs = base + 4 * gchunk;                  // 2 ring slots
+  const uint32_t tcols = p.n_b <= 64 ? 128u : (p.n_b <= 128 ? 256u : 512u);
+
+  if (tid == 0) {
+    mbar_init(&g_full, 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&x_full[s], 1);
+      mbar_init(&x_empty[s], 1);
+      mbar_init(&acc_full[s], 1);
+      mbar_init(&acc_empty[s], kPtEpiWarps);
+    }
+    fence_mbar_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(&tmem_base, tcols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base;
+  bool ok = true;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // G (the plan's table, never written by the stream) before the wait
+      // for the preceding grid; x and the workspace after it
+      mbar_expect_tx(&g_full, 4 * gchunk);
+      for (int c = 0; c < 2; ++c) {
+        tma_load_2d(gh + c * gchunk, &ghmap, 64 * c, 0, &g_full);
+        tma_load_2d(gl + c * gchunk, &glmap, 64 * c, 0, &g_full);
+      }
+      pdl_wait();
+      pdl_launch_dependents();
+      int i = 0;
+      for (int t = blockIdx.x; t < p.ntile && ok; t += gridDim.x, ++i) {
+        const int s = i & 1, r = i >> 1;
+        if (r > 0) ok = mbar_wait(&x_empty[s], (r - 1) & 1);
+        if (!ok) break;
+        mbar_expect_tx(&x_full[s], kPtXTile);
+        tma_load_2d(xs + s * kPtXTile, &xmap, 0, t * kPtRows, &x_full[s]);
+        tma_load_2d(xs + s * kPtXTile + kPtXTile / 2, &xmap, 64, t * kPtRows, &x_full[s]);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(p.n_b >> 3) << 17) |
+                             ((uint32_t)(kPtRows >> 4) << 24);
+      ok = mbar_wait(&g_full, 0);
+      int i = 0;
+      for (int t = blockIdx.x; t < p.ntile && ok; t += gridDim.x, ++i) {
+        const int s = i & 1, r = i >> 1;
+        ok = mbar_wait(&x_full[s], r & 1);
+        if (ok && r > 0) ok = mbar_wait(&acc_empty[s], (r - 1) & 1);
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t d = tmem + (uint32_t)(s * p.n_b);
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          const uint64_t ad = sw128_desc(sbase + 4 * gchunk + s * kPtXTile + c * (kPtXTile / 2));
+          const uint64_t bh = sw128_desc(sbase + c * gchunk);
+          const uint64_t bl = sw128_desc(sbase + (2 + c) * gchunk);
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {
+            umma_bf16(d, ad + 2 * kk, bh + 2 * kk, idesc, (c | kk) != 0);
+            umma_bf16(d, ad + 2 * kk, bl + 2 * kk, idesc, 1);
+          }
+        }
+        umma_commit(&x_empty[s]);
+        umma_commit(&acc_full[s]);
+      }
+    }
+  } else {
+    pdl_wait();   // the workspace belongs to the preceding grid until then
+    const int et = tid - 64, q = warp & 3, half = (warp - 2) >> 2;
+    // the K padding of every batch row (k_eff .. kpad, a multiple of 8)
+    for (int64_t z = (int64_t)blockIdx.x * (32 * kPtEpiWarps) + et; z < (int64_t)p.M * ((p.kpad - p.k_eff) / 8);
+         z += (int64_t)gridDim.x * (32 * kPtEpiWarps)) {
+      const int64_t per = (p.kpad - p.k_eff) / 8, m = z / per;
+      *reinterpret_cast<uint4*>(p.xtb + m * p.kpad + p.k_eff + 8 * (z - m * per)) = make_uint4(0, 0, 0, 0);
+    }
+    const int cw = p.n_b / 2;                                   // this warp's columns
+    const uint32_t lq = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(half * cw);
+    int i = 0;
+    for (int t = blockIdx.x; t < p.ntile && ok; t += gridDim.x, ++i) {
+      const int s = i & 1, r = i >> 1;
+      ok = mbar_wait(&acc_full[s], r & 1);
+      if (!ok) break;
+      tc_fence_after();
+      const int64_t row = (int64_t)t * kPtRows + 32 * q + lane;
+      const bool live = row < p.R;
+      const int64_t m = live ? row / p.nblk : 0;
+      uint16_t* out = p.xtb + m * p.kpad + (live ? (row - m * p.nblk) * p.n_b : 0) + half * cw;
+      const uint32_t acol = (uint32_t)(s * p.n_b);
+      // 32 columns at a time: a ternary operand permutes within 16, a binary
+      // one within 32 positions (prefill_pos64); physical pair (2k, 2k + 1)
+      // of a 16 (32) holds logical 7 - k and 15 - k (15 - k and 31 - k)
+      for (int c0 = 0; c0 < cw; c0 += 32) {
+        uint32_t a[16], b[16];
+        tmem_ld16(lq + acol + (uint32_t)c0, a);
+        tmem_ld16(lq + acol + (uint32_t)c0 + 16, b);
+        tmem_ld_wait();
+        if (c0 + 32 >= cw) {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&acc_empty[s]);
+        }
+        uint32_t w[16];
+        if (p.ternary) {
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            w[k] = pack_bf16x2(__uint_as_float(a[7 - k]), __uint_as_float(a[15 - k]));
+            w[8 + k] = pack_bf16x2(__uint_as_float(b[7 - k]), __uint_as_float(b[15 - k]));
+          }
+        } else {
+#pragma unroll
+          for (int k = 0; k < 16; ++k) {
+            const float lo = k < 16 ? __uint_as_float(a[15 - k]) : 0.f;
+            const float hi = __uint_as_float(b[15 - k]);
+            w[k] = pack_bf16x2(lo, hi);
+          }
+        }
+        if (live) {
+          uint4* o = reinterpret_cast<uint4*>(out + c0);
+          o[0] = make_uint4(w[0], w[1], w[2], w[3]);
+          o[1] = make_uint4(w[4], w[5], w[6], w[7]);
+          o[2] = make_uint4(w[8], w[9], w[10], w[11]);
+          o[3] = make_uint4(w[12], w[13], w[14], w[15]);
+        }
+      }
+    }
+  }
+  if (!ok) call_record_fail(p.rec, p.call);
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    __syncwarp();   // warp-collective: lane 0 ran the producer loop alone
+    tc_fence_after();
+    tmem_dealloc(tmem, tcols);
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_prefill(const sdq_plan_s* pl, const uint32_t* codes, const float* alpha, int M,
@@ -259,6 +444,58 @@ cudaError_t launch_prefill(const sdq_plan_s* pl, const uint32_t* codes, const fl
   if (e != cudaSuccess) return e;
   dim3 grid((g.n_out + kBN - 1) / kBN, (M + kBM - 1) / kBM);
   return launch_pdl(prefill_kernel, grid, dim3(kThreads), (size_t)kSmem, st, amap, p);
+}
+
+
+// The prefill prepare kernel on the tensor cores where it applies (B = 128,
+// n_b a multiple of 64 up to 256, x 16-byte aligned); *used = false otherwise.
+cudaError_t launch_prep_tc(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws, cudaStream_t st,
+                           bool* used) {
+  const Geometry& g = pl->geo;
+  *used = false;
+  if (g.block != 128 || g.n_b % 64 != 0 || g.n_b > 256 || (reinterpret_cast<uintptr_t>(x) & 15u)) return cudaSuccess;
+  auto enc = encode_fn();
+  if (!enc) return cudaSuccess;
+  const WsLayout L = workspace_layout(pl, M);
+  uint8_t* wbase = static_cast<uint8_t*>(ws);
+  const int64_t R = (int64_t)M * g.nblk;
+  if (R >= (int64_t(1) << 31) - kPtRows) return cudaSuccess;
+  CUtensorMap xmap, ghmap, glmap;
+  const cuuint32_t estr[2] = {1, 1};
+  {
+    const cuuint64_t dims[2] = {128, (cuuint64_t)R};
+    const cuuint64_t strides[1] = {256};
+    const cuuint32_t box[2] = {64, (cuuint32_t)kPtRows};
+    if (enc(&xmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t*>(x), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaSuccess;
+  }
+  {
+    const cuuint64_t dims[2] = {128, (cuuint64_t)g.n_b};
+    const cuuint64_t strides[1] = {256};
+    const cuuint32_t box[2] = {64, (cuuint32_t)g.n_b};
+    if (enc(&ghmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, pl->d_g_hi, dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS ||
+        enc(&glmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, pl->d_g_lo, dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaSuccess;
+  }
+  PrepTcParams p;   // (a timeout is recorded under this kernel's own call number)
+  p.xtb = reinterpret_cast<uint16_t*>(wbase + L.xt);
+  p.rec = reinterpret_cast<uint64_t*>(wbase + L.err);
+  p.call = call_tag(next_call_number());
+  p.R = R; p.k_eff = g.k_eff; p.kpad = g.k_eff_pad;
+  p.M = M; p.nblk = g.nblk; p.n_b = g.n_b; p.ternary = pl->desc.quantizer == SDQ_TERNARY;
+  p.ntile = (int)((R + kPtRows - 1) / kPtRows);
+  const size_t smem = 1024 + 4 * (size_t)g.n_b * 128 + 2 * (size_t)kPtXTile;
+  cudaError_t e = cudaFuncSetAttribute(prep_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  const int grid = std::min(p.ntile, std::max(1, pl->sm_count));
+  *used = true;
+  return launch_pdl(prep_tc_kernel, dim3(grid), dim3(kPtThreads), smem, st, xmap, ghmap, glmap, p);
 }
 
 }  // namespace sdq

@@ -351,6 +351,9 @@ cudaError_t launch_prep(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws
     dim3 grid((g.n_b + 63) / 64, (g.nblk + 15) / 16, M);
     return launch_pdl(prep_decode_kernel, grid, dim3(128), smem, st, p);
   }
+  bool used = false;
+  cudaError_t et = launch_prep_tc(pl, x, M, ws, st, &used);
+  if (et != cudaSuccess || used) return et;
   PrepParams p;
   p.x = x; p.g_hi = pl->d_g_hi; p.g_lo = pl->d_g_lo;
   p.xtb = reinterpret_cast<uint16_t*>(base + L.xt);
