@@ -240,7 +240,7 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 // pair carries G to ~2^-16; x is bf16, exact).  Persistent CTAs, one per SM,
 // over tiles of 128 rows:
 //   warp 0     TMEM allocation (two accumulators of n_b columns); lane 0
-//              loads G hi / lo once, then the x tiles into a 2-slot ring
+//              loads G hi / lo once, then the x tiles into a 3-slot ring
 //              (TMA, 128-byte swizzle: the canonical K-major operand layout)
 //   warp 1     lane 0 issues each tile's 16 MMAs into accumulator t mod 2
 //   warps 2-9  epilogue, two warps per TMEM lane quadrant (half of the n_b
@@ -252,6 +252,7 @@ constexpr int kPtEpiWarps = 8;
 constexpr int kPtThreads = 64 + 32 * kPtEpiWarps;
 constexpr int kPtRows = 128;
 constexpr int kPtXTile = kPtRows * 128 * 2;   // 32 KB: 128 rows x 128 bf16 (two 64-wide K chunks)
+constexpr int kPtSlots = 3;                   // x ring (with G hi / lo of n_b = 256: 225 KB)
 
 struct PrepTcParams {
   uint16_t* xtb;
@@ -265,7 +266,7 @@ __global__ void __launch_bounds__(kPtThreads, 1)
     prep_tc_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap ghmap,
                    const __grid_constant__ CUtensorMap glmap, PrepTcParams p) {
   extern __shared__ uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t g_full, x_full[2], x_empty[2], acc_full[2], acc_empty[2];
+  __shared__ __align__(8) uint64_t g_full, x_full[kPtSlots], x_empty[kPtSlots], acc_full[2], acc_empty[2];
   __shared__ uint32_t tmem_base;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
@@ -273,14 +274,16 @@ __global__ void __launch_bounds__(kPtThreads, 1)
   const uint32_t gchunk = (uint32_t)p.n_b * 128u;   // one 64-wide K chunk of G^T: n_b rows x 128 B
   uint8_t* gh = base;                               // 2 chunks
   uint8_t* gl = base + 2 * gchunk;                  // 2 chunks
-  uint8_t* xs = base + 4 * gchunk;                  // 2 ring slots
+  uint8_t* xs = base + 4 * gchunk;                  // kPtSlots ring slots
   const uint32_t tcols = p.n_b <= 64 ? 128u : (p.n_b <= 128 ? 256u : 512u);
 
   if (tid == 0) {
     mbar_init(&g_full, 1);
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < kPtSlots; ++s) {
       mbar_init(&x_full[s], 1);
       mbar_init(&x_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
       mbar_init(&acc_full[s], 1);
       mbar_init(&acc_empty[s], kPtEpiWarps);
     }
@@ -309,7 +312,7 @@ __global__ void __launch_bounds__(kPtThreads, 1)
       pdl_launch_dependents();
       int i = 0;
       for (int t = blockIdx.x; t < p.ntile && ok; t += gridDim.x, ++i) {
-        const int s = i & 1, r = i >> 1;
+        const int s = i % kPtSlots, r = i / kPtSlots;
         if (r > 0) ok = mbar_wait(&x_empty[s], (r - 1) & 1);
         if (!ok) break;
         mbar_expect_tx(&x_full[s], kPtXTile);
@@ -324,12 +327,12 @@ __global__ void __launch_bounds__(kPtThreads, 1)
       ok = mbar_wait(&g_full, 0);
       int i = 0;
       for (int t = blockIdx.x; t < p.ntile && ok; t += gridDim.x, ++i) {
-        const int s = i & 1, r = i >> 1;
+        const int s = i % kPtSlots, r = i / kPtSlots, a = i & 1, ra = i >> 1;
         ok = mbar_wait(&x_full[s], r & 1);
-        if (ok && r > 0) ok = mbar_wait(&acc_empty[s], (r - 1) & 1);
+        if (ok && ra > 0) ok = mbar_wait(&acc_empty[a], (ra - 1) & 1);
         if (!ok) break;
         tc_fence_after();
-        const uint32_t d = tmem + (uint32_t)(s * p.n_b);
+        const uint32_t d = tmem + (uint32_t)(a * p.n_b);
 #pragma unroll
         for (int c = 0; c < 2; ++c) {
           const uint64_t ad = sw128_desc(sbase + 4 * gchunk + s * kPtXTile + c * (kPtXTile / 2));
@@ -342,7 +345,7 @@ __global__ void __launch_bounds__(kPtThreads, 1)
           }
         }
         umma_commit(&x_empty[s]);
-        umma_commit(&acc_full[s]);
+        umma_commit(&acc_full[a]);
       }
     }
   } else {
@@ -490,7 +493,7 @@ cudaError_t launch_prep_tc(const sdq_plan_s* pl, const uint16_t* x, int M, void*
   p.R = R; p.k_eff = g.k_eff; p.kpad = g.k_eff_pad;
   p.M = M; p.nblk = g.nblk; p.n_b = g.n_b; p.ternary = pl->desc.quantizer == SDQ_TERNARY;
   p.ntile = (int)((R + kPtRows - 1) / kPtRows);
-  const size_t smem = 1024 + 4 * (size_t)g.n_b * 128 + 2 * (size_t)kPtXTile;
+  const size_t smem = 1024 + 4 * (size_t)g.n_b * 128 + kPtSlots * (size_t)kPtXTile;
   cudaError_t e = cudaFuncSetAttribute(prep_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const int grid = std::min(p.ntile, std::max(1, pl->sm_count));
