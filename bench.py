@@ -44,6 +44,9 @@ def parse():
     ap.add_argument("--m", type=int, default=1, help="decode batch")
     ap.add_argument("--no-extras", action="store_true", help="skip encode/prefill/sweep/cpu legs")
     ap.add_argument("--linears", default="", help="comma list of llama-70b-layer linears to run (default: all 7)")
+    ap.add_argument("--prefill-only", action="store_true",
+                    help="time only the prefill leg (M = 4096) on the chosen linears and print its JSON "
+                         "(for profiling the prefill kernels alone)")
     ap.add_argument("--eager", action="store_true",
                     help="launch every step eagerly instead of replaying a CUDA graph (same kernels; "
                          "for profilers that cannot follow stream capture)")
@@ -384,6 +387,10 @@ def run_sdq(args, rank, world, dist):
         cfg.linears = [l for l in cfg.linears if l.name in keep]
     M = args.m
     layers, enc_ms = build_layer(P, W, torch, cfg)
+    if args.prefill_only:
+        return {"prefill": prefill_leg(P, W, torch, layers, torch.cuda.Stream(), tf_burst, tf_sus, peak_src),
+                "config": {"workload": "llama70b-layer prefill, M = 4096"
+                                       + (f" [only {args.linears}]" if args.linears else "")}}
     code_bytes = sum(l["code_bytes"] for l in layers)
     # per-linear inputs / outputs / workspaces; the step's x and y each live in
     # one buffer (views per linear), so a step moves them with one copy each
