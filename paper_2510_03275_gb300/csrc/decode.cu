@@ -123,6 +123,7 @@ struct DecodeParams {
   int n_out, ntiles, ngroups, ternary, early;
   int atomic_y;          // add into y with float reductions (y zeroed by the prepare kernel, or y += result)
   uint32_t blk_bytes, slot_bytes, b_bytes, sfb_bytes;
+  int brow;   // image rows per block pair in shared memory (8 or NP)
 };
 
 // Bounded wait whose outcome is the same for all lanes of the warp (the
@@ -333,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       // Per stage: one wait, 2 nb MMAs, one commit; stage bookkeeping is
       // kept incremental (a single thread's scalar latency is on the path).
       const uint64_t bd0 = sw128_desc(sbase);
-      const uint64_t astep = (uint64_t)((p.NP * 128) >> 4);   // descriptor units per image row pair
+      const uint64_t astep = (uint64_t)((p.brow * 128) >> 4);   // descriptor units per image row pair
       const uint32_t sfa = tmem + (uint32_t)p.sfa, sfs = tmem + (uint32_t)p.sfs;
       const uint32_t sslot = (uint32_t)p.sss;   // B scale columns per TMEM slot
       const uint32_t aslot = (uint32_t)(kAColsPerBlk * p.sb);
@@ -391,8 +392,15 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       // the code stream the producers have started on the same SM,
       // microseconds of HBM traffic.
       const int a0 = kb0 >> 1, a1 = (kb0 + ncb - 1) >> 1;
-      copy_lsu(reinterpret_cast<uint4*>(bop), reinterpret_cast<const uint4*>(p.bimg + (size_t)a0 * p.NP * 128),
-               (a1 - a0 + 1) * p.NP * 8, et);
+      if (p.brow == p.NP) {
+        copy_lsu(reinterpret_cast<uint4*>(bop), reinterpret_cast<const uint4*>(p.bimg + (size_t)a0 * p.NP * 128),
+                 (a1 - a0 + 1) * p.NP * 8, et);
+      } else {   // the first 8 rows (1 KB) of every pair
+        const uint4* src = reinterpret_cast<const uint4*>(p.bimg + (size_t)a0 * p.NP * 128);
+        uint4* dst = reinterpret_cast<uint4*>(bop);
+        for (int t = et; t < (a1 - a0 + 1) * 64; t += kBuildThreads)
+          cp_async16(dst + t, src + (size_t)(t >> 6) * (p.NP * 8) + (t & 63), 16);
+      }
       copy_lsu(reinterpret_cast<uint4*>(sfbs), reinterpret_cast<const uint4*>(p.sfbw + (size_t)kb0 * p.NP * 4),
                ncb * p.NP / 4, et);
       cp_async_wait_all();
@@ -780,6 +788,8 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
   best.T = decode_terms(M);
   best.NP = (M * best.T + 15) / 16 * 16;
   best.ss = 4 * (((best.NP + 31) / 32 + 3) / 4);
+  best.brow = decode_image(pl) && M * best.T <= 8 ? 8 : best.NP;
+  const int brow = best.brow;
   const int KB = (int)(g.k_eff_pad / kBlk);
   const int sms = std::max(1, pl->sm_count);
   const int blk_bytes = kTileRows * kBlk * g.bits / 8;
@@ -815,7 +825,7 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
         for (int S = 1; S <= KB && (S <= sms || best.S == 0); ++S) {
           const int CB = (KB + S - 1) / S;
           if ((S - 1) * CB >= KB) continue;                      // no empty chunk
-          const int b_bytes = (CB / 2 + 1) * best.NP * 128;       // image rows of the chunk's blocks
+          const int b_bytes = (CB / 2 + 1) * brow * 128;          // image rows of the chunk's blocks
           const int sfb_bytes = (CB * best.NP * 4 + 15) / 16 * 16;  // its B scale words
           const int slot_bytes = sb * blk_bytes;
           // code bytes in flight per CTA: about the SM's share of HBM
@@ -884,7 +894,7 @@ extern "C" int sdq_decode_launch_shape(const sdq_layer_desc* desc, int32_t M, in
   if (dc.S < 1) return SDQ_ERR_UNSUPPORTED;
   const int64_t blk = (int64_t)kTileRows * kBlk * pl.geo.bits / 8;
   const int64_t v[15] = {dc.T, dc.NP, dc.S, dc.P, dc.CB, dc.ring, dc.sb, dc.nbuf, (int64_t)dc.smem,
-                         dc.sb * blk, (int64_t)(dc.CB / 2 + 1) * dc.NP * 128, dc.ss, kSmemMax + 1024, dc.npipe, dc.ns};
+                         dc.sb * blk, (int64_t)(dc.CB / 2 + 1) * dc.brow * 128, dc.ss, kSmemMax + 1024, dc.npipe, dc.ns};
   for (int i = 0; i < 15; ++i) out[i] = v[i];
   return SDQ_OK;
 }
@@ -921,7 +931,8 @@ cudaError_t launch_decode(const sdq_plan_s* pl, const uint32_t* codes, const flo
   p.atomic_y = y_mode == kYAdd || (y_mode == kYZeroed && dc.S > 1);
   p.blk_bytes = (uint32_t)(kTileRows * kBlk * g.bits / 8);
   p.slot_bytes = p.sb * p.blk_bytes;
-  p.b_bytes = (uint32_t)((dc.CB / 2 + 1) * dc.NP * 128);
+  p.b_bytes = (uint32_t)((dc.CB / 2 + 1) * dc.brow * 128);
+  p.brow = dc.brow;
   p.sfb_bytes = (uint32_t)((dc.CB * dc.NP * 4 + 15) / 16 * 16);
   static std::atomic<int> smem_set[64];   // per device: limit raised to kSmemMax + 1 KB
   static std::atomic<int> smem_set_b[64];

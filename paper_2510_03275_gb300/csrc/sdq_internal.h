@@ -55,6 +55,10 @@ struct DecodeConfig {
   int nbuf;               // accumulators per pipeline
   int npipe;              // MMA pipelines (issuing warps, each with its accumulators)
   int ns;                 // TMEM A slots (4 or 8)
+  int brow;               // B image rows per 128-code block pair in shared memory: 8 when
+                          // the M T term rows fit in the first 8-row group (the MMA's rows
+                          // 8..NP-1 then read whatever follows and land in accumulator
+                          // columns nothing reads), else NP
   int dbase;              // TMEM column of the first accumulator
   int sfa, sfs, ss, sss;  // TMEM columns of the A scales, of TMEM slot 0's B
                           // scales, between two blocks' B scales, and between
