@@ -1,13 +1,13 @@
 // K1: row-parallel Sigma-Delta encoder (SDQ-LLM Algorithm 1 without GPTQ
 // compensation; eqs. (3)-(8)).
 //
-// One warp owns 8 output rows.  For every block of B input columns it
+// One warp owns 4 output rows.  For every block of B input columns it
 // rebuilds the upsampled block x_up = A_enc w (A_enc = U Had^T, the
 // Hadamard smoothing of eq. (13) fused with the Resample upsampler) with all
-// 32 lanes, each lane producing 4 of every 128 samples for the 8 rows, in
+// 32 lanes, each lane producing 4 of every 128 samples for the 4 rows, in
 // the canonical fp32 order: one rounded product per term, k ascending, no
 // FMA.  Pass 1 reduces alpha per row (exact max, or the sequential fp32
-// mean); pass 2 recomputes x_up and lanes 0..7 run the first-order
+// mean); pass 2 recomputes x_up and lanes 0..3 run the first-order
 // Sigma-Delta recursion of eq. (8) over their row, reset at every block, and
 // write the codes in the plain packed layout.
 #include "common.cuh"
@@ -16,7 +16,8 @@ namespace sdq {
 
 namespace {
 
-constexpr int kRW = 8;     // rows per warp
+constexpr int kRW = 4;     // rows per warp
+constexpr int kMaxWarps = 16;
 constexpr int kJC = 128;   // upsampled samples per lane pass (4 per lane)
 
 struct EncodeParams {
@@ -28,11 +29,26 @@ struct EncodeParams {
   int64_t k_eff;
 };
 
-__global__ void __launch_bounds__(256) encode_kernel(EncodeParams p) {
+// kTable: the CTA first copies the table into shared memory (where it fits
+// beside the warps' buffers); its reads in the product loop are then
+// shared-memory hits instead of L2 round trips, on which the loop waited.
+template <bool kTable>
+__global__ void __launch_bounds__(32 * kMaxWarps) encode_kernel(EncodeParams p) {
   extern __shared__ float smem[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int xs_stride = p.n_b + 1;
-  float* ws = smem + (size_t)warp * (kRW * p.B + kRW * xs_stride);
+  const float* at = p.at;
+  float* wbuf = smem;
+  if constexpr (kTable) {
+    float* ts = smem;
+    const int n = p.B * p.n_b;
+    for (int i = threadIdx.x; i < n / 4; i += blockDim.x)
+      reinterpret_cast<float4*>(ts)[i] = __ldg(reinterpret_cast<const float4*>(p.at) + i);
+    __syncthreads();
+    at = ts;
+    wbuf = smem + n;
+  }
+  float* ws = wbuf + (size_t)warp * (kRW * p.B + kRW * xs_stride);
   float* xs = ws + kRW * p.B;
   const int row0 = (blockIdx.x * p.warps + warp) * kRW;
   if (row0 >= p.n_out) return;
@@ -66,18 +82,26 @@ __global__ void __launch_bounds__(256) encode_kernel(EncodeParams p) {
           jj[s] = jc + lane + 32 * s;
           jv[s] = jj[s] < p.n_b;
         }
-        for (int k = 0; k < p.B; ++k) {
+        {
           float a[4];
 #pragma unroll
-          for (int s = 0; s < 4; ++s) a[s] = jv[s] ? __ldg(p.at + (size_t)k * p.n_b + jj[s]) : 0.f;
+          for (int s = 0; s < 4; ++s) a[s] = jv[s] ? at[jj[s]] : 0.f;
+#pragma unroll
+          for (int r = 0; r < kRW; ++r) {
+            const float wk = ws[r * p.B];
+#pragma unroll
+            for (int s = 0; s < 4; ++s) acc[r][s] = __fmul_rn(a[s], wk);
+          }
+        }
+        for (int k = 1; k < p.B; ++k) {
+          float a[4];
+#pragma unroll
+          for (int s = 0; s < 4; ++s) a[s] = jv[s] ? at[(size_t)k * p.n_b + jj[s]] : 0.f;
 #pragma unroll
           for (int r = 0; r < kRW; ++r) {
             const float wk = ws[r * p.B + k];
 #pragma unroll
-            for (int s = 0; s < 4; ++s) {
-              const float prod = __fmul_rn(a[s], wk);
-              acc[r][s] = k == 0 ? prod : __fadd_rn(acc[r][s], prod);
-            }
+            for (int s = 0; s < 4; ++s) acc[r][s] = __fadd_rn(acc[r][s], __fmul_rn(a[s], wk));
           }
         }
         if (pass == 0 && !need_xs_pass0) {
@@ -164,17 +188,24 @@ cudaError_t launch_encode(const sdq_plan_s* pl, const float* W, uint32_t* codes,
   p.wpr = g.words_per_row; p.quantizer = pl->desc.quantizer; p.alpha_mode = pl->desc.alpha_mode;
   p.k_eff = g.k_eff;
   const size_t per_warp = sizeof(float) * ((size_t)kRW * g.block + (size_t)kRW * (g.n_b + 1));
-  int warps = (int)((200 * 1024) / per_warp);
-  warps = warps < 1 ? 1 : (warps > 8 ? 8 : warps);
+  const size_t table = sizeof(float) * (size_t)g.block * g.n_b;
   if (per_warp > 227 * 1024) return cudaErrorInvalidConfiguration;
+  // the table in shared memory when it fits beside at least 4 warps' buffers
+  // (a multiple of 4 floats: copied as float4)
+  const bool in_smem = (g.block * g.n_b) % 4 == 0 && table + 4 * per_warp <= 224 * 1024;
+  int warps = (int)(((in_smem ? 224 * 1024 - table : 200 * 1024)) / per_warp);
+  warps = warps < 1 ? 1 : (warps > kMaxWarps ? kMaxWarps : warps);
   p.warps = warps;
-  const size_t smem = per_warp * warps;
-  cudaError_t e = cudaFuncSetAttribute(encode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem);
+  const size_t smem = per_warp * warps + (in_smem ? table : 0);
+  cudaError_t e = in_smem ? cudaFuncSetAttribute(encode_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 (int)smem)
+                          : cudaFuncSetAttribute(encode_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 (int)smem);
   if (e != cudaSuccess) return e;
   const int rows_per_cta = warps * kRW;
   const int grid = (g.n_out + rows_per_cta - 1) / rows_per_cta;
-  encode_kernel<<<grid, warps * 32, smem, st>>>(p);
+  if (in_smem) encode_kernel<true><<<grid, warps * 32, smem, st>>>(p);
+  else encode_kernel<false><<<grid, warps * 32, smem, st>>>(p);
   return cudaGetLastError();
 }
 
