@@ -144,12 +144,14 @@ int sdq_build_tables(const sdq_layer_desc* desc, const int8_t* had_signs,
 
 /* Host-only (no GPU needed): the launch shape the decode contraction takes
  * at batch M (1..64) on a device with `sm_count` SMs, as sdq_plan_create
- * chooses it.  Writes 13 int64 values to `out_host`: T (e2m1 terms per
+ * chooses it.  Writes 16 int64 values to `out_host`: T (e2m1 terms per
  * activation), NP (MMA N), S (k chunks), P (CTAs per chunk), CB (128-code
  * blocks per chunk), ring (stages in the shared-memory ring), sb (blocks per
  * stage), nbuf (accumulators per pipeline), dynamic shared memory bytes,
- * bytes per ring slot, bytes of the B operand image, TMEM columns between
- * two blocks' B scales, and the kernel's shared-memory limit.
+ * bytes per ring slot, bytes of the chunk-resident B operand image (0 when
+ * it streams with the stages), TMEM columns between two blocks' B scales,
+ * the kernel's shared-memory limit, MMA pipelines, TMEM A slots, and 1 when
+ * each stage's B rows and scale words stream into its ring slot.
  * SDQ_ERR_UNSUPPORTED if no shape fits. */
 int sdq_decode_launch_shape(const sdq_layer_desc* desc, int32_t M, int32_t sm_count, int64_t* out_host);
 

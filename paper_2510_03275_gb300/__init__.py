@@ -179,7 +179,7 @@ def sdq_build_tables(desc: LayerDesc, had_signs=None):
 
 
 _SHAPE_KEYS = ("T", "NP", "S", "P", "CB", "ring", "sb", "nbuf", "smem", "slot_bytes", "b_bytes", "ss",
-               "smem_limit", "npipe", "ns")
+               "smem_limit", "npipe", "ns", "bstream")
 
 
 def sdq_decode_launch_shape(desc: LayerDesc, M: int, sm_count: int) -> dict:

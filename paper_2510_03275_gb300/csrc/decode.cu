@@ -68,7 +68,15 @@
 //                 side keep an SM's share of HBM busy
 // With `early` set the producers start the code stream (one stage each)
 // before waiting for the preceding grid (codes are never written by the
-// prep kernels).
+// prep kernels), except with bstream, where each stage also copies B rows
+// and scale words that grid writes.
+//
+// bstream (batches whose term rows make a chunk-resident B image bound the k
+// chunk): each stage's image pairs and scale words are bulk-copied into its
+// ring slot beside the codes, the MMA reads the stage's B rows there, and
+// the stage's MMAs (not the expanders) release the slot; the k chunk is then
+// free of shared-memory limits (S of 2 instead of 10-38 at M = 64, so far
+// fewer split-K partial sums per output).
 // Every mbarrier wait is bounded (about 2 s); a timeout writes the call's
 // tag into the workspace's call record and the CTA drains its copies and
 // MMAs before freeing TMEM.
@@ -124,6 +132,8 @@ struct DecodeParams {
   int atomic_y;          // add into y with float reductions (y zeroed by the prepare kernel, or y += result)
   uint32_t blk_bytes, slot_bytes, b_bytes, sfb_bytes;
   int brow;   // image rows per block pair in shared memory (8 or NP)
+  int bstream;          // stage B rows and scale words stream into the ring slot
+  uint32_t boff, soff;  // their offsets in the slot (bstream)
 };
 
 // Bounded wait whose outcome is the same for all lanes of the warp (the
@@ -231,7 +241,11 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   const int sidx = blockIdx.x % p.S, prow = blockIdx.x / p.S;
   const int kb0 = sidx * p.CB;
   const int ncb = min(p.CB, p.KB - kb0);                        // blocks of this chunk
-  const int spu = max((ncb + p.sb - 1) / p.sb, min(2, ncb));   // stages per tile
+  // stages per tile; with bstream whole block pairs per stage (the image
+  // interleaves a pair's two blocks in its 128-byte rows)
+  const int npairs = (ncb + 1) >> 1;
+  const int spu = p.bstream ? max((2 * npairs + p.sb - 1) / p.sb, min(2, npairs))
+                            : max((ncb + p.sb - 1) / p.sb, min(2, ncb));
   const int nunits = (p.ntiles - prow + p.P - 1) / p.P;         // row tiles of this CTA
   // The CTAs of a row set (one per k chunk) walk its tiles in rotated orders:
   // unit u is tile prow + ((u + rot) mod nunits) P.
@@ -248,7 +262,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   if (warp == 1) {
     if (lane < p.ring) {
       mbar_init(&c_full[lane], 1);
-      mbar_init(&c_empty[lane], 4);   // one arrival per expander warp of the slot's set
+      // one arrival per expander warp of the slot's set, or (bstream: the
+      // MMAs read the slot's B rows) the commit of the stage's MMAs
+      mbar_init(&c_empty[lane], p.bstream ? 1 : 4);
     }
   } else if (warp == 2) {
     if (lane < kASlots) {
@@ -266,7 +282,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
     }
   } else if (warp >= kExpWarp0 && warp < kExpWarp0 + (kMaxSpu + 32) / 32) {
     const int j = tid - 32 * kExpWarp0;
-    if (j <= spu) sblk[j] = stage_block(j, ncb, spu);
+    if (j <= spu) sblk[j] = p.bstream ? min(ncb, 2 * stage_block(j, npairs, spu)) : stage_block(j, ncb, spu);
   } else if (warp >= kExpWarp0 + 6 && warp < kExpWarp0 + 8) {
     red_bits[tid - 32 * (kExpWarp0 + 6)] = 0u;
   }
@@ -284,7 +300,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
   // after their stages)
   const bool builder = warp >= kExpWarp0 && warp < kProducerWarp0;
   const bool epilogue = warp >= kEpiWarp0 && warp < kExpWarp0;
-  if (!builder && !epilogue && (warp < kProducerWarp0 || !p.early)) pdl_wait();
+  // (with bstream the producers copy B rows the preceding grid writes: they
+  // wait for it before their first stage)
+  const bool early = p.early && !p.bstream;
+  if (!builder && !epilogue && (warp < kProducerWarp0 || !early)) pdl_wait();
   const uint32_t tmem = tmem_base;
   bool ok = true;
 
@@ -297,7 +316,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       int last_i = -1, u = 0, j = x, slot = x, r = 0;
       while (j >= spu) { j -= spu; ++u; }
       const uint64_t pol = l2_policy_evict_first();   // codes are read once per call
-      bool waited = !p.early;
+      bool waited = !early;
       for (int i = x; i < nstages && ok; i += kExpSets) {
         // with `early`, kEarlyStages stages ahead of the preceding grid: more
         // would queue ahead of the loads that grid and this CTA's prologue
@@ -310,8 +329,21 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         const uint8_t* src = reinterpret_cast<const uint8_t*>(p.codes) +
                              ((size_t)tile * p.KB + kb0 + b0) * p.blk_bytes;
         const uint32_t bytes = (uint32_t)(b1 - b0) * p.blk_bytes;
-        mbar_expect_tx(&c_full[slot], bytes);
-        bulk_g2s_hint(ring + (size_t)slot * p.slot_bytes, src, bytes, &c_full[slot], pol);
+        uint8_t* dst = ring + (size_t)slot * p.slot_bytes;
+        if (p.bstream) {
+          // the stage's image pairs and scale words (L2 hits: the prepare
+          // kernel wrote them, every CTA of the k chunk reads them)
+          const int pa0 = (kb0 + b0) >> 1, pa1 = (kb0 + b1 + 1) >> 1;
+          const uint32_t bb = (uint32_t)(pa1 - pa0) * (uint32_t)p.NP * 128u;
+          const uint32_t sbytes = (uint32_t)(b1 - b0) * (uint32_t)p.NP * 4u;
+          mbar_expect_tx(&c_full[slot], bytes + bb + sbytes);
+          bulk_g2s_hint(dst, src, bytes, &c_full[slot], pol);
+          bulk_g2s(dst + p.boff, p.bimg + (size_t)pa0 * p.NP * 128, bb, &c_full[slot]);
+          bulk_g2s(dst + p.soff, p.sfbw + (size_t)(kb0 + b0) * p.NP * 4, sbytes, &c_full[slot]);
+        } else {
+          mbar_expect_tx(&c_full[slot], bytes);
+          bulk_g2s_hint(dst, src, bytes, &c_full[slot], pol);
+        }
         last_i = i;
         j += kExpSets;
         while (j >= spu) { j -= spu; ++u; }
@@ -334,6 +366,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
       // Per stage: one wait, 2 nb MMAs, one commit; stage bookkeeping is
       // kept incremental (a single thread's scalar latency is on the path).
       const uint64_t bd0 = sw128_desc(sbase);
+      const uint32_t ring_s = smem_u32(ring);
       const uint64_t astep = (uint64_t)((p.brow * 128) >> 4);   // descriptor units per image row pair
       const uint32_t sfa = tmem + (uint32_t)p.sfa, sfs = tmem + (uint32_t)p.sfs;
       const uint32_t sslot = (uint32_t)p.sss;   // B scale columns per TMEM slot
@@ -357,13 +390,19 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         const int b0 = sblk[j], nb = sblk[j + 1] - b0;
         uint32_t at = tmem + (uint32_t)s * aslot;
         uint32_t sfb = sfs + (uint32_t)s * sslot;
+        const int rslot = i % p.ring;
+        // B rows: the chunk's resident image, or (bstream) the stage's pairs
+        // in its ring slot
+        const uint64_t bdb = p.bstream ? sw128_desc(ring_s + (uint32_t)rslot * p.slot_bytes + p.boff) : bd0;
+        const int pbase = p.bstream ? (kb0 + b0) >> 1 : kb0 >> 1;
         for (int bb = 0; bb < nb; ++bb, at += kAColsPerBlk, sfb += (uint32_t)p.ss) {
           const int bl = b0 + bb, kb = kb0 + bl;
-          const uint64_t bd = bd0 + (uint64_t)((kb >> 1) - (kb0 >> 1)) * astep + 4u * (uint32_t)(kb & 1);
+          const uint64_t bd = bdb + (uint64_t)((kb >> 1) - pbase) * astep + 4u * (uint32_t)(kb & 1);
           umma_mxf4_ts(dt, at, bd, idesc0, sfa, sfb, (first && bb == 0) ? 0u : 1u);
           umma_mxf4_ts(dt, at + 8, bd + 2, idesc1, sfa, sfb, 1u);
         }
         umma_commit(&a_empty[s]);
+        if (p.bstream) umma_commit(&c_empty[rslot]);
         last = i;
         const int u0 = u;
         j += np;
@@ -385,7 +424,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
     // ------------------------------------------------ builders, then expanders
     const int et = tid - 32 * kExpWarp0;
     pdl_wait();
-    if (p.bsrc == 2) {
+    if (p.bstream) {
+      // (the B rows and scale words arrive with each stage)
+    } else if (p.bsrc == 2) {
       // The prepared image rows of the chunk's blocks and their scale words,
       // with 16-byte cp.async copies, all in flight at once (L2 hits: the
       // prepare kernel just wrote them).  A bulk copy here would queue behind
@@ -456,7 +497,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         }
       }
       __syncwarp();
-      if (lane == 0) mbar_arrive(&c_empty[slot]);
+      if (lane == 0 && !p.bstream) mbar_arrive(&c_empty[slot]);
+      // (bstream: the slot's scale words are read below; the MMAs release it)
+      const uint32_t* sws = p.bstream ? reinterpret_cast<const uint32_t*>(cs + p.soff)
+                                      : reinterpret_cast<const uint32_t*>(sfbs) + (size_t)sb0 * p.NP;
       slot += kExpSets;
       if (slot >= p.ring) { slot -= p.ring; ++rnd; }
       if (i >= p.ns) {
@@ -510,8 +554,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
 #pragma unroll
         for (int cc = 0; cc < 4 * kMaxSb; ++cc) {
           const int bb = cc >> 2, n = 32 * (cc & 3) + lane;
-          sv[cc] = (bb < nb && n < MT) ? reinterpret_cast<const uint32_t*>(sfbs)[(sb0 + bb) * p.NP + n]
-                                       : kUnitScales;
+          sv[cc] = (bb < nb && n < MT) ? sws[bb * p.NP + n] : kUnitScales;
         }
         if (p.sss == 16) {
           tmem_st16(sc, sv);
@@ -524,7 +567,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(DecodeParams p) {
         }
       } else {
         for (int bb = 0; bb < nb; ++bb) {
-          const uint32_t* sw = reinterpret_cast<const uint32_t*>(sfbs) + (size_t)(sb0 + bb) * p.NP;
+          const uint32_t* sw = sws + (size_t)bb * p.NP;
           for (int c = 0; 32 * c < p.NP; ++c) {
             const int n = 32 * c + lane;
             tmem_st1(sc + (uint32_t)(bb * p.ss + c), n < MT ? sw[n] : kUnitScales);
@@ -788,13 +831,13 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
   best.T = decode_terms(M);
   best.NP = (M * best.T + 15) / 16 * 16;
   best.ss = 4 * (((best.NP + 31) / 32 + 3) / 4);
-  best.brow = decode_image(pl) && M * best.T <= 8 ? 8 : best.NP;
-  const int brow = best.brow;
+  const int brow = decode_image(pl) && M * best.T <= 8 ? 8 : best.NP;
   const int KB = (int)(g.k_eff_pad / kBlk);
   const int sms = std::max(1, pl->sm_count);
   const int blk_bytes = kTileRows * kBlk * g.bits / 8;
   const double clk = 1.9e9;
   const double hbm = 6.0e12, cta_bw = 30e9;                    // bytes/s: HBM, one CTA's copy ring
+  const double l2_bw = 20e12;                                  // bytes/s: L2 reads of streamed B rows
   const double t_tail = 2.0e-6, ring_latency = 4.0e-6;   // a ring slot's round trip under load
   const double c_mma = 150.0 + 0.5 * best.NP, c_stage = 550.0;   // issuing thread, cycles
   const double c_xblk = 200.0, c_xstage = 600.0;                 // expander set, cycles
@@ -805,6 +848,11 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
   for (int pi = 0; pi < 3; ++pi)
     t_epi[pi] = MT <= 16 ? 0.0   // (one or two batch rows: within the fitted per-tile cost below)
                          : ((MT + 15) / 16) * (385.0 * pipes[pi] + 650.0) / clk;
+  // bstream 1: the stage's B rows and scale words stream into its ring slot
+  // (whole block pairs per stage); only where the prepare kernel writes the
+  // image, and for batches whose chunk-resident image would bound the k
+  // chunk (M T > 8)
+  for (int bs = 0; bs <= (decode_image(pl) && MT > 8 ? 1 : 0); ++bs)
   for (int pi = 0; pi < 3; ++pi) {
     const int np = pipes[pi];
     for (int ns = 4; ns <= kASlots; ns *= 2)
@@ -818,23 +866,29 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
         // store that writes them); then A's scales
         int sb = kMaxSb, sss = 0;
         for (; sb >= 1; --sb) {
+          if (bs && (sb & 1)) continue;
           sss = best.ss == 4 ? (sb == 1 ? 4 : (sb == 2 ? 8 : 16)) : sb * best.ss;
           if (ns * (kAColsPerBlk * sb + sss) + kSfaCols <= dbase) break;
         }
         if (sb < 1) continue;                                    // TMEM
         for (int S = 1; S <= KB && (S <= sms || best.S == 0); ++S) {
-          const int CB = (KB + S - 1) / S;
+          int CB = (KB + S - 1) / S;
+          if (bs && S > 1) CB += CB & 1;                         // chunks start on a block pair
           if ((S - 1) * CB >= KB) continue;                      // no empty chunk
-          const int b_bytes = (CB / 2 + 1) * brow * 128;          // image rows of the chunk's blocks
-          const int sfb_bytes = (CB * best.NP * 4 + 15) / 16 * 16;  // its B scale words
-          const int slot_bytes = sb * blk_bytes;
+          const int b_bytes = bs ? 0 : (CB / 2 + 1) * brow * 128;    // image rows of the chunk's blocks
+          const int sfb_bytes = bs ? 0 : (CB * best.NP * 4 + 15) / 16 * 16;  // its B scale words
+          const int code_slot = sb * blk_bytes;
+          const int bslot = (sb / 2) * best.NP * 128 + sb * best.NP * 4;    // streamed B rows + scales
+          const int slot_bytes = bs ? (code_slot + bslot + 1023) / 1024 * 1024 : code_slot;
           // code bytes in flight per CTA: about the SM's share of HBM
           // bandwidth at the loaded latency, at least two stages per set
           int ring = std::min(kMaxRing, (kSmemMax - 2048 - b_bytes - sfb_bytes) / slot_bytes);
-          ring = std::min(ring, std::max(2 * kExpSets, (kRingBytes + slot_bytes - 1) / slot_bytes + kExpSets - 1));
+          ring = std::min(ring, std::max(2 * kExpSets, (kRingBytes + code_slot - 1) / code_slot + kExpSets - 1));
           ring -= ring % kExpSets;          // each ring slot belongs to one expander set
           if (ring < kExpSets) continue;
-          const int spu = std::max((CB + sb - 1) / sb, std::min(2, CB));
+          const int npr = (CB + 1) / 2;
+          const int spu = bs ? std::max((2 * npr + sb - 1) / sb, std::min(2, npr))
+                             : std::max((CB + sb - 1) / sb, std::min(2, CB));
           if (spu > kMaxSpu) continue;
           const double issue = 2.0 * sb * c_mma + c_stage;        // cycles per stage, one pipeline
           const double expand = c_xstage + c_xblk * sb;           // cycles per stage, one set
@@ -842,7 +896,7 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
           const double mma_rate = std::min(np / issue, kExpSets / set_cyc) * clk;   // stages per second per CTA
           // the prologue: the wait for the prepare kernel, the B operand (image
           // copy or terms formed in the CTA)
-          const double t_build = 2.0e-6 + (b_bytes + sfb_bytes) / 25e9 + CB * M * best.T * 2.0e-9;
+          const double t_build = bs ? 2.0e-6 : 2.0e-6 + (b_bytes + sfb_bytes) / 25e9 + CB * M * best.T * 2.0e-9;
           for (int P = 1; P <= std::min(g.ntiles, std::max(1, sms / S)); ++P) {
             const int grid = S * P;
             const int waves = (grid + sms - 1) / sms;
@@ -850,13 +904,15 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
             // A CTA streams its units row tiles (CB blocks each) at the
             // lowest of: the measured per-CTA ceiling of the copy ring, its
             // share of HBM bandwidth, and the rate its MMA pipelines and
-            // expander sets sustain; every row tile adds a cost that grows
+            // expander sets sustain (and, streaming B, its share of the L2's
+            // bandwidth for the B rows); every row tile adds a cost that grows
             // with the k chunks adding into the same rows of y (accumulator
             // hand-off, epilogue, split-K contention: fitted to measured
             // calls), every call a prologue and a tail.
             const double tile_bytes = (double)CB * blk_bytes;
-            const double rate = std::min({cta_bw, hbm / std::min(grid, sms), mma_rate * slot_bytes,
-                                          (double)ring * slot_bytes / ring_latency});
+            double rate = std::min({cta_bw, hbm / std::min(grid, sms), mma_rate * code_slot,
+                                    (double)ring * code_slot / ring_latency});
+            if (bs) rate = std::min(rate, l2_bw / std::min(grid, sms) * code_slot / bslot);
             // the tile's epilogue (accumulator loads per pipeline and the
             // terms' sums and writes per 16 columns, measured per tile) runs
             // beside the next tile's MMAs with two accumulators, else between
@@ -868,6 +924,8 @@ DecodeConfig decode_config_search(const sdq_plan_s* pl, int M) {
               best_t = t;
               best.S = S; best.P = P; best.CB = CB; best.ring = ring; best.sb = sb;
               best.npipe = np; best.ns = ns; best.nbuf = nbuf; best.dbase = dbase; best.sss = sss;
+              best.bstream = bs; best.brow = bs ? best.NP : brow;
+              best.slot_bytes = slot_bytes; best.boff = code_slot; best.soff = code_slot + (sb / 2) * best.NP * 128;
               best.smem = std::max<size_t>(kSmemMin, 1024 + (size_t)b_bytes + sfb_bytes + (size_t)ring * slot_bytes);
             }
           }
@@ -893,9 +951,10 @@ extern "C" int sdq_decode_launch_shape(const sdq_layer_desc* desc, int32_t M, in
   const DecodeConfig dc = decode_config_search(&pl, M);
   if (dc.S < 1) return SDQ_ERR_UNSUPPORTED;
   const int64_t blk = (int64_t)kTileRows * kBlk * pl.geo.bits / 8;
-  const int64_t v[15] = {dc.T, dc.NP, dc.S, dc.P, dc.CB, dc.ring, dc.sb, dc.nbuf, (int64_t)dc.smem,
-                         dc.sb * blk, (int64_t)(dc.CB / 2 + 1) * dc.brow * 128, dc.ss, kSmemMax + 1024, dc.npipe, dc.ns};
-  for (int i = 0; i < 15; ++i) out[i] = v[i];
+  const int64_t v[16] = {dc.T, dc.NP, dc.S, dc.P, dc.CB, dc.ring, dc.sb, dc.nbuf, (int64_t)dc.smem,
+                         dc.slot_bytes, dc.bstream ? 0 : (int64_t)(dc.CB / 2 + 1) * dc.brow * 128, dc.ss,
+                         kSmemMax + 1024, dc.npipe, dc.ns, dc.bstream};
+  for (int i = 0; i < 16; ++i) out[i] = v[i];
   return SDQ_OK;
 }
 
@@ -930,10 +989,11 @@ cudaError_t launch_decode(const sdq_plan_s* pl, const uint32_t* codes, const flo
   p.early = early;
   p.atomic_y = y_mode == kYAdd || (y_mode == kYZeroed && dc.S > 1);
   p.blk_bytes = (uint32_t)(kTileRows * kBlk * g.bits / 8);
-  p.slot_bytes = p.sb * p.blk_bytes;
-  p.b_bytes = (uint32_t)((dc.CB / 2 + 1) * dc.brow * 128);
+  p.slot_bytes = (uint32_t)dc.slot_bytes;
+  p.bstream = dc.bstream; p.boff = (uint32_t)dc.boff; p.soff = (uint32_t)dc.soff;
+  p.b_bytes = dc.bstream ? 0u : (uint32_t)((dc.CB / 2 + 1) * dc.brow * 128);
   p.brow = dc.brow;
-  p.sfb_bytes = (uint32_t)((dc.CB * dc.NP * 4 + 15) / 16 * 16);
+  p.sfb_bytes = dc.bstream ? 0u : (uint32_t)((dc.CB * dc.NP * 4 + 15) / 16 * 16);
   static std::atomic<int> smem_set[64];   // per device: limit raised to kSmemMax + 1 KB
   static std::atomic<int> smem_set_b[64];
   cudaError_t e = p.ternary ? smem_limit_once(decode_kernel<true>, kSmemMax + 1024, pl->device, smem_set)

@@ -59,6 +59,11 @@ struct DecodeConfig {
                           // the M T term rows fit in the first 8-row group (the MMA's rows
                           // 8..NP-1 then read whatever follows and land in accumulator
                           // columns nothing reads), else NP
+  int bstream;            // 1: each stage's B image rows and scale words stream into its
+                          // ring slot beside the codes (no chunk-resident image), so the
+                          // k chunk is not bounded by shared memory
+  int slot_bytes;         // ring slot: codes, then (bstream) B rows at boff, scales at soff
+  int boff, soff;
   int dbase;              // TMEM column of the first accumulator
   int sfa, sfs, ss, sss;  // TMEM columns of the A scales, of TMEM slot 0's B
                           // scales, between two blocks' B scales, and between

@@ -125,8 +125,8 @@ def test_decode_launch_shapes_fit(sdq, sms):
     16 sb code columns and their B-scale columns: sb 4-aligned sets, with
     4-column sets rounded up to one 4, 8 or 16-column store, 4 A-scale
     columns, npipe x nbuf accumulators), the B
-    image (8 or NP rows per block pair), its scale words and the ring within
-    the shared-memory limit, and
+    image (8 or NP rows per block pair) or the streamed stage slots, its
+    scale words and the ring within the shared-memory limit, and
     the e2m1 term count of the batch size."""
     for n, k, b, osr, qz in _launch_shapes():
         d = sdq.LayerDesc(n, k, b, osr, qz, 1, 0)
@@ -144,15 +144,28 @@ def test_decode_launch_shapes_fit(sdq, sms):
             assert 1 <= s["sb"] <= 4
             sss = ({1: 4, 2: 8}.get(s["sb"], 16) if s["ss"] == 4 else s["sb"] * s["ss"])
             assert s["ns"] * (16 * s["sb"] + sss) + 4 + s["npipe"] * s["nbuf"] * s["NP"] <= 512
-            assert s["slot_bytes"] == s["sb"] * blk
-            # the image's rows per block pair: the first 8-row group alone when
-            # the batch's term rows fit in it and the prepare kernel writes
-            # the image (n_b a multiple of 64)
             n_b = sdq.sdq_k_eff(d) // (k // b)
-            brow = 8 if (n_b % 64 == 0 and m * t <= 8) else s["NP"]
-            assert s["b_bytes"] == (s["CB"] // 2 + 1) * brow * 128
-            sfb = -(-(s["CB"] * s["NP"] * 4) // 16) * 16   # the chunk's B scale words
-            assert 1024 + s["b_bytes"] + sfb + s["ring"] * s["slot_bytes"] <= s["smem"] <= s["smem_limit"]
-            assert max(-(-s["CB"] // s["sb"]), min(2, s["CB"])) <= 128   # stages per row tile
+            if s["bstream"]:
+                # B rows and scale words stream with each stage: whole block
+                # pairs (even sb, chunks starting on a pair), only where the
+                # prepare kernel writes the image, slots 1 KB-aligned
+                assert n_b % 64 == 0 and m * t > 8 and s["sb"] % 2 == 0
+                assert s["S"] == 1 or s["CB"] % 2 == 0
+                bslot = s["sb"] // 2 * s["NP"] * 128 + s["sb"] * s["NP"] * 4
+                assert s["slot_bytes"] == -(-(s["sb"] * blk + bslot) // 1024) * 1024
+                assert s["b_bytes"] == 0
+                assert 1024 + s["ring"] * s["slot_bytes"] <= s["smem"] <= s["smem_limit"]
+                npr = -(-s["CB"] // 2)
+                assert max(-(-2 * npr // s["sb"]), min(2, npr)) <= 128   # stages per row tile
+            else:
+                assert s["slot_bytes"] == s["sb"] * blk
+                # the image's rows per block pair: the first 8-row group alone
+                # when the batch's term rows fit in it and the prepare kernel
+                # writes the image (n_b a multiple of 64)
+                brow = 8 if (n_b % 64 == 0 and m * t <= 8) else s["NP"]
+                assert s["b_bytes"] == (s["CB"] // 2 + 1) * brow * 128
+                sfb = -(-(s["CB"] * s["NP"] * 4) // 16) * 16   # the chunk's B scale words
+                assert 1024 + s["b_bytes"] + sfb + s["ring"] * s["slot_bytes"] <= s["smem"] <= s["smem_limit"]
+                assert max(-(-s["CB"] // s["sb"]), min(2, s["CB"])) <= 128   # stages per row tile
 
 
