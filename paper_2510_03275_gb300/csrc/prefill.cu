@@ -235,7 +235,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 //              columns each): bf16 x_tilde (round to nearest even) in the
 //              prefill operand order (prefill_pos64) with 16-byte stores;
 //              the K padding of every batch row set to zero
-// Bounded waits as in the contraction kernels.
+// Layers with n_b above 256 take one launch per 256 or fewer columns (x read
+// once per launch).  Bounded waits as in the contraction kernels.
 constexpr int kPtEpiWarps = 8;
 constexpr int kPtThreads = 64 + 32 * kPtEpiWarps;
 constexpr int kPtRows = 128;
@@ -248,6 +249,7 @@ struct PrepTcParams {
   uint64_t call;
   int64_t R, k_eff, kpad;
   int M, nblk, n_b, ntile, ternary;
+  int j0, ncol;   // this launch's x_tilde columns j0 .. j0 + ncol - 1 of every block (ncol <= 256)
 };
 
 __global__ void __launch_bounds__(kPtThreads, 1)
@@ -259,11 +261,11 @@ __global__ void __launch_bounds__(kPtThreads, 1)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
   uint8_t* base = smem_raw + (sbase - smem_u32(smem_raw));
-  const uint32_t gchunk = (uint32_t)p.n_b * 128u;   // one 64-wide K chunk of G^T: n_b rows x 128 B
+  const uint32_t gchunk = (uint32_t)p.ncol * 128u;  // one 64-wide K chunk of G^T: ncol rows x 128 B
   uint8_t* gh = base;                               // 2 chunks
   uint8_t* gl = base + 2 * gchunk;                  // 2 chunks
   uint8_t* xs = base + 4 * gchunk;                  // kPtSlots ring slots
-  const uint32_t tcols = p.n_b <= 64 ? 128u : (p.n_b <= 128 ? 256u : 512u);
+  const uint32_t tcols = p.ncol <= 64 ? 128u : (p.ncol <= 128 ? 256u : 512u);
 
   if (tid == 0) {
     mbar_init(&g_full, 1);
@@ -310,7 +312,7 @@ __global__ void __launch_bounds__(kPtThreads, 1)
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(p.n_b >> 3) << 17) |
+      const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(p.ncol >> 3) << 17) |
                              ((uint32_t)(kPtRows >> 4) << 24);
       ok = mbar_wait(&g_full, 0);
       int i = 0;
@@ -320,7 +322,7 @@ __global__ void __launch_bounds__(kPtThreads, 1)
         if (ok && ra > 0) ok = mbar_wait(&acc_empty[a], (ra - 1) & 1);
         if (!ok) break;
         tc_fence_after();
-        const uint32_t d = tmem + (uint32_t)(a * p.n_b);
+        const uint32_t d = tmem + (uint32_t)(a * p.ncol);
 #pragma unroll
         for (int c = 0; c < 2; ++c) {
           const uint64_t ad = sw128_desc(sbase + 4 * gchunk + s * kPtXTile + c * (kPtXTile / 2));
@@ -339,13 +341,15 @@ __global__ void __launch_bounds__(kPtThreads, 1)
   } else {
     pdl_wait();   // the workspace belongs to the preceding grid until then
     const int et = tid - 64, q = warp & 3, half = (warp - 2) >> 2;
-    // the K padding of every batch row (k_eff .. kpad, a multiple of 8)
+    // the K padding of every batch row (k_eff .. kpad, a multiple of 8; by
+    // the launch of the first columns)
+    if (p.j0 == 0)
     for (int64_t z = (int64_t)blockIdx.x * (32 * kPtEpiWarps) + et; z < (int64_t)p.M * ((p.kpad - p.k_eff) / 8);
          z += (int64_t)gridDim.x * (32 * kPtEpiWarps)) {
       const int64_t per = (p.kpad - p.k_eff) / 8, m = z / per;
       *reinterpret_cast<uint4*>(p.xtb + m * p.kpad + p.k_eff + 8 * (z - m * per)) = make_uint4(0, 0, 0, 0);
     }
-    const int cw = p.n_b / 2;                                   // this warp's columns
+    const int cw = p.ncol / 2;                                  // this warp's columns
     const uint32_t lq = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(half * cw);
     int i = 0;
     for (int t = blockIdx.x; t < p.ntile && ok; t += gridDim.x, ++i) {
@@ -356,8 +360,8 @@ __global__ void __launch_bounds__(kPtThreads, 1)
       const int64_t row = (int64_t)t * kPtRows + 32 * q + lane;
       const bool live = row < p.R;
       const int64_t m = live ? row / p.nblk : 0;
-      uint16_t* out = p.xtb + m * p.kpad + (live ? (row - m * p.nblk) * p.n_b : 0) + half * cw;
-      const uint32_t acol = (uint32_t)(s * p.n_b);
+      uint16_t* out = p.xtb + m * p.kpad + (live ? (row - m * p.nblk) * p.n_b : 0) + p.j0 + half * cw;
+      const uint32_t acol = (uint32_t)(s * p.ncol);
       // 32 columns at a time: a ternary operand permutes within 16, a binary
       // one within 32 positions (prefill_pos64); physical pair (2k, 2k + 1)
       // of a 16 (32) holds logical 7 - k and 15 - k (15 - k and 31 - k)
@@ -439,19 +443,22 @@ cudaError_t launch_prefill(const sdq_plan_s* pl, const uint32_t* codes, const fl
 
 
 // The prefill prepare kernel on the tensor cores where it applies (B = 128,
-// n_b a multiple of 64 up to 256, x 16-byte aligned); *used = false otherwise.
+// n_b a multiple of 64, x 16-byte aligned), one launch per 256 or fewer of
+// the n_b columns; *used = false otherwise.
 cudaError_t launch_prep_tc(const sdq_plan_s* pl, const uint16_t* x, int M, void* ws, cudaStream_t st,
                            bool* used) {
   const Geometry& g = pl->geo;
   *used = false;
-  if (g.block != 128 || g.n_b % 64 != 0 || g.n_b > 256 || (reinterpret_cast<uintptr_t>(x) & 15u)) return cudaSuccess;
+  if (g.block != 128 || g.n_b % 64 != 0 || (reinterpret_cast<uintptr_t>(x) & 15u)) return cudaSuccess;
   auto enc = encode_fn();
   if (!enc) return cudaSuccess;
   const WsLayout L = workspace_layout(pl, M);
   uint8_t* wbase = static_cast<uint8_t*>(ws);
   const int64_t R = (int64_t)M * g.nblk;
   if (R >= (int64_t(1) << 31) - kPtRows) return cudaSuccess;
-  CUtensorMap xmap, ghmap, glmap;
+  const int nparts = (g.n_b + 255) / 256;
+  CUtensorMap xmap, ghmap[16], glmap[16];
+  if (nparts > 16) return cudaSuccess;
   const cuuint32_t estr[2] = {1, 1};
   {
     const cuuint64_t dims[2] = {128, (cuuint64_t)R};
@@ -462,31 +469,42 @@ cudaError_t launch_prep_tc(const sdq_plan_s* pl, const uint16_t* x, int M, void*
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaSuccess;
   }
-  {
-    const cuuint64_t dims[2] = {128, (cuuint64_t)g.n_b};
+  int j0s[16], ncols[16];
+  for (int q = 0, j0 = 0; q < nparts; ++q) {
+    const int ncol = std::min(256, g.n_b - j0);
+    const cuuint64_t dims[2] = {128, (cuuint64_t)ncol};
     const cuuint64_t strides[1] = {256};
-    const cuuint32_t box[2] = {64, (cuuint32_t)g.n_b};
-    if (enc(&ghmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, pl->d_g_hi, dims, strides, box, estr,
+    const cuuint32_t box[2] = {64, (cuuint32_t)ncol};
+    if (enc(&ghmap[q], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, pl->d_g_hi + (size_t)j0 * 128, dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS ||
-        enc(&glmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, pl->d_g_lo, dims, strides, box, estr,
+        enc(&glmap[q], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, pl->d_g_lo + (size_t)j0 * 128, dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaSuccess;
+    j0s[q] = j0;
+    ncols[q] = ncol;
+    j0 += ncol;
   }
   PrepTcParams p;   // (a timeout is recorded under this kernel's own call number)
   p.xtb = reinterpret_cast<uint16_t*>(wbase + L.xt);
   p.rec = reinterpret_cast<uint64_t*>(wbase + L.err);
-  p.call = call_tag(next_call_number());
   p.R = R; p.k_eff = g.k_eff; p.kpad = g.k_eff_pad;
   p.M = M; p.nblk = g.nblk; p.n_b = g.n_b; p.ternary = pl->desc.quantizer == SDQ_TERNARY;
   p.ntile = (int)((R + kPtRows - 1) / kPtRows);
-  const size_t smem = 1024 + 4 * (size_t)g.n_b * 128 + kPtSlots * (size_t)kPtXTile;
-  cudaError_t e = cudaFuncSetAttribute(prep_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  const size_t smem_max = 1024 + 4 * (size_t)256 * 128 + kPtSlots * (size_t)kPtXTile;
+  cudaError_t e = cudaFuncSetAttribute(prep_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_max);
   if (e != cudaSuccess) return e;
   const int grid = std::min(p.ntile, std::max(1, pl->sm_count));
   *used = true;
-  return launch_pdl(prep_tc_kernel, dim3(grid), dim3(kPtThreads), smem, st, xmap, ghmap, glmap, p);
+  for (int q = 0; q < nparts; ++q) {
+    p.call = call_tag(next_call_number());
+    p.j0 = j0s[q];
+    p.ncol = ncols[q];
+    const size_t smem = 1024 + 4 * (size_t)p.ncol * 128 + kPtSlots * (size_t)kPtXTile;
+    e = launch_pdl(prep_tc_kernel, dim3(grid), dim3(kPtThreads), smem, st, xmap, ghmap[q], glmap[q], p);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
-
 }  // namespace sdq
