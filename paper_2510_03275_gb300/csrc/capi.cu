@@ -82,6 +82,8 @@ WsLayout workspace_layout(const sdq_plan_s* pl, int M) {
     off = align_up(off + 2 * sizeof(uint64_t), 256);
   } else {
     off = align_up(off + sizeof(uint16_t) * (size_t)M * g.k_eff_pad, 256);
+    L.what = off;                                  // dense route: W', n_out x k_in bf16
+    if (dense_route_applies(pl, M)) off = align_up(off + sizeof(uint16_t) * (size_t)g.n_out * g.k_in, 256);
     L.bimg = L.sfbw = L.part = L.cnt = L.err = off;   // call record only
     off = align_up(off + 2 * sizeof(uint64_t), 256);
   }
@@ -119,6 +121,23 @@ extern "C" int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_sig
     ghi[i] = host_bf16(gm[i]);
     glo[i] = host_bf16((double)gm[i] - host_bf16_value(ghi[i]));
   }
+  // G^T for the dense large-batch route: row k (an input of the block), its
+  // n_b codes' weights in the order the code expansion presents them to the
+  // tensor cores (within each 64-code chunk, logical code kl at position
+  // prefill_pos64(kl)); hi and lo parts as for G
+  const bool dense_tabs = g.block == 128 && g.n_b % 64 == 0 && g.n_b <= kDenseMaxNb;
+  std::vector<uint16_t> gthi, gtlo;
+  if (dense_tabs) {
+    gthi.resize(tab);
+    gtlo.resize(tab);
+    const bool ter = desc->quantizer == SDQ_TERNARY;
+    for (int k = 0; k < g.block; ++k)
+      for (int j = 0; j < g.n_b; ++j) {
+        const size_t dst = (size_t)k * g.n_b + (j & ~63) + prefill_pos64(j & 63, ter);
+        gthi[dst] = ghi[(size_t)j * g.block + k];
+        gtlo[dst] = glo[(size_t)j * g.block + k];
+      }
+  }
 
   sdq_plan_s* p = new (std::nothrow) sdq_plan_s();
   if (!p) return SDQ_ERR_ALLOC;
@@ -131,6 +150,16 @@ extern "C" int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_sig
       cudaMalloc(&p->d_g_lo, sizeof(uint16_t) * tab) != cudaSuccess) {
     sdq_plan_destroy(p);
     return SDQ_ERR_ALLOC;
+  }
+  if (dense_tabs && (cudaMalloc(&p->d_gt_hi, sizeof(uint16_t) * tab) != cudaSuccess ||
+                     cudaMalloc(&p->d_gt_lo, sizeof(uint16_t) * tab) != cudaSuccess)) {
+    sdq_plan_destroy(p);
+    return SDQ_ERR_ALLOC;
+  }
+  if (dense_tabs && (cudaMemcpy(p->d_gt_hi, gthi.data(), sizeof(uint16_t) * tab, cudaMemcpyHostToDevice) != cudaSuccess ||
+                     cudaMemcpy(p->d_gt_lo, gtlo.data(), sizeof(uint16_t) * tab, cudaMemcpyHostToDevice) != cudaSuccess)) {
+    sdq_plan_destroy(p);
+    return SDQ_ERR_CUDA;
   }
   if (cudaMemcpy(p->d_at, at.data(), sizeof(float) * tab, cudaMemcpyHostToDevice) != cudaSuccess ||
       cudaMemcpy(p->d_g_hi, ghi.data(), sizeof(uint16_t) * tab, cudaMemcpyHostToDevice) != cudaSuccess ||
@@ -149,6 +178,8 @@ extern "C" int sdq_plan_destroy(sdq_plan p) {
   if (p->d_at && (e2 = cudaFree(p->d_at)) != cudaSuccess) e = e2;
   if (p->d_g_hi && (e2 = cudaFree(p->d_g_hi)) != cudaSuccess) e = e2;
   if (p->d_g_lo && (e2 = cudaFree(p->d_g_lo)) != cudaSuccess) e = e2;
+  if (p->d_gt_hi && (e2 = cudaFree(p->d_gt_hi)) != cudaSuccess) e = e2;
+  if (p->d_gt_lo && (e2 = cudaFree(p->d_gt_lo)) != cudaSuccess) e = e2;
   delete p;
   return cuda_status(e);
 }
@@ -229,6 +260,12 @@ extern "C" int sdq_linear_forward(sdq_plan p, const uint32_t* codes_tiled, const
   int st = check_ws(p, M, ws, ws_bytes);
   if (st != SDQ_OK) return st;
   if (!x || !aligned16(x) || !y || !aligned16(y)) return SDQ_ERR_INVALID_ARG;
+  if (M > kMaxDecodeM && dense_route_applies(p, M)) {
+    // large batches: rebuild the weights, then one dense GEMM
+    if (!codes_tiled || !alpha || !aligned16(codes_tiled)) return SDQ_ERR_INVALID_ARG;
+    const cudaError_t e = launch_dense_forward(p, codes_tiled, alpha, x, M, y, ws, (cudaStream_t)stream);
+    if (e != cudaErrorNotSupported) return cuda_status(e);
+  }
   st = cuda_status(launch_prep(p, x, M, ws, (cudaStream_t)stream, zero_y ? y : nullptr));
   if (st != SDQ_OK) return st;
   return contract(p, codes_tiled, alpha, M, y, ws, ws_bytes, stream, 1, zero_y ? kYZeroed : kYStore);

@@ -19,6 +19,7 @@ inline const DecodeConfig& decode_config(const sdq_plan_s* plan, int M) { return
 // tile; err: the call record (two 64-bit words, see call_record_*).
 struct WsLayout {
   size_t xt, bimg, sfbw, part, cnt, err, total;
+  size_t what;   // rebuilt weights W' (n_out x k_in bf16) of the dense large-batch route
 };
 WsLayout workspace_layout(const sdq_plan_s* plan, int M);
 // SDQ_OK when the current device is the plan's, else SDQ_ERR_INVALID_ARG (or
@@ -43,6 +44,13 @@ cudaError_t launch_unpack(const sdq_plan_s* p, const uint32_t* tiled, uint32_t* 
 // y_zero (M x n_out, may be null): cleared by the decode prepare kernel.
 cudaError_t launch_prep(const sdq_plan_s* p, const uint16_t* x, int M, void* ws, cudaStream_t st,
                         float* y_zero = nullptr);
+// The dense large-batch route (rebuild W' = 2 C G, then y = alpha / 2 W' x):
+// whether it applies to plan p at batch M, and its two launches.
+bool dense_route_applies(const sdq_plan_s* p, int M);
+cudaError_t launch_dense_forward(const sdq_plan_s* p, const uint32_t* codes, const float* alpha,
+                                 const uint16_t* x, int M, float* y, void* ws, cudaStream_t st);
+// cuTensorMapEncodeTiled from the driver (null if unavailable), as void*.
+void* tensor_map_encoder();
 // Prefill prepare (M > 64) on the tensor cores where the layer allows it;
 // *used = false (nothing launched) otherwise.
 cudaError_t launch_prep_tc(const sdq_plan_s* p, const uint16_t* x, int M, void* ws, cudaStream_t st,

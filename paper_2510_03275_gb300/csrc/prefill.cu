@@ -412,6 +412,8 @@ __global__ void __launch_bounds__(kPtThreads, 1)
 
 }  // namespace
 
+void* tensor_map_encoder() { return reinterpret_cast<void*>(encode_fn()); }
+
 cudaError_t launch_prefill(const sdq_plan_s* pl, const uint32_t* codes, const float* alpha, int M,
                            float* y, void* ws, cudaStream_t st) {
   const Geometry& g = pl->geo;

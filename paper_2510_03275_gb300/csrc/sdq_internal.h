@@ -42,6 +42,11 @@ constexpr int kMaxDecodeM = 64;
 // where the MMA N = M T stays within 32 columns, 4 (2^-12) up to 16, 3
 // (2^-9, the level of the single bf16 rounding of x_tilde on the prefill
 // path) above.
+// Large batches (M >= kDenseMinM) run sdq_linear_forward as "rebuild the
+// weights, then one dense GEMM" (csrc/dense.cu) where the plan allows it.
+constexpr int kDenseMinM = 1024;
+constexpr int kDenseMaxNb = 384;   // G^T hi + lo resident in shared memory
+
 inline int decode_terms(int M) { return M <= 4 ? 6 : (M <= 16 ? 4 : 3); }
 
 // Launch shape of the decode kernel for one batch size (chosen at plan time).
@@ -81,5 +86,9 @@ struct sdq_plan_s {
   float* d_at;         // encode table, transposed: B x n_b (At[k][j] = A_enc[j][k])
   uint16_t* d_g_hi;    // G as bf16 hi part, n_b x B row-major
   uint16_t* d_g_lo;    // G - hi as bf16, n_b x B row-major
+  uint16_t* d_gt_hi;   // G^T as bf16 hi / lo parts, B x n_b, each 64-code chunk in the
+  uint16_t* d_gt_lo;   // code expansion's K order (prefill_pos64); null where the dense
+                       // large-batch route does not apply (B != 128, n_b not a multiple
+                       // of 64 or above kDenseMaxNb)
   sdq::DecodeConfig dcfg[sdq::kMaxDecodeM + 1];  // decode launch shape per batch size
 };
