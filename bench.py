@@ -349,8 +349,12 @@ def extra_configs_leg(P, W, torch, stream, hbm):
         "osr": sorted({str(l.osr) for l in cfg.linears}),
         "decode_m8": dec,
         "prefill_m2048": {"tflops_contraction": round(flops / (ms_k5 * 1e-3) / 1e12, 1),
-                          "tflops_with_prepare": round(flops / (ms_all * 1e-3) / 1e12, 1),
-                          "ms_contraction": round(ms_k5, 3), "ms_with_prepare": round(ms_all, 3),
+                          "tflops_forward": round(flops / (ms_all * 1e-3) / 1e12, 1),
+                          "ms_contraction": round(ms_k5, 3), "ms_forward": round(ms_all, 3),
+                          "forward_routes": sorted({P.sdq_forward_route(lay["plan"].handle, M) for lay in lays}),
+                          "what": "code-domain flops (2 M N K_eff) per time: the code-domain contraction "
+                                  "kernel alone, and sdq_linear_forward as it runs at this batch (route 3: "
+                                  "weights rebuilt, then one GEMM; route 2: prepare + contraction)",
                           "flops": flops}}
     del lays, flush
     torch.cuda.empty_cache()
@@ -611,44 +615,73 @@ def decode_sweep(P, W, torch, layers, stream, hbm_gbs, tf_bf16, peak_src):
 
 
 def prefill_leg(P, W, torch, layers, stream, tf_burst, tf_sus, peak_src):
+    """M = 4096 over the 7 linears: the code-domain contraction kernel alone
+    (its roofline), the code-domain route with its prepare kernel, and
+    sdq_linear_forward as it runs at this batch (the dense route where the
+    plan allows it: weights rebuilt, then one GEMM)."""
     import numpy as np
     M = 4096
-    flops, ms, ms_p = 0, 0.0, 0.0
+    flops, exe, ms, ms_p, ms_f = 0, 0, 0.0, 0.0, 0.0
+    routes = set()
+
+    def timed(fn, n=5):
+        evs = []
+        for _ in range(n):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            evs.append((a, b))
+        return evs
+
     try:
         for lay in layers:
             lin = lay["lin"]
+            h = lay["plan"].handle
             x = torch.from_numpy(W.activations(lin, M).view(np.int16)).view(torch.bfloat16).cuda()
             y = torch.empty((M, lin.n_out), dtype=torch.float32, device="cuda")
             ws = lay["plan"].alloc_workspace(M)
-            P.sdq_prep_activations(lay["plan"].handle, x, M, ws, stream)
-            P.sdq_contract(lay["plan"].handle, lay["tiled"], lay["alpha"], M, y, ws, stream)
-            evs, evp = [], []
-            for _ in range(5):
-                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                a.record(stream)
-                P.sdq_contract(lay["plan"].handle, lay["tiled"], lay["alpha"], M, y, ws, stream)
-                b.record(stream)
-                evs.append((a, b))
-            for _ in range(5):
-                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                a.record(stream)
-                P.sdq_linear_forward(lay["plan"].handle, lay["tiled"], lay["alpha"], x, M, y, ws, stream)
-                b.record(stream)
-                evp.append((a, b))
+            P.sdq_prep_activations(h, x, M, ws, stream)
+            P.sdq_contract(h, lay["tiled"], lay["alpha"], M, y, ws, stream)
+            P.sdq_linear_forward(h, lay["tiled"], lay["alpha"], x, M, y, ws, stream)
+            evs = timed(lambda: P.sdq_contract(h, lay["tiled"], lay["alpha"], M, y, ws, stream))
+            evp = timed(lambda: (P.sdq_prep_activations(h, x, M, ws, stream),
+                                 P.sdq_contract(h, lay["tiled"], lay["alpha"], M, y, ws, stream)))
+            evf = timed(lambda: P.sdq_linear_forward(h, lay["tiled"], lay["alpha"], x, M, y, ws, stream))
             torch.cuda.synchronize()
             ms += sum(a.elapsed_time(b) for a, b in evs) / len(evs)
             ms_p += sum(a.elapsed_time(b) for a, b in evp) / len(evp)
-            flops += 2 * M * lin.n_out * lay["plan"].k_eff
+            ms_f += sum(a.elapsed_time(b) for a, b in evf) / len(evf)
+            keff = lay["plan"].k_eff
+            flops += 2 * M * lin.n_out * keff
+            route = P.sdq_forward_route(h, M)
+            routes.add(route)
+            # executed tensor work of the route sdq_linear_forward takes: the
+            # dense GEMM plus the rebuild (hi and lo parts of G), or the
+            # code-domain contraction plus the prepare GEMM (hi and lo)
+            b_ = W.config(4).block
+            exe += (2 * M * lin.n_out * lin.k_in + 4 * lin.n_out * keff * b_) if route == 3 \
+                else (2 * M * lin.n_out * keff + 4 * M * keff * b_)
             del x, y, ws
     except P.SdqError as e:
         return {"unavailable": str(e)}
     tflops = flops / (ms * 1e-3) / 1e12
+    names = {1: "decode", 2: "code domain (prepare + contraction)", 3: "dense (weights rebuilt, then one GEMM)"}
     return {"value": round(tflops, 1), "unit": "TFLOP/s", "M": M, "ms_per_layer": round(ms, 3),
             "flops_per_layer": flops,
+            "what": "the code-domain contraction kernel alone (sdq_contract), 2 M N K_eff flops",
             "with_prepare": {"value": round(flops / (ms_p * 1e-3) / 1e12, 1), "unit": "TFLOP/s",
                              "ms_per_layer": round(ms_p, 3),
-                             "what": "sdq_linear_forward: the prepare kernel (x_tilde in bf16) and the "
-                                     "contraction"},
+                             "what": "code-domain route: sdq_prep_activations (x_tilde in bf16) + sdq_contract"},
+            "forward": {"route": " / ".join(names[r] for r in sorted(routes)),
+                        "ms_per_layer": round(ms_f, 3),
+                        "code_domain_tflops": round(flops / (ms_f * 1e-3) / 1e12, 1),
+                        "executed_flops_per_layer": exe,
+                        "executed_tflops": round(exe / (ms_f * 1e-3) / 1e12, 1),
+                        "frac_of_bf16_peak": round(exe / (ms_f * 1e-3) / 1e12 / tf_burst, 4),
+                        "what": "sdq_linear_forward as it runs at M = 4096; code_domain_tflops = the "
+                                "code-domain flops (2 M N K_eff) / its time, executed_tflops = the tensor "
+                                "work its route performs / its time"},
             "roofline": {"bound": "tensor", "achieved": round(tflops, 1), "peak": tf_burst,
                          "unit": "TFLOP/s", "frac": round(tflops / tf_burst, 4),
                          "peak_source": peak_src + " bf16 burst"}}

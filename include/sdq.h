@@ -220,15 +220,30 @@ int sdq_contract_add(sdq_plan plan, const uint32_t* codes_tiled, const float* al
  * into it with float reductions (as sdq_contract_add): results agree with
  * sdq_contract to within the order of those additions, not bit for bit.
  * The contraction may start streaming the codes before the prepare kernel
- * completes (it reads nothing the prepare kernel writes until then). */
+ * completes (it reads nothing the prepare kernel writes until then).  Large
+ * batches take the dense route where sdq_forward_route says 3: the weights
+ * are rebuilt into the workspace (sdq_workspace_bytes includes n_out x k_in
+ * bf16 for those batch sizes), then multiplied by x in one GEMM. */
 int sdq_linear_forward(sdq_plan plan, const uint32_t* codes_tiled, const float* alpha,
                        const uint16_t* x, int32_t M, float* y, void* ws, size_t ws_bytes,
                        void* stream);
 
 /* Kernels sdq_linear_forward launches for this plan, batch M and
- * activation pointer x: 2 (the prepare kernel, then the contraction).  0 on
- * invalid input.  Host only. */
+ * activation pointer x: 2 (the prepare kernel, then the contraction; or, on
+ * the dense route, the weight rebuild, then the dense GEMM).  0 on invalid
+ * input.  Host only. */
 int sdq_forward_kernels(sdq_plan plan, int32_t M, const uint16_t* x);
+
+/* The route sdq_linear_forward takes for this plan and batch M: 1 decode
+ * (M <= 64: prepare kernel, tcgen05 block-scaled 4-bit contraction); 2
+ * prefill in the code domain (x_tilde = G x in bf16, tcgen05 bf16
+ * contraction with the codes); 3 dense (M >= 1024 where the plan allows it:
+ * B = 128, n_b a multiple of 64 up to 384: the kernel rebuilds the weights
+ * W' = 2 C G per block in bf16 into the workspace, then y = alpha / 2 x W'^T
+ * as one bf16 GEMM with fp32 accumulation, the same result as route 2 up to
+ * the bf16 rounding of W' in place of x_tilde's).  0 on invalid input.
+ * Host only. */
+int sdq_forward_route(sdq_plan plan, int32_t M);
 
 /* Wait for `stream`, then report whether the last contraction that used
  * `ws` (same plan and M) completed its bounded device-side waits: SDQ_OK or

@@ -24,7 +24,7 @@ __all__ = [
     "sdq_workspace_bytes", "sdq_build_tables", "sdq_decode_launch_shape", "sdq_encode_rows", "sdq_pack", "sdq_unpack",
     "sdq_prep_activations", "sdq_contract", "sdq_contract_add", "sdq_linear_forward", "sdq_read_prep",
     "sdq_workspace_status", "sdq_linear_forward_noalloc", "sdq_noalloc_scratch_bytes", "sdq_noalloc_status",
-    "sdq_forward_kernels", "sdq_status_string", "Plan",
+    "sdq_forward_kernels", "sdq_forward_route", "sdq_status_string", "Plan",
 ]
 
 SDQ_OK = 0
@@ -92,6 +92,7 @@ _SIGS = {
     "sdq_read_prep": (ctypes.c_int, [_vp, _i32, _vp, _vp, _vp]),
     "sdq_workspace_status": (ctypes.c_int, [_vp, _i32, _vp, _vp]),
     "sdq_forward_kernels": (ctypes.c_int, [_vp, _i32, _vp]),
+    "sdq_forward_route": (ctypes.c_int, [_vp, _i32]),
     "sdq_linear_forward_noalloc": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _vp, _vp]),
     "sdq_noalloc_status": (ctypes.c_int, [_vp, _i32, _vp]),
     "sdq_noalloc_scratch_bytes": (_sz, []),
@@ -237,8 +238,14 @@ def sdq_workspace_status(plan, M, ws, stream=None) -> int:
 
 
 def sdq_forward_kernels(plan, M, x) -> int:
-    """Number of kernels sdq_linear_forward launches (2: prepare, contraction)."""
+    """Number of kernels sdq_linear_forward launches (2)."""
     return lib().sdq_forward_kernels(plan, M, _ptr(x))
+
+
+def sdq_forward_route(plan, M) -> int:
+    """Route of sdq_linear_forward at batch M: 1 decode, 2 code-domain
+    prefill, 3 dense (weights rebuilt, then one GEMM); see include/sdq.h."""
+    return lib().sdq_forward_route(plan, M)
 
 
 def sdq_linear_forward_noalloc(plan, codes_tiled, alpha, x, M, y, stream=None):

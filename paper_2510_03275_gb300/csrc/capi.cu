@@ -276,6 +276,12 @@ extern "C" int sdq_forward_kernels(sdq_plan p, int32_t M, const uint16_t* x) {
   return 2;
 }
 
+extern "C" int sdq_forward_route(sdq_plan p, int32_t M) {
+  if (!p || M < 1 || M > 65535) return 0;
+  if (M <= kMaxDecodeM) return 1;
+  return dense_route_applies(p, M) ? 3 : 2;
+}
+
 extern "C" int sdq_workspace_status(sdq_plan p, int32_t M, const void* ws, void* stream) {
   if (!p || M < 1 || M > 65535 || !ws) return SDQ_ERR_INVALID_ARG;
   return workspace_record_status(p, M, ws, stream);

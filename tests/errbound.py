@@ -18,6 +18,13 @@ fp64 oracle by
                      The group maximum is bounded by the 128-code block's.
   prefill (M > 64)   x_tilde rounded once to bf16 (8 significant bits):
                      |error| <= 2^-8 |x_tilde_j|.
+  dense (large M)    the route that rebuilds the weights: W'' = 2 C G per
+                     block in fp32 (G as bf16 hi + lo, ~2^-16), rounded once
+                     to bf16 (|delta W''_rk| <= 2^-9 |W''_rk|), then
+                     y = alpha / 2 x W''^T.  Since |W''_rk| <= 2 sum_j |c_rj|
+                     |G_jk|, the error is at most alpha (2^-9 + 2^-16)
+                     sum_j |c_rj| sum_k |G_jk| |x_k|: a per-code term of
+                     2^-9 sum_i |G_ji x_i| in the sum below.
 
 plus, for both, the fp32 work: x_tilde from bf16 x and G split into two
 bf16 parts (about 2^-16 of sum_i |G_ji x_i|), and fp32 accumulation over K
@@ -51,11 +58,13 @@ class Bound(np.ndarray):
     (``rms``)."""
 
 
-def forward_bound(x, codes, alpha, block, n_b, signs, T=None, hadamard=True):
+def forward_bound(x, codes, alpha, block, n_b, signs, T=None, hadamard=True, dense=False):
     """Per-element bound on |y_cuda - y_oracle| for batch rows x (M, K) and
     the output rows whose codes are ``codes`` (rows, K_eff) and scales
     ``alpha``.  T: e2m1 terms of the decode path; None for the bf16 prefill
-    path."""
+    path; dense: the route that rebuilds the weights in bf16."""
+    if dense:
+        return _dense_bound(x, codes, alpha, block, n_b, signs, hadamard)
     xt = O.prep_activations(x, block, n_b, signs, hadamard)
     m, keff = xt.shape
     if T is None:
@@ -74,6 +83,34 @@ def forward_bound(x, codes, alpha, block, n_b, signs, T=None, hadamard=True):
     var = ((per ** 2 / 3.0) @ (c ** 2).T) * a ** 2
     out = np.asarray(b).view(Bound)
     # the fp32 part, as independent errors of at most `slack` per code
+    var = var + ((slack ** 2) @ (c ** 2).T) * a ** 2
+    out.rms = float(np.sqrt(var.mean())) + 1e-30
+    return out
+
+
+def rebuilt_weights(codes, block, n_b, signs, hadamard=True):
+    """W' = C G per block (fp64): the weights the dense route rebuilds (up
+    to its factor 2 and the bf16 rounding), rows x K."""
+    g = O.decode_table(block, n_b, signs, hadamard)           # n_b x B
+    c = np.asarray(codes, dtype=np.float64)
+    rows, keff = c.shape
+    nblk = keff // n_b
+    return (c.reshape(rows, nblk, n_b) @ g).reshape(rows, nblk * block)
+
+
+def _dense_bound(x, codes, alpha, block, n_b, signs, hadamard):
+    gx = _gx_abs(x, block, n_b, signs, hadamard)              # M x K_eff
+    c = np.abs(np.asarray(codes, dtype=np.float64))
+    a = np.abs(np.asarray(alpha, dtype=np.float64))[None, :]
+    per = (2.0 ** -9 + 2.0 ** -16) * gx
+    slack = FP32_SLACK * gx
+    b = ((per + slack) @ c.T) * a + 1e-30
+    out = np.asarray(b).view(Bound)
+    # independent roundings of the rebuilt weights, each uniform within
+    # +-2^-9 |W''_rk| = +-2^-8 |W'_rk|: error_r = alpha / 2 sum_k x_k dW''_rk
+    wp = rebuilt_weights(codes, block, n_b, signs, hadamard)
+    xf = np.asarray(x, dtype=np.float64)
+    var = ((xf ** 2) @ (wp ** 2).T) * (2.0 ** -18 / 3.0) * a ** 2
     var = var + ((slack ** 2) @ (c ** 2).T) * a ** 2
     out.rms = float(np.sqrt(var.mean())) + 1e-30
     return out

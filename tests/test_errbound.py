@@ -1,7 +1,9 @@
 """CPU: the error bounds the GPU parity tests apply (tests/errbound.py)
-against an fp64 emulation of each path's arithmetic, and against planted
-mistakes in that emulation: the bounds must hold for the arithmetic as
-described and fail for a term too few, a flipped sign or a wrong scale."""
+against an fp64 emulation of each path's arithmetic (decode terms, the bf16
+prefill operand, the dense route's bf16 rebuilt weights), and against
+planted mistakes in that emulation: the bounds must hold for the arithmetic
+as described and fail for a term too few, a flipped sign, a wrong scale,
+coarser weights, a wrong G or misplaced blocks."""
 import numpy as np
 import pytest
 
@@ -102,3 +104,46 @@ def test_transposed_batch_rows_fail(layer):
     y = (_terms(xt[::-1].copy(), 6) @ codes.T) * alpha
     with pytest.raises(AssertionError):
         EB.check(y, yr, EB.forward_bound(x, codes, alpha, b, nb, signs, T=6))
+
+
+def _dense_y(x, codes, alpha, b, nb, signs, mant_bits=8, g=None, shift=0):
+    """The dense route's arithmetic in fp64: W'' = 2 C G per block, rounded
+    to `mant_bits` significant bits (8: bf16), y = alpha / 2 x W''^T; with
+    optional mistakes (another G, blocks of codes shifted by `shift`)."""
+    g = O.decode_table(b, nb, signs, True) if g is None else g
+    c = np.asarray(codes, dtype=np.float64)
+    rows, keff = c.shape
+    nblk = keff // nb
+    cb = np.roll(c.reshape(rows, nblk, nb), shift, axis=1)
+    w2 = 2.0 * (cb @ g).reshape(rows, nblk * b)
+    e = np.floor(np.log2(np.maximum(np.abs(w2), 1e-300)))
+    q = 2.0 ** (e - (mant_bits - 1))
+    w2r = np.where(w2 == 0, 0.0, np.round(w2 / q) * q)
+    return (np.asarray(x, dtype=np.float64) @ w2r.T) * (alpha / 2.0)
+
+
+def test_dense_arithmetic_within_bound(layer):
+    x, codes, alpha, b, nb, signs, yr, xt = layer
+    y = _dense_y(x, codes, alpha, b, nb, signs)
+    EB.check(y, yr, EB.forward_bound(x, codes, alpha, b, nb, signs, dense=True))
+
+
+def test_dense_rebuilt_weights_are_c_times_g(layer):
+    """W' = C G reproduces the code-domain forward exactly (associativity):
+    x W'^T = C x_tilde per row, in fp64."""
+    x, codes, alpha, b, nb, signs, yr, xt = layer
+    wp = EB.rebuilt_weights(codes, b, nb, signs)
+    np.testing.assert_allclose((x @ wp.T) * alpha, yr, rtol=1e-10, atol=1e-12 * np.abs(yr).max())
+
+
+@pytest.mark.parametrize("mistake", ["coarse", "signs", "shift"])
+def test_dense_mistakes_fail(layer, mistake):
+    x, codes, alpha, b, nb, signs, yr, xt = layer
+    if mistake == "coarse":      # weights rounded to 4 significant bits instead of 8
+        y = _dense_y(x, codes, alpha, b, nb, signs, mant_bits=4)
+    elif mistake == "signs":     # G built without the Hadamard signs
+        y = _dense_y(x, codes, alpha, b, nb, signs, g=O.decode_table(b, nb, np.ones_like(signs), True))
+    else:                        # each block's weights rebuilt from the next block's codes
+        y = _dense_y(x, codes, alpha, b, nb, signs, shift=1)
+    with pytest.raises(AssertionError):
+        EB.check(y, yr, EB.forward_bound(x, codes, alpha, b, nb, signs, dense=True))

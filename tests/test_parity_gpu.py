@@ -252,8 +252,9 @@ def _check_forward(plan, d, signs, codes, alpha, tiled, sdq, torch, m, seed, row
     yg = y.cpu().numpy()
     if rows is not None:
         yg = yg[:, rows]
-    EB.check(yg, yr, EB.forward_bound(xf, codes, a, d.block, d.n_b, signs, T=_terms(sdq, d, m)),
-             f"M={m} n={d.n_out} k={d.k_in} B={d.block} OSR={d.osr}")
+    dense = sdq.sdq_forward_route(plan.handle, m) == 3
+    EB.check(yg, yr, EB.forward_bound(xf, codes, a, d.block, d.n_b, signs, T=_terms(sdq, d, m), dense=dense),
+             f"M={m} n={d.n_out} k={d.k_in} B={d.block} OSR={d.osr}" + (" dense" if dense else ""))
     return np.abs(yg - yr).max() / np.abs(yr).max()
 
 
