@@ -237,7 +237,7 @@ int sdq_forward_kernels(sdq_plan plan, int32_t M, const uint16_t* x);
 /* The route sdq_linear_forward takes for this plan and batch M: 1 decode
  * (M <= 64: prepare kernel, tcgen05 block-scaled 4-bit contraction); 2
  * prefill in the code domain (x_tilde = G x in bf16, tcgen05 bf16
- * contraction with the codes); 3 dense (M >= 1024 where the plan allows it:
+ * contraction with the codes); 3 dense (M >= 768 where the plan allows it:
  * B = 128, n_b a multiple of 64 up to 384: the kernel rebuilds the weights
  * W' = 2 C G per block in bf16 into the workspace, then y = alpha / 2 x W'^T
  * as one bf16 GEMM with fp32 accumulation, the same result as route 2 up to

@@ -44,7 +44,7 @@ constexpr int kMaxDecodeM = 64;
 // path) above.
 // Large batches (M >= kDenseMinM) run sdq_linear_forward as "rebuild the
 // weights, then one dense GEMM" (csrc/dense.cu) where the plan allows it.
-constexpr int kDenseMinM = 1024;
+constexpr int kDenseMinM = 768;
 constexpr int kDenseMaxNb = 384;   // G^T hi + lo resident in shared memory
 
 inline int decode_terms(int M) { return M <= 4 ? 6 : (M <= 16 ? 4 : 3); }

@@ -414,6 +414,20 @@ def test_forward_prefill_small(sdq, torch_cuda, q, m, shape):
     assert err <= TOL, err
 
 
+@pytest.mark.parametrize("q", [O.TERNARY, O.BINARY])
+@pytest.mark.parametrize("m,shape", [(768, (300, 512, 128, 2)), (1000, (130, 640, 128, 3)),
+                                     (800, (520, 768, 128, Fraction(3, 2)))])
+def test_forward_dense_route_small(sdq, torch_cuda, q, m, shape):
+    """The dense large-batch route (weights rebuilt in bf16, then one GEMM) on
+    ragged rows and batches, OSR 2 / 3 / 1.5, against the oracle within its
+    bound."""
+    n, k, b, osr = shape
+    lay = _setup_layer(sdq, torch_cuda, n, k, b, osr, q, seed=n + k + m)
+    assert sdq.sdq_forward_route(lay[0].handle, m) == 3
+    err = _check_forward(*lay, sdq, torch_cuda, m, seed=m)
+    assert err <= TOL, err
+
+
 @pytest.mark.parametrize("ci,name,m", [(4, "q", 4096), (4, "gate", 4096), (4, "down", 4096),
                                        (3, "l0.gate", 2048), (3, "l3.down", 2048)])
 def test_forward_prefill_full_size_sampled(sdq, torch_cuda, ci, name, m):
