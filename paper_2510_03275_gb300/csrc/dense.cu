@@ -22,9 +22,9 @@
 //   warp 1     lane 0: 8 MMAs per 64 codes (4 K steps x hi / lo)
 //   warps 2-9  two expander sets (stages of one parity each)
 //   warps 10-13 epilogue
-// K7: a plain tcgen05 GEMM, D[r, m] = W' x^T per CTA tile of 128 weight rows
-// x 256 batch rows, both operands TMA-loaded (128-byte swizzle), 4 stages;
-// epilogue as K5's.
+// K7: a plain tcgen05 GEMM, D[r, m] = W' x^T per CTA tile of 128 (or 2 x 128)
+// weight rows x 256 batch rows, both operands TMA-loaded (128-byte swizzle),
+// 4 (3) stages; epilogue as K5's.
 // Every wait on an mbarrier is bounded (about 2 s); a timeout writes the call
 // number into the workspace's call record and the CTA finishes without
 // further waits.
@@ -248,11 +248,20 @@ __global__ void __launch_bounds__(kRbThreads, 1)
 }
 
 // ------------------------------------------------------------ K7 dense GEMM
-constexpr int kDnBN = 256, kDnStages = 4;
+// WT = 1 or 2 weight tiles of 128 rows per CTA against one 256-row batch
+// tile: with two, the x tile in shared memory serves two MMAs per K step
+// (shared-memory traffic per MMA 136 instead of 163 bytes per cycle of tensor
+// work), where the grid still fills the SMs.
+constexpr int kDnBN = 256;
 constexpr int kDnATile = 128 * kBK * 2;     // 16 KB: 128 weight rows x 64 inputs
 constexpr int kDnBTile = kDnBN * kBK * 2;   // 32 KB: 256 batch rows x 64 inputs
-constexpr int kDnSmem = kDnStages * (kDnATile + kDnBTile) + 1024;
 constexpr int kDnThreads = 320;
+template <int WT> struct DnShape {
+  static constexpr int kStages = WT == 1 ? 4 : 3;
+  static constexpr int kStage = WT * kDnATile + kDnBTile;
+  static constexpr int kSmem = kStages * kStage + 1024;
+  static constexpr uint32_t kCols = WT == 1 ? 256u : 512u;
+};
 
 struct DenseParams {
   const float* alpha;
@@ -262,18 +271,20 @@ struct DenseParams {
   int M, N, nks;
 };
 
+template <int WT>
 __global__ void __launch_bounds__(kDnThreads, 1)
     dense_kernel(const __grid_constant__ CUtensorMap wmap, const __grid_constant__ CUtensorMap xmap,
                  DenseParams p) {
+  constexpr int kStages = DnShape<WT>::kStages, kStage = DnShape<WT>::kStage;
   extern __shared__ uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t full[kDnStages], empty[kDnStages], acc_bar;
+  __shared__ __align__(8) uint64_t full[kStages], empty[kStages], acc_bar;
   __shared__ uint32_t tmem_base;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int n0 = blockIdx.x * 128, m0 = blockIdx.y * kDnBN;
+  const int n0 = blockIdx.x * 128 * WT, m0 = blockIdx.y * kDnBN;
   const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
   uint8_t* base = smem_raw + (sbase - smem_u32(smem_raw));
   if (tid == 0) {
-    for (int s = 0; s < kDnStages; ++s) {
+    for (int s = 0; s < kStages; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
@@ -281,7 +292,7 @@ __global__ void __launch_bounds__(kDnThreads, 1)
     fence_mbar_init();
   }
   if (warp == 0) {
-    tmem_alloc(&tmem_base, kDnBN);
+    tmem_alloc(&tmem_base, DnShape<WT>::kCols);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -295,50 +306,60 @@ __global__ void __launch_bounds__(kDnThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       for (int ks = 0; ks < p.nks && ok; ++ks) {
-        const int s = ks % kDnStages, r = ks / kDnStages;
+        const int s = ks % kStages, r = ks / kStages;
         if (r > 0) ok = mbar_wait(&empty[s], (r - 1) & 1);
         if (!ok) break;
-        mbar_expect_tx(&full[s], kDnATile + kDnBTile);
-        tma_load_2d(base + s * kDnATile, &wmap, ks * kBK, n0, &full[s]);
-        tma_load_2d(base + kDnStages * kDnATile + s * kDnBTile, &xmap, ks * kBK, m0, &full[s]);
+        mbar_expect_tx(&full[s], kStage);
+        uint8_t* st = base + s * kStage;
+#pragma unroll
+        for (int w = 0; w < WT; ++w) tma_load_2d(st + w * kDnATile, &wmap, ks * kBK, n0 + 128 * w, &full[s]);
+        tma_load_2d(st + WT * kDnATile, &xmap, ks * kBK, m0, &full[s]);
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idesc = f16_idesc(kDnBN);
       for (int ks = 0; ks < p.nks && ok; ++ks) {
-        const int s = ks % kDnStages, r = ks / kDnStages;
+        const int s = ks % kStages, r = ks / kStages;
         ok = mbar_wait(&full[s], r & 1);
         if (!ok) break;
         tc_fence_after();
-        const uint64_t ad = sw128_desc(sbase + s * kDnATile);
-        const uint64_t bd = sw128_desc(sbase + kDnStages * kDnATile + s * kDnBTile);
+        const uint32_t st = sbase + s * kStage;
+        const uint64_t bd = sw128_desc(st + WT * kDnATile);
 #pragma unroll
-        for (int kk = 0; kk < kBK / 16; ++kk) umma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (ks | kk) != 0);
+        for (int w = 0; w < WT; ++w) {
+          const uint64_t ad = sw128_desc(st + w * kDnATile);
+#pragma unroll
+          for (int kk = 0; kk < kBK / 16; ++kk)
+            umma_bf16(tmem + (uint32_t)(w * kDnBN), ad + 2 * kk, bd + 2 * kk, idesc, (ks | kk) != 0);
+        }
         umma_commit(&empty[s]);
       }
       umma_commit(&acc_bar);
     }
   } else {
-    // Epilogue: lane quadrant q holds weight rows n0 + 32 q + lane; this warp
-    // writes accumulator columns (batch rows) 128 h .. 128 h + 127.
+    // Epilogue: lane quadrant q holds weight rows n0 + 128 w + 32 q + lane of
+    // accumulator w; this warp writes its columns (batch rows) 128 h .. 128 h + 127.
     const int q = warp & 3, h = (warp - 2) >> 2, rr = 32 * q + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(32 * q) << 16);
     ok = mbar_wait(&acc_bar, 0);
     ok = __all_sync(0xffffffffu, ok);
     tc_fence_after();
     if (ok) {
-      const int row = n0 + rr;
-      const float sa = row < p.N ? 0.5f * __ldg(p.alpha + row) : 0.f;
-      for (int c0 = 128 * h; c0 < 128 * h + 128; c0 += 16) {
-        uint32_t a[16];
-        tmem_ld16(lane_addr + (uint32_t)c0, a);
-        tmem_ld_wait();
-        if (row < p.N) {
+#pragma unroll 1
+      for (int w = 0; w < WT; ++w) {
+        const int row = n0 + 128 * w + rr;
+        const float sa = row < p.N ? 0.5f * __ldg(p.alpha + row) : 0.f;
+        for (int c0 = 128 * h; c0 < 128 * h + 128; c0 += 16) {
+          uint32_t a[16];
+          tmem_ld16(lane_addr + (uint32_t)(w * kDnBN + c0), a);
+          tmem_ld_wait();
+          if (row < p.N) {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const int m = m0 + c0 + i;
-            if (m < p.M) p.y[(size_t)m * p.N + row] = __uint_as_float(a[i]) * sa;
+            for (int i = 0; i < 16; ++i) {
+              const int m = m0 + c0 + i;
+              if (m < p.M) p.y[(size_t)m * p.N + row] = __uint_as_float(a[i]) * sa;
+            }
           }
         }
       }
@@ -350,7 +371,7 @@ __global__ void __launch_bounds__(kDnThreads, 1)
   if (warp == 0) {
     __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tmem, kDnBN);
+    tmem_dealloc(tmem, DnShape<WT>::kCols);
   }
 }
 
@@ -425,10 +446,19 @@ cudaError_t launch_dense_forward(const sdq_plan_s* pl, const uint32_t* codes, co
   dp.rec = rp.rec;
   dp.call = call_tag(next_call_number());
   dp.M = M; dp.N = g.n_out; dp.nks = g.k_in / kBK;
-  e = cudaFuncSetAttribute(dense_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kDnSmem);
+  // two weight tiles per CTA where that still gives two waves of CTAs
+  const int sms = std::max(1, pl->sm_count);
+  const int mt = (M + kDnBN - 1) / kDnBN;
+  if ((int64_t)((g.ntiles + 1) / 2) * mt >= 2 * sms) {
+    e = cudaFuncSetAttribute(dense_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, DnShape<2>::kSmem);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(dense_kernel<2>, dim3((g.ntiles + 1) / 2, mt), dim3(kDnThreads), (size_t)DnShape<2>::kSmem,
+                      st, wmap, xmap, dp);
+  }
+  e = cudaFuncSetAttribute(dense_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, DnShape<1>::kSmem);
   if (e != cudaSuccess) return e;
-  return launch_pdl(dense_kernel, dim3(g.ntiles, (M + kDnBN - 1) / kDnBN), dim3(kDnThreads), (size_t)kDnSmem, st,
-                    wmap, xmap, dp);
+  return launch_pdl(dense_kernel<1>, dim3(g.ntiles, mt), dim3(kDnThreads), (size_t)DnShape<1>::kSmem, st, wmap,
+                    xmap, dp);
 }
 
 }  // namespace sdq
