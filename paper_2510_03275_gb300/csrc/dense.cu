@@ -269,6 +269,9 @@ struct DenseParams {
   uint64_t* rec;
   uint64_t call;
   int M, N, nks;
+  // CTA u < nfull takes unit u (weight-tile group u mod ngroups, batch tile u / ngroups, WT
+  // tiles); CTAs from nfull on split the remaining units into their WT single tiles
+  int ngroups, nfull;
 };
 
 template <int WT>
@@ -280,7 +283,13 @@ __global__ void __launch_bounds__(kDnThreads, 1)
   __shared__ __align__(8) uint64_t full[kStages], empty[kStages], acc_bar;
   __shared__ uint32_t tmem_base;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int n0 = blockIdx.x * 128 * WT, m0 = blockIdx.y * kDnBN;
+  int unit = blockIdx.x, nt = WT, sub = 0;
+  if (unit >= p.nfull) {
+    sub = (unit - p.nfull) % WT;
+    unit = p.nfull + (unit - p.nfull) / WT;
+    nt = 1;
+  }
+  const int n0 = (unit % p.ngroups) * 128 * WT + 128 * sub, m0 = (unit / p.ngroups) * kDnBN;
   const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
   uint8_t* base = smem_raw + (sbase - smem_u32(smem_raw));
   if (tid == 0) {
@@ -309,10 +318,11 @@ __global__ void __launch_bounds__(kDnThreads, 1)
         const int s = ks % kStages, r = ks / kStages;
         if (r > 0) ok = mbar_wait(&empty[s], (r - 1) & 1);
         if (!ok) break;
-        mbar_expect_tx(&full[s], kStage);
+        mbar_expect_tx(&full[s], (uint32_t)(nt * kDnATile + kDnBTile));
         uint8_t* st = base + s * kStage;
 #pragma unroll
-        for (int w = 0; w < WT; ++w) tma_load_2d(st + w * kDnATile, &wmap, ks * kBK, n0 + 128 * w, &full[s]);
+        for (int w = 0; w < WT; ++w)
+          if (w < nt) tma_load_2d(st + w * kDnATile, &wmap, ks * kBK, n0 + 128 * w, &full[s]);
         tma_load_2d(st + WT * kDnATile, &xmap, ks * kBK, m0, &full[s]);
       }
     }
@@ -328,6 +338,7 @@ __global__ void __launch_bounds__(kDnThreads, 1)
         const uint64_t bd = sw128_desc(st + WT * kDnATile);
 #pragma unroll
         for (int w = 0; w < WT; ++w) {
+          if (w >= nt) break;
           const uint64_t ad = sw128_desc(st + w * kDnATile);
 #pragma unroll
           for (int kk = 0; kk < kBK / 16; ++kk)
@@ -347,7 +358,7 @@ __global__ void __launch_bounds__(kDnThreads, 1)
     tc_fence_after();
     if (ok) {
 #pragma unroll 1
-      for (int w = 0; w < WT; ++w) {
+      for (int w = 0; w < nt; ++w) {
         const int row = n0 + 128 * w + rr;
         const float sa = row < p.N ? 0.5f * __ldg(p.alpha + row) : 0.f;
         for (int c0 = 128 * h; c0 < 128 * h + 128; c0 += 16) {
@@ -450,15 +461,22 @@ cudaError_t launch_dense_forward(const sdq_plan_s* pl, const uint32_t* codes, co
   const int sms = std::max(1, pl->sm_count);
   const int mt = (M + kDnBN - 1) / kDnBN;
   if ((int64_t)((g.ntiles + 1) / 2) * mt >= 2 * sms) {
+    dp.ngroups = (g.ntiles + 1) / 2;
+    const int units = dp.ngroups * mt, waves = units / sms, rest = units - waves * sms;
+    // a last wave of at most half the SMs runs as single tiles on twice the CTAs: the
+    // wave then takes a single tile's time (~0.6 of a pair's) instead of a pair's
+    dp.nfull = (rest > 0 && 2 * rest <= sms) ? waves * sms : units;
+    const int grid = dp.nfull + 2 * (units - dp.nfull);
     e = cudaFuncSetAttribute(dense_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, DnShape<2>::kSmem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(dense_kernel<2>, dim3((g.ntiles + 1) / 2, mt), dim3(kDnThreads), (size_t)DnShape<2>::kSmem,
-                      st, wmap, xmap, dp);
+    return launch_pdl(dense_kernel<2>, dim3(grid), dim3(kDnThreads), (size_t)DnShape<2>::kSmem, st, wmap, xmap, dp);
   }
+  dp.ngroups = g.ntiles;
+  dp.nfull = g.ntiles * mt;
   e = cudaFuncSetAttribute(dense_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, DnShape<1>::kSmem);
   if (e != cudaSuccess) return e;
-  return launch_pdl(dense_kernel<1>, dim3(g.ntiles, mt), dim3(kDnThreads), (size_t)DnShape<1>::kSmem, st, wmap,
-                    xmap, dp);
+  return launch_pdl(dense_kernel<1>, dim3(dp.nfull), dim3(kDnThreads), (size_t)DnShape<1>::kSmem, st, wmap, xmap,
+                    dp);
 }
 
 }  // namespace sdq
