@@ -40,9 +40,13 @@ Readings of points the paper leaves open:
   The inverse FFT carries numpy's ``1/N_new`` factor, then the gain
   ``N_new/d_col`` of Algorithm 1 is applied, so amplitudes are preserved.
 * OSR is rational, ``OSR = n_b / B`` with ``n_b`` an integer.
-* GPTQ block compensation (Algorithm 1, lines that update later columns with
-  the inverse Hessian) is not applied: without calibration data the Hessian
-  is ``lambda I`` and the update vanishes, so blocks are independent.
+* GPTQ block compensation (Algorithm 1's update of later columns with the
+  inverse Hessian): :func:`encode` leaves it out (with no calibration data
+  the Hessian is ``lambda I`` and the update vanishes, so blocks are
+  independent); :func:`encode_gptq` applies it with a given factor of
+  ``H^-1``, reading the update as the exact block update ``E U_FF^-1 U_FR``
+  (Algorithm 1 prints ``E . H^-1_{F,R}``), with alpha from the original
+  weights.
 
 Canonical fp32 mode (the bit-exact contract with the CUDA encoder): the
 composed table ``A_enc = fp32(U . Had^T)`` is built in fp64 and rounded once;
@@ -73,6 +77,7 @@ __all__ = [
     "reconstruct", "forward", "forward_code_domain", "prep_activations",
     "compression_ratio", "plain_words_per_row", "pack_plain", "unpack_plain",
     "tiled_geometry", "pack_tiled", "unpack_tiled",
+    "gptq_hessian", "gptq_factor", "decode_table32", "encode_gptq",
 ]
 
 
@@ -496,3 +501,109 @@ def unpack_tiled(words, quantizer: int, n_out: int, k_eff: int) -> np.ndarray:
             else:
                 out[r, kk] = 1 if f else -1
     return out
+
+
+# --------------------------------------------------------------------------
+# GPTQ block compensation (Algorithm 1, outer loop with the inverse Hessian)
+# --------------------------------------------------------------------------
+def gptq_hessian(X, damp_rel: float = 0.01) -> np.ndarray:
+    """``H = 2 X^T X + lambda I`` (fp64, K x K) from calibration activations
+    ``X`` (tokens x K), the Hessian of Algorithm 1's caption, with the
+    dampening ``lambda = damp_rel * mean(diag(2 X^T X))``."""
+    X = np.asarray(X, dtype=np.float64)
+    h = 2.0 * (X.T @ X)
+    lam = damp_rel * float(np.mean(np.diag(h)))
+    return h + lam * np.eye(h.shape[0])
+
+
+def gptq_factor(H) -> np.ndarray:
+    """Algorithm 1's first step: ``U = Cholesky(H^-1)^T`` (fp64, upper
+    triangular, positive diagonal), so that ``U^T U = H^-1``."""
+    P = np.linalg.inv(np.asarray(H, dtype=np.float64))
+    P = 0.5 * (P + P.T)
+    return np.linalg.cholesky(P).T
+
+
+def decode_table32(block: int, n_b: int, signs=None, hadamard: bool = True) -> np.ndarray:
+    """``G`` rounded once to fp32 (n_b x B), entries below 2^-46 (fp64 noise
+    on exact zeros of the real table) set to zero first, as for A_enc."""
+    g = decode_table(block, n_b, signs, hadamard).copy()
+    g[np.abs(g) < ZERO_FLUSH] = 0.0
+    return g.astype(np.float32)
+
+
+def encode_gptq(W, U, block: int, n_b: int, quantizer: int = TERNARY,
+                alpha_mode: int = ALPHA_MAXABS, signs=None, hadamard: bool = True,
+                trace: bool = False):
+    """Canonical fp32 SDQ encoder with GPTQ block compensation (Algorithm 1).
+
+    ``U``: the upper-triangular factor of ``H^-1`` (``U^T U = H^-1``), used in
+    fp32.  Blocks of B columns are taken in order; for block b (columns F,
+    later columns R):
+
+    1. codes ``c`` = SDQuant of the current weights of F (canonical upsample
+       and eq. (8) scan, as :func:`encode`), with the per-row alpha of the
+       ORIGINAL weights (it must be known before the first block's scan);
+    2. ``Q = alpha * (c . G)``: the block's reconstruction (Algorithm 1's
+       ``SDQuant(W Had, OSR) Had^T``), ``s = sum_j c_j G[j, :]`` summed in
+       ascending j from +0, then ``Q = fl(alpha s)``;
+    3. ``E = W_F - Q``;
+    4. the block's error normalised by the diagonal block of the factor,
+       ``E~ = E U_FF^-1`` (forward substitution, ascending column l:
+       ``E~_l = t_l / U_ll``, then ``t_k -= E~_l U_lk`` for k > l);
+    5. ``W_R -= E~ U_FR`` (per element ``acc = sum_k fl(E~_k U_kj)`` in
+       ascending k, then ``W = fl(W - acc)``).
+
+    Step 4 is the reading of Algorithm 1's update ``W_R -= E H^-1_{F,R}``
+    (with ``H^-1`` replaced by its Cholesky factor) as the exact block
+    update of GPTQ / optimal brain surgeon: for one column it is GPTQ's
+    division by the diagonal, and for a block it makes the update equal to
+    ``E H_FR H_RR^-1`` (the minimiser of the layer-output error over the
+    later columns given the block's error), independent of H's scale.
+    Every operation is a rounded fp32 operation in the order stated (numpy
+    float32 elementwise ops never fuse a multiply-add).
+
+    Returns ``(codes, alpha)`` as :func:`encode`; with ``trace`` also a list
+    of per-block dicts (``E``, ``Et``, ``W_before``, ``W_after`` of the
+    later columns, fp32).
+    """
+    a32 = encode_table(block, n_b, signs, hadamard)
+    g32 = decode_table32(block, n_b, signs, hadamard)
+    Wc = np.array(W, dtype=np.float32, copy=True)
+    U32 = np.asarray(U, dtype=np.float32)
+    n, k = Wc.shape
+    if k % block or U32.shape != (k, k):
+        raise ValueError("W must be N x K with K a multiple of B, U K x K")
+    nblk = k // block
+    alpha = row_alpha(upsample_canonical(Wc, a32), alpha_mode)
+    codes = np.zeros((n, nblk * n_b), dtype=np.int8)
+    steps = []
+    for b in range(nblk):
+        f0, f1 = b * block, (b + 1) * block
+        x = upsample_canonical(Wc[:, f0:f1], a32)
+        c = sigma_delta_scan(x, alpha, quantizer)[:, 0, :]
+        codes[:, b * n_b:(b + 1) * n_b] = c
+        cf = c.astype(np.float32)
+        s = np.zeros((n, block), dtype=np.float32)
+        for j in range(n_b):
+            s = s + cf[:, j:j + 1] * g32[j, :]
+        q = alpha[:, None] * s
+        e = Wc[:, f0:f1] - q
+        if f1 == k:
+            break
+        uff = U32[f0:f1, f0:f1]
+        t = e.copy()
+        et = np.zeros_like(e)
+        for l in range(block):
+            et[:, l] = t[:, l] / uff[l, l]
+            t[:, l + 1:] = t[:, l + 1:] - et[:, l:l + 1] * uff[l, l + 1:]
+        ufr = U32[f0:f1, f1:]
+        acc = et[:, 0:1] * ufr[0, :]
+        for kk in range(1, block):
+            acc = acc + et[:, kk:kk + 1] * ufr[kk, :]
+        before = Wc[:, f1:].copy()
+        Wc[:, f1:] = Wc[:, f1:] - acc
+        assert Wc.dtype == np.float32
+        if trace:
+            steps.append({"E": e, "Et": et, "W_before": before, "W_after": Wc[:, f1:].copy()})
+    return (codes, alpha, steps) if trace else (codes, alpha)

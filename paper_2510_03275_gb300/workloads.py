@@ -22,7 +22,8 @@ same linear shapes stand in for them:
         28672x8192, down 8192x28672), Student-t(5) scaled to std 0.015,
         OSR 2, ternary, M = 4096 (prefill) and 1..64 (decode).
 
-Activations: x ~ N(0, 1) rounded to bf16.  Hadamard sign vectors: +-1 drawn
+Activations: x ~ N(0, 1) rounded to bf16.  GPTQ calibration activations:
+:func:`calibration_activations` (correlated channels with outliers).  Hadamard sign vectors: +-1 drawn
 uniformly.  Seeds: ``20251003 + 1000 * index + linear`` (weights; activations
 ``+ 250``; Hadamard signs ``+ 500``).  Matrices are (N, K) = (out, in).
 """
@@ -184,6 +185,21 @@ def activations(lin: Linear, m: int, seed_offset: int = 250) -> np.ndarray:
     rng = np.random.default_rng(lin.seed + seed_offset + 7919 * m)
     x = rng.standard_normal((m, lin.k_in)).astype(np.float32)
     return float_to_bf16(x)
+
+
+def calibration_activations(k_in: int, n_tokens: int, seed: int) -> np.ndarray:
+    """Synthetic calibration activations (n_tokens, k_in) fp32 for the GPTQ
+    Hessian: channels correlated through a rank-16 shared component, per-
+    channel scales log-normal (sigma 0.5) and round(0.005 k_in) outlier
+    channels scaled x20 (the outlier-channel structure of LLM activations;
+    the paper calibrates on C4 samples, which are not available)."""
+    rng = np.random.default_rng([seed, 31337])
+    z = rng.standard_normal((n_tokens, k_in))
+    f = rng.standard_normal((n_tokens, 16))
+    a = rng.standard_normal((16, k_in)) / 4.0
+    scale = np.exp(rng.normal(0.0, 0.5, size=k_in))
+    scale[rng.permutation(k_in)[:int(round(0.005 * k_in))]] *= 20.0
+    return ((z + 2.0 * (f @ a)) * scale).astype(np.float32)
 
 
 def float_to_bf16(x: np.ndarray) -> np.ndarray:
