@@ -9,8 +9,9 @@
  *                        randomised Hadamard smoothing (eq. 13), band-limited
  *                        upsampling, per-row scale, first-order Sigma-Delta
  *                        scan (eqs. 7-8) with the binary (eqs. 3-4) or ternary
- *                        (eqs. 5-6) quantizer.  GPTQ block compensation is
- *                        not applied (no calibration data; blocks independent).
+ *                        (eqs. 5-6) quantizer, blocks independent.
+ *   sdq_encode_rows_gptq the same with Algorithm 1's GPTQ block compensation
+ *                        (inverse-Hessian update of the later columns).
  *   sdq_pack/sdq_unpack  plain <-> tiled code layouts (bit-exact).
  *   sdq_prep_activations x_tilde = G x per block of B inputs, G = D^T Had^T:
  *                        the exact adjoint of the decimation and Hadamard
@@ -141,6 +142,12 @@ size_t sdq_workspace_bytes(sdq_plan plan, int32_t M);
  * sdq_plan_create minus CUDA/UNSUPPORTED. */
 int sdq_build_tables(const sdq_layer_desc* desc, const int8_t* had_signs,
                      float* a_enc_host, float* g_host);
+/* Host-only: the fp32 G of sdq_encode_rows_gptq's block reconstruction (n_b x
+ * block, row-major): the fp64 G rounded to the nearest multiple of 2^-30
+ * (ties to even), then to fp32, so that its value does not depend on fp64
+ * rounding in entries that result from cancellation.  INVALID_ARG for a NULL
+ * g_host or an invalid descriptor. */
+int sdq_build_gptq_table(const sdq_layer_desc* desc, const int8_t* had_signs, float* g_host);
 
 /* Host-only (no GPU needed): the launch shape the decode contraction takes
  * at batch M (1..64) on a device with `sm_count` SMs, as sdq_plan_create
@@ -166,6 +173,34 @@ int sdq_decode_launch_shape(const sdq_layer_desc* desc, int32_t M, int32_t sm_co
  * Needs no workspace.  Pointers must be 16-byte aligned. */
 int sdq_encode_rows(sdq_plan plan, const float* W, uint32_t* codes_plain, float* alpha,
                     void* stream);
+
+/* Bytes of the workspace sdq_encode_rows_gptq needs: a working copy of W
+ * (n_out x k_in fp32) and one block's normalised error per row (n_out x B
+ * fp32).  0 for a NULL plan. */
+size_t sdq_gptq_workspace_bytes(sdq_plan plan);
+/* Algorithm 1 WITH its GPTQ block compensation (the outer loop's update of
+ * the later columns with the inverse Hessian H^-1 = (2 X X^T + lambda I)^-1
+ * of calibration activations X).  U (device, fp32, k_in x k_in row-major):
+ * the upper-triangular factor with U^T U = H^-1 (Algorithm 1's
+ * Cholesky(H^-1)^T), computed by the caller; only its upper triangle is read.
+ * W (device, fp32, n_out x k_in) is not modified: the blocks are encoded in
+ * order on a copy in `ws`.  Outputs as sdq_encode_rows.  alpha is taken from
+ * the original W (pass 0 of sdq_encode_rows).  Then for every block b of B
+ * columns F (later columns R), on the copy: the block's codes c by the same
+ * canonical upsample and scan as sdq_encode_rows; s_k = sum_j fl(c_j G[j][k])
+ * from +0 in ascending j (G = D^T Had^T in fp32, the reconstruction of the
+ * block: Algorithm 1's SDQuant(W Had, OSR) Had^T = alpha c G); E_k =
+ * fl(W_k - fl(alpha s_k)); the normalised error E~ = E U_FF^-1 by forward
+ * substitution (l ascending: E~_l = fl(t_l / U_ll), then t_k = fl(t_k -
+ * fl(E~_l U_lk)) for k > l, t = E at first); and W_R -= E~ U_FR with
+ * acc = fl(...fl(fl(E~_0 U_0c) + fl(E~_1 U_1c))...) in ascending k and
+ * W = fl(W - acc).  E~ U_FR is the exact block update E H_FR H_RR^-1 (the
+ * printed update E H^-1_{F,R} read with GPTQ's normalisation by the factor's
+ * diagonal block).  Requires B a multiple of 4; 2 nblk launches on `stream`.
+ * Pointers 16-byte aligned; SDQ_ERR_WORKSPACE if ws_bytes is below
+ * sdq_gptq_workspace_bytes; SDQ_ERR_UNSUPPORTED for B not a multiple of 4. */
+int sdq_encode_rows_gptq(sdq_plan plan, const float* W, const float* U, uint32_t* codes_plain,
+                         float* alpha, void* ws, size_t ws_bytes, void* stream);
 
 /* Plain -> tiled (sdq_tiled_bytes).  Input and output must not overlap. */
 int sdq_pack(sdq_plan plan, const uint32_t* codes_plain, uint32_t* codes_tiled, void* stream);

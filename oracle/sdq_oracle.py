@@ -524,12 +524,22 @@ def gptq_factor(H) -> np.ndarray:
     return np.linalg.cholesky(P).T
 
 
+# Grid of the fp32 G used by the GPTQ reconstruction (see decode_table32).
+GPTQ_G_GRID = 2.0 ** -30
+
+
 def decode_table32(block: int, n_b: int, signs=None, hadamard: bool = True) -> np.ndarray:
-    """``G`` rounded once to fp32 (n_b x B), entries below 2^-46 (fp64 noise
-    on exact zeros of the real table) set to zero first, as for A_enc."""
-    g = decode_table(block, n_b, signs, hadamard).copy()
-    g[np.abs(g) < ZERO_FLUSH] = 0.0
-    return g.astype(np.float32)
+    """``G`` for the GPTQ block reconstruction (n_b x B, fp32): the fp64 table
+    rounded to the nearest multiple of 2^-30 (ties to even), then to fp32.
+
+    Entries of G that come out of cancellations (~1e-9) carry fp64 errors
+    that are a sizeable part of their fp32 unit in the last place, so two
+    correct fp64 evaluations can round them to different fp32 values; the
+    absolute grid (far coarser than the fp64 error, finer than fp32's
+    resolution at the table's scale) makes the fp32 table a function of the
+    real table only, as the zero flush does for A_enc."""
+    g = decode_table(block, n_b, signs, hadamard)
+    return (np.round(g / GPTQ_G_GRID) * GPTQ_G_GRID).astype(np.float32)
 
 
 def encode_gptq(W, U, block: int, n_b: int, quantizer: int = TERNARY,

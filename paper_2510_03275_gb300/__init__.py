@@ -21,7 +21,8 @@ __all__ = [
     "SDQ_OK", "SDQ_BINARY", "SDQ_TERNARY", "SDQ_ALPHA_MAXABS", "SDQ_ALPHA_MEANABS",
     "SdqError", "LayerDesc", "lib", "library_path",
     "sdq_plan_create", "sdq_plan_destroy", "sdq_k_eff", "sdq_plain_bytes", "sdq_tiled_bytes",
-    "sdq_workspace_bytes", "sdq_build_tables", "sdq_decode_launch_shape", "sdq_encode_rows", "sdq_pack", "sdq_unpack",
+    "sdq_workspace_bytes", "sdq_build_tables", "sdq_build_gptq_table", "sdq_decode_launch_shape", "sdq_encode_rows", "sdq_gptq_workspace_bytes",
+    "sdq_encode_rows_gptq", "sdq_pack", "sdq_unpack",
     "sdq_prep_activations", "sdq_contract", "sdq_contract_add", "sdq_linear_forward", "sdq_read_prep",
     "sdq_workspace_status", "sdq_linear_forward_noalloc", "sdq_noalloc_scratch_bytes", "sdq_noalloc_status",
     "sdq_forward_kernels", "sdq_forward_route", "sdq_status_string", "Plan",
@@ -81,8 +82,11 @@ _SIGS = {
     "sdq_tiled_bytes": (_sz, [ctypes.POINTER(_Desc)]),
     "sdq_workspace_bytes": (_sz, [_vp, _i32]),
     "sdq_build_tables": (ctypes.c_int, [ctypes.POINTER(_Desc), _vp, _vp, _vp]),
+    "sdq_build_gptq_table": (ctypes.c_int, [ctypes.POINTER(_Desc), _vp, _vp]),
     "sdq_decode_launch_shape": (ctypes.c_int, [ctypes.POINTER(_Desc), _i32, _i32, _vp]),
     "sdq_encode_rows": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp]),
+    "sdq_gptq_workspace_bytes": (ctypes.c_size_t, [_vp]),
+    "sdq_encode_rows_gptq": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp, _vp, ctypes.c_size_t, _vp]),
     "sdq_pack": (ctypes.c_int, [_vp, _vp, _vp, _vp]),
     "sdq_unpack": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp]),
     "sdq_prep_activations": (ctypes.c_int, [_vp, _vp, _i32, _vp, _sz, _vp]),
@@ -179,6 +183,17 @@ def sdq_build_tables(desc: LayerDesc, had_signs=None):
     return a, g
 
 
+def sdq_build_gptq_table(desc: LayerDesc, had_signs=None):
+    """Host-only: the fp32 G of the GPTQ block reconstruction (n_b x B)."""
+    import numpy as np
+    g = np.zeros((desc.n_b, desc.block), np.float32)
+    signs = None if had_signs is None else np.ascontiguousarray(had_signs, dtype=np.int8)
+    st = lib().sdq_build_gptq_table(ctypes.byref(desc.c()), None if signs is None else signs.ctypes.data_as(_vp),
+                                    g.ctypes.data_as(_vp))
+    _check(st, "sdq_build_gptq_table")
+    return g
+
+
 _SHAPE_KEYS = ("T", "NP", "S", "P", "CB", "ring", "sb", "nbuf", "smem", "slot_bytes", "b_bytes", "ss",
                "smem_limit", "npipe", "ns", "bstream")
 
@@ -195,6 +210,16 @@ def sdq_decode_launch_shape(desc: LayerDesc, M: int, sm_count: int) -> dict:
 def sdq_encode_rows(plan, W, codes_plain, alpha, stream=None):
     _check(lib().sdq_encode_rows(plan, _ptr(W), _ptr(codes_plain), _ptr(alpha), _stream(stream)),
            "sdq_encode_rows")
+
+
+def sdq_gptq_workspace_bytes(plan) -> int:
+    return int(lib().sdq_gptq_workspace_bytes(plan))
+
+
+def sdq_encode_rows_gptq(plan, W, U, codes_plain, alpha, ws, stream=None):
+    _check(lib().sdq_encode_rows_gptq(plan, _ptr(W), _ptr(U), _ptr(codes_plain), _ptr(alpha), _ptr(ws),
+                                      ws.numel() * ws.element_size(), _stream(stream)),
+           "sdq_encode_rows_gptq")
 
 
 def sdq_pack(plan, codes_plain, codes_tiled, stream=None):
@@ -308,6 +333,16 @@ class Plan:
         codes = self.alloc_plain(W.device)
         alpha = torch.empty(self.desc.n_out, dtype=torch.float32, device=W.device)
         sdq_encode_rows(self.handle, W.contiguous(), codes, alpha, stream)
+        return codes, alpha
+
+    def encode_gptq(self, W, U, stream=None):
+        """W (n_out x k_in fp32, device), U (k_in x k_in fp32, device, upper,
+        U^T U = H^-1) -> (plain codes, alpha) with GPTQ block compensation."""
+        import torch
+        codes = self.alloc_plain(W.device)
+        alpha = torch.empty(self.desc.n_out, dtype=torch.float32, device=W.device)
+        ws = torch.empty(sdq_gptq_workspace_bytes(self.handle), dtype=torch.uint8, device=W.device)
+        sdq_encode_rows_gptq(self.handle, W.contiguous(), U.contiguous(), codes, alpha, ws, stream)
         return codes, alpha
 
     def pack(self, plain, stream=None):

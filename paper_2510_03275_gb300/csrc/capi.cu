@@ -110,9 +110,9 @@ extern "C" int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_sig
   if (major != 10 || minor != 3) return SDQ_ERR_UNSUPPORTED;
 
   const size_t tab = (size_t)g.n_b * g.block;
-  std::vector<float> a_enc(tab), gm(tab), at(tab);
+  std::vector<float> a_enc(tab), gm(tab), at(tab), g32(tab);
   std::vector<double> dt(tab);
-  st = build_tables(desc, had_signs, a_enc.data(), gm.data(), dt.data());
+  st = build_tables(desc, had_signs, a_enc.data(), gm.data(), dt.data(), g32.data());
   if (st != SDQ_OK) return st;
   for (int j = 0; j < g.n_b; ++j)
     for (int k = 0; k < g.block; ++k) at[(size_t)k * g.n_b + j] = a_enc[(size_t)j * g.block + k];
@@ -146,6 +146,7 @@ extern "C" int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_sig
   p->device = dev;
   p->sm_count = sms;
   if (cudaMalloc(&p->d_at, sizeof(float) * tab) != cudaSuccess ||
+      cudaMalloc(&p->d_g32, sizeof(float) * tab) != cudaSuccess ||
       cudaMalloc(&p->d_g_hi, sizeof(uint16_t) * tab) != cudaSuccess ||
       cudaMalloc(&p->d_g_lo, sizeof(uint16_t) * tab) != cudaSuccess) {
     sdq_plan_destroy(p);
@@ -162,6 +163,7 @@ extern "C" int sdq_plan_create(const sdq_layer_desc* desc, const int8_t* had_sig
     return SDQ_ERR_CUDA;
   }
   if (cudaMemcpy(p->d_at, at.data(), sizeof(float) * tab, cudaMemcpyHostToDevice) != cudaSuccess ||
+      cudaMemcpy(p->d_g32, g32.data(), sizeof(float) * tab, cudaMemcpyHostToDevice) != cudaSuccess ||
       cudaMemcpy(p->d_g_hi, ghi.data(), sizeof(uint16_t) * tab, cudaMemcpyHostToDevice) != cudaSuccess ||
       cudaMemcpy(p->d_g_lo, glo.data(), sizeof(uint16_t) * tab, cudaMemcpyHostToDevice) != cudaSuccess) {
     sdq_plan_destroy(p);
@@ -176,6 +178,7 @@ extern "C" int sdq_plan_destroy(sdq_plan p) {
   if (!p) return SDQ_ERR_INVALID_ARG;
   cudaError_t e = cudaSuccess, e2;
   if (p->d_at && (e2 = cudaFree(p->d_at)) != cudaSuccess) e = e2;
+  if (p->d_g32 && (e2 = cudaFree(p->d_g32)) != cudaSuccess) e = e2;
   if (p->d_g_hi && (e2 = cudaFree(p->d_g_hi)) != cudaSuccess) e = e2;
   if (p->d_g_lo && (e2 = cudaFree(p->d_g_lo)) != cudaSuccess) e = e2;
   if (p->d_gt_hi && (e2 = cudaFree(p->d_gt_hi)) != cudaSuccess) e = e2;

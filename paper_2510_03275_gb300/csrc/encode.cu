@@ -1,5 +1,5 @@
-// K1: row-parallel Sigma-Delta encoder (SDQ-LLM Algorithm 1 without GPTQ
-// compensation; eqs. (3)-(8)).
+// K1: row-parallel Sigma-Delta encoder (SDQ-LLM Algorithm 1, eqs. (3)-(8)),
+// and the per-block half of its GPTQ compensation.
 //
 // One warp owns 4 output rows.  For every block of B input columns it
 // rebuilds the upsampled block x_up = A_enc w (A_enc = U Had^T, the
@@ -10,6 +10,13 @@
 // mean); pass 2 recomputes x_up and lanes 0..3 run the first-order
 // Sigma-Delta recursion of eq. (8) over their row, reset at every block, and
 // write the codes in the plain packed layout.
+//
+// The kernel covers a range of passes and blocks.  The encoder with GPTQ
+// block compensation (Algorithm 1's outer loop with the inverse Hessian)
+// runs pass 1 one block at a time on a working copy of W: after the scan,
+// the warp rebuilds the block Q = alpha (c . G), forms E = W_F - Q and the
+// normalised error E~ = E U_FF^-1 (forward substitution over the block's
+// columns), which gptq_update_kernel then applies to the later columns.
 #include "common.cuh"
 
 namespace sdq {
@@ -23,16 +30,75 @@ constexpr int kJC = 128;   // upsampled samples per lane pass (4 per lane)
 struct EncodeParams {
   const float* W;
   uint32_t* codes;
-  float* alpha;
+  float* alpha;       // written by pass 0, read by pass 1 when pass 0 is not run
   const float* at;  // B x n_b, At[k][j] = A_enc[j][k]
   int n_out, k_in, B, n_b, nblk, wpr, quantizer, alpha_mode, warps;
   int64_t k_eff;
+  int pass0, pass1, b0, b1;  // passes [pass0, pass1), blocks [b0, b1)
+  // GPTQ (et non-null): G in fp32 (n_b x B), the factor U (k_in x k_in,
+  // upper), and the normalised block error E~ written per row (n_out x B)
+  const float* g32;
+  const float* U;
+  float* et;
 };
+
+// The warp's GPTQ step for block b of its rows, after the scan: xs holds the
+// rows' codes (as +-1 / 0 floats), ws the block's current weights.  In the
+// order of the oracle's canonical definition: s_k = sum_j c_j G[j][k] from
+// +0 in ascending j, E_k = W_k - alpha s_k; then for l ascending E~_l =
+// t_l / U_ll and t_k -= E~_l U_lk for k > l (t starts as E).  Lane owns
+// columns k = lane (mod 32); t and E~ live in ws in place.
+__device__ __noinline__ void gptq_block_error(const EncodeParams p, int b, int row0, int nrows, float* ws,
+                                              const float* xs, int xs_stride, float alpha_row) {
+  const int lane = threadIdx.x & 31;
+  float ar[kRW];
+#pragma unroll
+  for (int r = 0; r < kRW; ++r) ar[r] = __shfl_sync(0xffffffffu, alpha_row, r);
+  __syncwarp();
+  for (int k = lane; k < p.B; k += 32) {
+    float sacc[kRW];
+#pragma unroll
+    for (int r = 0; r < kRW; ++r) sacc[r] = 0.f;
+    for (int j = 0; j < p.n_b; ++j) {
+      const float gv = __ldg(p.g32 + (size_t)j * p.B + k);
+#pragma unroll
+      for (int r = 0; r < kRW; ++r) sacc[r] = __fadd_rn(sacc[r], __fmul_rn(xs[r * xs_stride + j], gv));
+    }
+#pragma unroll
+    for (int r = 0; r < kRW; ++r) ws[r * p.B + k] = __fsub_rn(ws[r * p.B + k], __fmul_rn(ar[r], sacc[r]));
+  }
+  const size_t ldu = (size_t)p.k_in;
+  const float* uff = p.U + (size_t)b * p.B * ldu + (size_t)b * p.B;
+  for (int l = 0; l < p.B; ++l) {
+    __syncwarp();
+    const float d = __ldg(uff + (size_t)l * ldu + l);
+    float el[kRW];
+#pragma unroll
+    for (int r = 0; r < kRW; ++r) el[r] = __fdiv_rn(ws[r * p.B + l], d);
+    __syncwarp();
+    if ((l & 31) == lane) {
+#pragma unroll
+      for (int r = 0; r < kRW; ++r) ws[r * p.B + l] = el[r];
+    }
+    for (int k = lane; k < p.B; k += 32) {
+      if (k <= l) continue;
+      const float u = __ldg(uff + (size_t)l * ldu + k);
+#pragma unroll
+      for (int r = 0; r < kRW; ++r) ws[r * p.B + k] = __fsub_rn(ws[r * p.B + k], __fmul_rn(el[r], u));
+    }
+  }
+  __syncwarp();
+  for (int i = lane; i < nrows * p.B; i += 32) {
+    const int r = i / p.B, k = i - r * p.B;
+    p.et[(size_t)(row0 + r) * p.B + k] = ws[i];
+  }
+  __syncwarp();
+}
 
 // kTable: the CTA first copies the table into shared memory (where it fits
 // beside the warps' buffers); its reads in the product loop are then
 // shared-memory hits instead of L2 round trips, on which the loop waited.
-template <bool kTable>
+template <bool kTable, bool kGptq>
 __global__ void __launch_bounds__(32 * kMaxWarps) encode_kernel(EncodeParams p) {
   extern __shared__ float smem[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -61,11 +127,16 @@ __global__ void __launch_bounds__(32 * kMaxWarps) encode_kernel(EncodeParams p) 
   float mean_acc = 0.f;  // lane r < 8: sequential sum for MEANABS
   bool mean_first = true;
   float alpha_row = 0.f;  // lane r < 8: alpha of row row0 + r
+  if (p.pass0 == 1 && lane < nrows) alpha_row = p.alpha[row0 + lane];
+  const int per = 32 / p.quantizer;
 
-  for (int pass = 0; pass < 2; ++pass) {
-    // pass-2 scan state of lane r (< nrows)
+  for (int pass = p.pass0; pass < p.pass1; ++pass) {
+    // pass-2 scan state of lane r (< nrows): the partial code word; a range
+    // that starts inside a word continues the word its predecessor wrote
     uint32_t cw = 0;
-    for (int b = 0; b < p.nblk; ++b) {
+    if (pass == 1 && lane < nrows && ((int64_t)p.b0 * p.n_b) % per != 0)
+      cw = p.codes[(size_t)(row0 + lane) * p.wpr + (int64_t)p.b0 * p.n_b / per];
+    for (int b = p.b0; b < p.b1; ++b) {
       __syncwarp();
       const float* wsrc = p.W + (size_t)row0 * p.k_in + (size_t)b * p.B;
       for (int i = lane; i < kRW * p.B; i += 32) {
@@ -131,28 +202,31 @@ __global__ void __launch_bounds__(32 * kMaxWarps) encode_kernel(EncodeParams p) 
         // Eq. (8): i = (i + x) - y_prev, reset per block.
         const float a = alpha_row, theta = 0.5f * alpha_row;
         float integ = 0.f, yp = 0.f;
-        const int per = 32 / p.quantizer;
         uint32_t* crow = p.codes + (size_t)(row0 + lane) * p.wpr;
+        const bool range_end = b == p.b1 - 1;
         for (int j = 0; j < p.n_b; ++j) {
           integ = __fsub_rn(__fadd_rn(integ, xs[lane * xs_stride + j]), yp);
           uint32_t field;
+          float cv;
           if (p.quantizer == SDQ_TERNARY) {
-            if (integ > theta) { field = 1u; yp = a; }
-            else if (integ < -theta) { field = 3u; yp = -a; }
-            else { field = 0u; yp = 0.f; }
+            if (integ > theta) { field = 1u; yp = a; cv = 1.f; }
+            else if (integ < -theta) { field = 3u; yp = -a; cv = -1.f; }
+            else { field = 0u; yp = 0.f; cv = 0.f; }
           } else {
-            if (integ >= 0.f) { field = 1u; yp = a; }
-            else { field = 0u; yp = -a; }
+            if (integ >= 0.f) { field = 1u; yp = a; cv = 1.f; }
+            else { field = 0u; yp = -a; cv = -1.f; }
           }
+          if (kGptq) xs[lane * xs_stride + j] = cv;
           const int64_t kk = (int64_t)b * p.n_b + j;
           const int pos = (int)(kk % per);
           cw |= field << (p.quantizer * pos);
-          if (pos == per - 1 || kk == p.k_eff - 1) {
+          if (pos == per - 1 || kk == p.k_eff - 1 || (range_end && j == p.n_b - 1)) {
             crow[kk / per] = cw;
             cw = 0;
           }
         }
       }
+      if (kGptq && pass == 1) gptq_block_error(p, b, row0, nrows, ws, xs, xs_stride, alpha_row);
     }
     if (pass == 0) {
       if (p.alpha_mode == SDQ_ALPHA_MAXABS) {
@@ -170,8 +244,7 @@ __global__ void __launch_bounds__(32 * kMaxWarps) encode_kernel(EncodeParams p) 
     }
   }
   // Zero the row padding words past the last code.
-  if (lane < nrows) {
-    const int per = 32 / p.quantizer;
+  if (p.pass1 == 2 && p.b1 == p.nblk && lane < nrows) {
     uint32_t* crow = p.codes + (size_t)(row0 + lane) * p.wpr;
     for (int64_t w = (p.k_eff + per - 1) / per; w < p.wpr; ++w) crow[w] = 0u;
   }
@@ -181,12 +254,20 @@ __global__ void __launch_bounds__(32 * kMaxWarps) encode_kernel(EncodeParams p) 
 
 cudaError_t launch_encode(const sdq_plan_s* pl, const float* W, uint32_t* codes, float* alpha,
                           cudaStream_t st) {
+  return launch_encode_range(pl, W, codes, alpha, st, 0, 2, 0, pl->geo.nblk, nullptr, nullptr);
+}
+
+cudaError_t launch_encode_range(const sdq_plan_s* pl, const float* W, uint32_t* codes, float* alpha,
+                                cudaStream_t st, int pass0, int pass1, int b0, int b1, const float* U,
+                                float* et) {
   const Geometry& g = pl->geo;
   EncodeParams p;
   p.W = W; p.codes = codes; p.alpha = alpha; p.at = pl->d_at;
   p.n_out = g.n_out; p.k_in = g.k_in; p.B = g.block; p.n_b = g.n_b; p.nblk = g.nblk;
   p.wpr = g.words_per_row; p.quantizer = pl->desc.quantizer; p.alpha_mode = pl->desc.alpha_mode;
   p.k_eff = g.k_eff;
+  p.pass0 = pass0; p.pass1 = pass1; p.b0 = b0; p.b1 = b1;
+  p.g32 = pl->d_g32; p.U = U; p.et = et;
   const size_t per_warp = sizeof(float) * ((size_t)kRW * g.block + (size_t)kRW * (g.n_b + 1));
   const size_t table = sizeof(float) * (size_t)g.block * g.n_b;
   if (per_warp > 227 * 1024) return cudaErrorInvalidConfiguration;
@@ -197,15 +278,14 @@ cudaError_t launch_encode(const sdq_plan_s* pl, const float* W, uint32_t* codes,
   warps = warps < 1 ? 1 : (warps > kMaxWarps ? kMaxWarps : warps);
   p.warps = warps;
   const size_t smem = per_warp * warps + (in_smem ? table : 0);
-  cudaError_t e = in_smem ? cudaFuncSetAttribute(encode_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 (int)smem)
-                          : cudaFuncSetAttribute(encode_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 (int)smem);
+  const bool gptq = et != nullptr;
+  auto kern = in_smem ? (gptq ? encode_kernel<true, true> : encode_kernel<true, false>)
+                      : (gptq ? encode_kernel<false, true> : encode_kernel<false, false>);
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const int rows_per_cta = warps * kRW;
   const int grid = (g.n_out + rows_per_cta - 1) / rows_per_cta;
-  if (in_smem) encode_kernel<true><<<grid, warps * 32, smem, st>>>(p);
-  else encode_kernel<false><<<grid, warps * 32, smem, st>>>(p);
+  kern<<<grid, warps * 32, smem, st>>>(p);
   return cudaGetLastError();
 }
 

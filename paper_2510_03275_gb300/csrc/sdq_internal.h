@@ -31,7 +31,8 @@ int validate(const sdq_layer_desc* d, Geometry* g);
 //   a_enc: n_b x B row-major, A_enc[j][k] = fp32(sum_k' U[j][k'] Had[k][k'])
 //   g:     n_b x B row-major, G[j][k]     = fp32(sum_k' Dt[j][k'] Had[k][k'])
 //   dt:    n_b x B row-major, D^T itself in fp64 (optional)
-int build_tables(const sdq_layer_desc* d, const int8_t* signs, float* a_enc, float* g, double* dt = nullptr);
+int build_tables(const sdq_layer_desc* d, const int8_t* signs, float* a_enc, float* g, double* dt = nullptr,
+                 float* g_gptq = nullptr);
 
 constexpr int kMaxDecodeM = 64;
 
@@ -84,6 +85,7 @@ struct sdq_plan_s {
   int device;
   int sm_count;
   float* d_at;         // encode table, transposed: B x n_b (At[k][j] = A_enc[j][k])
+  float* d_g32;        // G in fp32, n_b x B row-major (GPTQ block reconstruction)
   uint16_t* d_g_hi;    // G as bf16 hi part, n_b x B row-major
   uint16_t* d_g_lo;    // G - hi as bf16, n_b x B row-major
   uint16_t* d_gt_hi;   // G^T as bf16 hi / lo parts, B x n_b, each 64-code chunk in the

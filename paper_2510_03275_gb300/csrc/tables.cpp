@@ -71,7 +71,8 @@ void fwht(double* v, int n) {
 
 }  // namespace
 
-int build_tables(const sdq_layer_desc* desc, const int8_t* signs, float* a_enc, float* gout, double* dt_out) {
+int build_tables(const sdq_layer_desc* desc, const int8_t* signs, float* a_enc, float* gout, double* dt_out,
+                 float* g_gptq) {
   Geometry g;
   int st = validate(desc, &g);
   if (st != SDQ_OK) return st;
@@ -123,7 +124,7 @@ int build_tables(const sdq_layer_desc* desc, const int8_t* signs, float* a_enc, 
   for (int which = 0; which < 2; ++which) {
     std::vector<double>& M = which ? Dt : U;
     float* out = which ? gout : a_enc;
-    if (!out) continue;
+    if (!out && !(which && g_gptq)) continue;
     for (int j = 0; j < nb; ++j) {
       std::memcpy(row.data(), &M[(size_t)j * B], sizeof(double) * B);
       if (had) {
@@ -133,8 +134,14 @@ int build_tables(const sdq_layer_desc* desc, const int8_t* signs, float* a_enc, 
       // Entries that are exactly zero in real arithmetic (interpolation nodes
       // at integer OSR, Hadamard cancellations) carry fp64 noise of ~1e-16;
       // they are set to exact zero, below 2^-46, before rounding to fp32.
-      for (int k = 0; k < B; ++k)
-        out[(size_t)j * B + k] = std::fabs(row[k]) < 0x1p-46 ? 0.0f : (float)row[k];
+      if (out)
+        for (int k = 0; k < B; ++k)
+          out[(size_t)j * B + k] = std::fabs(row[k]) < 0x1p-46 ? 0.0f : (float)row[k];
+      // G of the GPTQ block reconstruction: rounded to the nearest multiple of
+      // 2^-30 (ties to even) before fp32, so that fp64 errors of entries that
+      // come out of cancellations cannot change their fp32 value
+      if (which && g_gptq)
+        for (int k = 0; k < B; ++k) g_gptq[(size_t)j * B + k] = (float)(std::nearbyint(row[k] * 0x1p30) * 0x1p-30);
     }
   }
   return SDQ_OK;
@@ -145,6 +152,11 @@ int build_tables(const sdq_layer_desc* desc, const int8_t* signs, float* a_enc, 
 extern "C" int sdq_build_tables(const sdq_layer_desc* desc, const int8_t* had_signs,
                                 float* a_enc_host, float* g_host) {
   return sdq::build_tables(desc, had_signs, a_enc_host, g_host);
+}
+
+extern "C" int sdq_build_gptq_table(const sdq_layer_desc* desc, const int8_t* had_signs, float* g_host) {
+  if (!g_host) return SDQ_ERR_INVALID_ARG;
+  return sdq::build_tables(desc, had_signs, nullptr, nullptr, nullptr, g_host);
 }
 
 extern "C" int64_t sdq_k_eff(const sdq_layer_desc* desc) {

@@ -101,6 +101,8 @@ def test_tables_match_oracle(sdq, block, osr, signs, had):
     nb = d.n_b
     assert np.array_equal(a, O.encode_table(block, nb, signs, bool(had)))
     assert np.abs(g - O.decode_table(block, nb, signs, bool(had))).max() < 1e-6
+    # the fp32 G of the GPTQ block reconstruction: the same rounding of the same real table
+    assert np.array_equal(sdq.sdq_build_gptq_table(d, signs), O.decode_table32(block, nb, signs, bool(had)))
 
 
 def _launch_shapes():
