@@ -209,6 +209,49 @@ def build_layer(P, W, torch, cfg):
     return layers, enc_ms
 
 
+def encode_gptq_leg(P, W, torch, cfg):
+    """sdq_encode_rows_gptq on every linear of the layer (device weights).
+    The factor U of H^-1 (H = 2 X^T X / n + 1 % mean-diagonal dampening, X
+    synthetic calibration activations on the device) is made per input width
+    with torch's fp32 Cholesky routines, outside the timed region; the
+    encoder's work does not depend on U's values."""
+    factors = {}
+    per = {}
+    total = 0.0
+    for lin in cfg.linears:
+        k = lin.k_in
+        if k not in factors:
+            x = W.calibration_activations_device(k, 4096, 4242 + k)
+            h = (2.0 / x.shape[0]) * (x.T @ x)
+            del x
+            h += 0.01 * torch.mean(torch.diagonal(h)) * torch.eye(k, device="cuda")
+            lo = torch.linalg.cholesky(h)
+            del h
+            factors[k] = torch.linalg.cholesky(torch.cholesky_inverse(lo), upper=True).contiguous()
+            del lo
+        desc = P.LayerDesc(lin.n_out, lin.k_in, cfg.block, lin.osr, cfg.quantizer)
+        plan = P.Plan(desc, W.hadamard_signs(lin, cfg.block))
+        w = W.weights_device(lin)
+        codes = plan.alloc_plain()
+        alpha = torch.empty(lin.n_out, dtype=torch.float32, device="cuda")
+        ws = torch.empty(P.sdq_gptq_workspace_bytes(plan.handle), dtype=torch.uint8, device="cuda")
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        P.sdq_encode_rows_gptq(plan.handle, w, factors[k], codes, alpha, ws)
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        per[lin.name] = round(ms, 2)
+        total += ms
+        del w, codes, alpha, ws, plan
+    del factors
+    torch.cuda.empty_cache()
+    return {"ms_per_layer": round(total, 1), "per_linear_ms": per,
+            "what": "sdq_encode_rows_gptq (encode with GPTQ block compensation), 7 linears; codes bit-exact "
+                    "with the oracle's canonical definition"}
+
+
 def alg_bytes(lay, M):
     lin = lay["lin"]
     # packed codes (2 bits/code) + alpha + bf16 x + fp32 y
@@ -560,6 +603,7 @@ def run_sdq(args, rank, world, dist):
         out["decode_sweep"] = decode_sweep(P, W, torch, layers, stream, hbm, tf_burst, peak_src)
         out["other_configs"] = extra_configs_leg(P, W, torch, stream, hbm)
         out["prefill"] = prefill_leg(P, W, torch, layers, stream, tf_burst, tf_sus, peak_src)
+        out["encode_gptq"] = encode_gptq_leg(P, W, torch, W.config(4))
         out["cpu_baseline"] = cpu_baseline_leg()
         try:
             out["encode"]["cpu"] = encode_cpu_leg()

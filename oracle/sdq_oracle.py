@@ -20,7 +20,8 @@ What it computes (SDQ-LLM, arXiv 2510.03275):
   exact adjoint of the decimation, which is how activations are "upsampled
   with the same OSR" at inference (section 3.5, Fig. 5, with eq. (12)).
 * Storage accounting, eq. (14).
-* The packed code layouts (plain and tiled) of the C-ABI header.
+* The packed code layouts (plain and tiled) of the C-ABI header, and the
+  base-3 storage of ternary codes (5 trits per byte, 1.6 bits per code).
 
 Readings of points the paper leaves open:
 
@@ -78,6 +79,7 @@ __all__ = [
     "compression_ratio", "plain_words_per_row", "pack_plain", "unpack_plain",
     "tiled_geometry", "pack_tiled", "unpack_tiled",
     "gptq_hessian", "gptq_factor", "decode_table32", "encode_gptq",
+    "TRITS_PER_BYTE", "base3_bytes_per_row", "pack_base3", "unpack_base3",
 ]
 
 
@@ -501,6 +503,52 @@ def unpack_tiled(words, quantizer: int, n_out: int, k_eff: int) -> np.ndarray:
             else:
                 out[r, kk] = 1 if f else -1
     return out
+
+
+# --------------------------------------------------------------------------
+# Base-3 storage of ternary codes (eq. (14)'s ~1.58 bits: 5 trits per byte)
+# --------------------------------------------------------------------------
+TRITS_PER_BYTE = 5
+
+
+def base3_bytes_per_row(k_eff: int) -> int:
+    """Bytes per row of the base-3 layout: ceil(K_eff / 5) rounded up to a
+    multiple of 16."""
+    return 16 * ((-(-k_eff // TRITS_PER_BYTE) + 15) // 16)
+
+
+def pack_base3(codes) -> np.ndarray:
+    """Ternary codes (N, K_eff) -> base-3 bytes (N, bytes_per_row) uint8.
+
+    Code j of a row is trit ``t = code mod 3`` (0 -> 0, +1 -> 1, -1 -> 2) at
+    digit ``j mod 5`` of byte ``j // 5``: ``byte = sum_d t_d 3^d``, at most
+    242.  Codes past K_eff and padding bytes are 0.
+    """
+    c = np.asarray(codes)
+    n, k = c.shape
+    bpr = base3_bytes_per_row(k)
+    t = np.zeros((n, bpr * TRITS_PER_BYTE), dtype=np.int64)
+    t[:, :k] = np.where(c < 0, 2, c)
+    t = t.reshape(n, bpr, TRITS_PER_BYTE)
+    out = np.zeros((n, bpr), dtype=np.int64)
+    for d in range(TRITS_PER_BYTE):
+        out += t[:, :, d] * 3 ** d
+    return out.astype(np.uint8)
+
+
+def unpack_base3(data, k_eff: int):
+    """Inverse of :func:`pack_base3`: (codes (N, K_eff) int8, number of
+    invalid bytes).  A byte above 242 has no 5-trit reading; it is counted
+    and its 5 codes read as 0."""
+    b = np.asarray(data, dtype=np.int64)
+    bad = b > 242
+    v = np.where(bad, 0, b)
+    trits = np.zeros(b.shape + (TRITS_PER_BYTE,), dtype=np.int64)
+    for d in range(TRITS_PER_BYTE):
+        trits[..., d] = v % 3
+        v //= 3
+    codes = np.where(trits == 2, -1, trits).reshape(b.shape[0], -1)[:, :k_eff]
+    return codes.astype(np.int8), int(bad.sum())
 
 
 # --------------------------------------------------------------------------
