@@ -252,6 +252,45 @@ def encode_gptq_leg(P, W, torch, cfg):
                     "with the oracle's canonical definition"}
 
 
+def base3_leg(P, torch, layers):
+    """Base-3 storage of the layer's codes: bytes against the 2-bit layout and
+    the throughput of sdq_pack_base3 / sdq_unpack_base3 (plain <-> base-3;
+    bytes read + written per call over the call's time, events)."""
+    plain_b = b3_b = 0
+    t_pack = t_unpack = 0.0
+    for lay in layers:
+        plan = lay["plan"]
+        d = plan.desc
+        plain = plan.alloc_plain()
+        P.sdq_unpack(plan.handle, lay["tiled"], plain, None)
+        b3 = torch.empty(P.sdq_base3_bytes(d), dtype=torch.uint8, device="cuda")
+        back = torch.empty_like(plain)
+        for _ in range(2):                                 # warm-up
+            P.sdq_pack_base3(plan.handle, plain, b3)
+            P.sdq_unpack_base3(plan.handle, b3, back, None)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        torch.cuda.synchronize()
+        ev[0].record()
+        P.sdq_pack_base3(plan.handle, plain, b3)
+        ev[1].record()
+        P.sdq_unpack_base3(plan.handle, b3, back, None)
+        ev[2].record()
+        torch.cuda.synchronize()
+        assert torch.equal(back, plain), "base-3 round trip"
+        t_pack += ev[0].elapsed_time(ev[1])
+        t_unpack += ev[1].elapsed_time(ev[2])
+        plain_b += plain.numel() * 4
+        b3_b += b3.numel()
+        del plain, b3, back
+    torch.cuda.empty_cache()
+    gbs = (plain_b + b3_b) / 1e9
+    return {"base3_bytes": b3_b, "plain_2bit_bytes": plain_b, "ratio": round(b3_b / plain_b, 4),
+            "bits_per_code": 1.6, "pack_GBps": round(gbs / (t_pack * 1e-3), 1),
+            "unpack_GBps": round(gbs / (t_unpack * 1e-3), 1),
+            "what": "LLaMA-70B layer codes: plain 2-bit <-> base-3 (5 trits per byte), one call per linear; "
+                    "GB/s = (plain + base-3 bytes) / time"}
+
+
 def alg_bytes(lay, M):
     lin = lay["lin"]
     # packed codes (2 bits/code) + alpha + bf16 x + fp32 y
@@ -603,6 +642,7 @@ def run_sdq(args, rank, world, dist):
         out["decode_sweep"] = decode_sweep(P, W, torch, layers, stream, hbm, tf_burst, peak_src)
         out["other_configs"] = extra_configs_leg(P, W, torch, stream, hbm)
         out["prefill"] = prefill_leg(P, W, torch, layers, stream, tf_burst, tf_sus, peak_src)
+        out["base3"] = base3_leg(P, torch, layers)
         out["encode_gptq"] = encode_gptq_leg(P, W, torch, W.config(4))
         out["cpu_baseline"] = cpu_baseline_leg()
         try:

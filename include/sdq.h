@@ -13,6 +13,8 @@
  *   sdq_encode_rows_gptq the same with Algorithm 1's GPTQ block compensation
  *                        (inverse-Hessian update of the later columns).
  *   sdq_pack/sdq_unpack  plain <-> tiled code layouts (bit-exact).
+ *   sdq_pack_base3 /     plain <-> base-3 storage of ternary codes (5 trits
+ *   sdq_unpack_base3     per byte, 1.6 bits per code; eq. 14).
  *   sdq_prep_activations x_tilde = G x per block of B inputs, G = D^T Had^T:
  *                        the exact adjoint of the decimation and Hadamard
  *                        reconstruction, i.e. the activation upsampling of
@@ -210,6 +212,29 @@ int sdq_pack(sdq_plan plan, const uint32_t* codes_plain, uint32_t* codes_tiled, 
  * non-zero count as SDQ_ERR_BAD_CODE. */
 int sdq_unpack(sdq_plan plan, const uint32_t* codes_tiled, uint32_t* codes_plain,
                uint32_t* bad_count, void* stream);
+
+/* Base-3 storage of ternary codes (eq. 14 counts a ternary code as log2(3) =
+ * 1.58 bits; 5 trits per byte store it in 1.6 bits, 80 % of the 2-bit plain
+ * layout).  Row r starts at byte r * bpr, bpr = ceil(K_eff / 5) rounded up to
+ * a multiple of 16; code j is trit t = code mod 3 (0 -> 0, +1 -> 1, -1 -> 2)
+ * at digit j mod 5 of byte j / 5: byte = sum_d t_d 3^d (at most 242); trits
+ * past K_eff and padding bytes are 0.  A storage and transfer format: the
+ * contraction kernels read the tiled 2-bit layout (sdq_unpack_base3 then
+ * sdq_pack rebuilds it).  Ternary plans only.
+ * sdq_base3_bytes: n_out * bpr, host only; 0 for a binary or invalid
+ * descriptor. */
+size_t sdq_base3_bytes(const sdq_layer_desc* desc);
+/* Plain (2-bit) -> base-3 (sdq_base3_bytes).  The invalid pattern 10 is
+ * stored as 0.  Both pointers 16-byte aligned; SDQ_ERR_UNSUPPORTED for a
+ * binary plan. */
+int sdq_pack_base3(sdq_plan plan, const uint32_t* codes_plain, uint8_t* codes_base3, void* stream);
+/* Base-3 -> plain (2-bit, padding 0).  A byte above 242 has no 5-trit
+ * reading: it decodes as five 0 codes and, if `bad_count` (device, one
+ * uint32) is not NULL, is ADDED to it (read it after the stream completes; a
+ * non-zero count is SDQ_ERR_BAD_CODE's condition).  Both pointers 16-byte
+ * aligned; SDQ_ERR_UNSUPPORTED for a binary plan. */
+int sdq_unpack_base3(sdq_plan plan, const uint8_t* codes_base3, uint32_t* codes_plain, uint32_t* bad_count,
+                     void* stream);
 
 /* x_tilde = G x_b for every block b of every row of x (device, bf16 bits,
  * M x k_in row-major), written into the workspace `ws` for sdq_contract.

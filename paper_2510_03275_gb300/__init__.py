@@ -22,7 +22,7 @@ __all__ = [
     "SdqError", "LayerDesc", "lib", "library_path",
     "sdq_plan_create", "sdq_plan_destroy", "sdq_k_eff", "sdq_plain_bytes", "sdq_tiled_bytes",
     "sdq_workspace_bytes", "sdq_build_tables", "sdq_build_gptq_table", "sdq_decode_launch_shape", "sdq_encode_rows", "sdq_gptq_workspace_bytes",
-    "sdq_encode_rows_gptq", "sdq_pack", "sdq_unpack",
+    "sdq_encode_rows_gptq", "sdq_base3_bytes", "sdq_pack_base3", "sdq_unpack_base3", "sdq_pack", "sdq_unpack",
     "sdq_prep_activations", "sdq_contract", "sdq_contract_add", "sdq_linear_forward", "sdq_read_prep",
     "sdq_workspace_status", "sdq_linear_forward_noalloc", "sdq_noalloc_scratch_bytes", "sdq_noalloc_status",
     "sdq_forward_kernels", "sdq_forward_route", "sdq_status_string", "Plan",
@@ -86,6 +86,9 @@ _SIGS = {
     "sdq_decode_launch_shape": (ctypes.c_int, [ctypes.POINTER(_Desc), _i32, _i32, _vp]),
     "sdq_encode_rows": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp]),
     "sdq_gptq_workspace_bytes": (ctypes.c_size_t, [_vp]),
+    "sdq_base3_bytes": (ctypes.c_size_t, [ctypes.POINTER(_Desc)]),
+    "sdq_pack_base3": (ctypes.c_int, [_vp, _vp, _vp, _vp]),
+    "sdq_unpack_base3": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp]),
     "sdq_encode_rows_gptq": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp, _vp, ctypes.c_size_t, _vp]),
     "sdq_pack": (ctypes.c_int, [_vp, _vp, _vp, _vp]),
     "sdq_unpack": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp]),
@@ -220,6 +223,20 @@ def sdq_encode_rows_gptq(plan, W, U, codes_plain, alpha, ws, stream=None):
     _check(lib().sdq_encode_rows_gptq(plan, _ptr(W), _ptr(U), _ptr(codes_plain), _ptr(alpha), _ptr(ws),
                                       ws.numel() * ws.element_size(), _stream(stream)),
            "sdq_encode_rows_gptq")
+
+
+def sdq_base3_bytes(desc: LayerDesc) -> int:
+    return int(lib().sdq_base3_bytes(ctypes.byref(desc.c())))
+
+
+def sdq_pack_base3(plan, codes_plain, codes_base3, stream=None):
+    _check(lib().sdq_pack_base3(plan, _ptr(codes_plain), _ptr(codes_base3), _stream(stream)), "sdq_pack_base3")
+
+
+def sdq_unpack_base3(plan, codes_base3, codes_plain, bad_count=None, stream=None):
+    _check(lib().sdq_unpack_base3(plan, _ptr(codes_base3), _ptr(codes_plain),
+                                  None if bad_count is None else _ptr(bad_count), _stream(stream)),
+           "sdq_unpack_base3")
 
 
 def sdq_pack(plan, codes_plain, codes_tiled, stream=None):

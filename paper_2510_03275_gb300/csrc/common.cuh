@@ -38,15 +38,6 @@ uint64_t call_tag(uint64_t n);
 // Kernel launchers (return cudaError_t of the launch).
 cudaError_t launch_encode(const sdq_plan_s* p, const float* W, uint32_t* codes, float* alpha,
                           cudaStream_t st);
-// Passes [pass0, pass1) (0: alpha, 1: scan) over blocks [b0, b1); with `et`
-// non-null, pass 1 also writes each block's normalised GPTQ error (n_out x B)
-// using the factor U (k_in x k_in).
-cudaError_t launch_encode_range(const sdq_plan_s* p, const float* W, uint32_t* codes, float* alpha,
-                                cudaStream_t st, int pass0, int pass1, int b0, int b1, const float* U,
-                                float* et);
-// W[:, col0:] -= E~ U[b B : (b + 1) B, col0:] (col0 = (b + 1) B) in the canonical order.
-cudaError_t launch_gptq_update(const sdq_plan_s* p, float* W, const float* et, const float* U, int b,
-                               cudaStream_t st);
 cudaError_t launch_pack(const sdq_plan_s* p, const uint32_t* plain, uint32_t* tiled, cudaStream_t st);
 cudaError_t launch_unpack(const sdq_plan_s* p, const uint32_t* tiled, uint32_t* plain,
                           uint32_t* bad, cudaStream_t st);

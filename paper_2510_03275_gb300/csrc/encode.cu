@@ -17,7 +17,7 @@
 // the warp rebuilds the block Q = alpha (c . G), forms E = W_F - Q and the
 // normalised error E~ = E U_FF^-1 (forward substitution over the block's
 // columns), which gptq_update_kernel then applies to the later columns.
-#include "common.cuh"
+#include "encode.cuh"
 
 namespace sdq {
 

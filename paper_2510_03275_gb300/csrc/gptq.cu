@@ -11,7 +11,7 @@
 // division by the diagonal), equal to E H_FR H_RR^-1.  Every product and sum
 // is a rounded fp32 operation in a fixed order (ascending k, first product
 // not added to a zero), so the codes are a deterministic function of W and U.
-#include "common.cuh"
+#include "encode.cuh"
 
 namespace sdq {
 

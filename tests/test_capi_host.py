@@ -171,3 +171,11 @@ def test_decode_launch_shapes_fit(sdq, sms):
                 assert max(-(-s["CB"] // s["sb"]), min(2, s["CB"])) <= 128   # stages per row tile
 
 
+@pytest.mark.parametrize("n,k,osr,q", [(16, 128, Fraction(2), 2), (7, 640, Fraction(17, 16), 2),
+                                       (16, 128, Fraction(2), 1)])
+def test_base3_bytes_geometry(sdq, n, k, osr, q):
+    d = sdq.LayerDesc(n, k, 128, osr, q)
+    if q == 1:
+        assert sdq.sdq_base3_bytes(d) == 0
+    else:
+        assert sdq.sdq_base3_bytes(d) == n * O.base3_bytes_per_row(sdq.sdq_k_eff(d))
