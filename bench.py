@@ -252,6 +252,29 @@ def encode_gptq_leg(P, W, torch, cfg):
                     "with the oracle's canonical definition"}
 
 
+def build_group_layers(P, W, torch, cfg):
+    """The layer as the linears that share an input (q/k/v, gate/up; see
+    workloads.shared_input_groups): one plan per group over the members'
+    rows concatenated, with the first member's Hadamard signs; encoded and
+    packed on the device.  Each entry's "lin" describes the group's matrix."""
+    layers = []
+    for name, members in W.shared_input_groups(cfg):
+        first = members[0]
+        n = sum(m.n_out for m in members)
+        desc = P.LayerDesc(n, first.k_in, cfg.block, first.osr, cfg.quantizer)
+        plan = P.Plan(desc, W.hadamard_signs(first, cfg.block))
+        w = torch.cat([W.weights_device(m) for m in members]) if len(members) > 1 else W.weights_device(first)
+        codes, alpha = plan.encode(w)
+        tiled = plan.pack(codes)
+        torch.cuda.synchronize()
+        del w, codes
+        lin = W.Linear(name, n, first.k_in, first.osr, first.dist, first.std, first.seed)
+        layers.append({"lin": lin, "members": [m.name for m in members], "plan": plan, "tiled": tiled,
+                       "alpha": alpha, "code_bytes": P.sdq_tiled_bytes(desc)})
+    torch.cuda.empty_cache()
+    return layers
+
+
 def base3_leg(P, torch, layers):
     """Base-3 storage of the layer's codes: bytes against the 2-bit layout and
     the throughput of sdq_pack_base3 / sdq_unpack_base3 (plain <-> base-3;
@@ -443,40 +466,11 @@ def extra_configs_leg(P, W, torch, stream, hbm):
     return out
 
 
-def fused_groups_leg(P, torch, stream, hbm, M=1):
-    """The LLaMA-70B layer with q/k/v and gate/up each stored as one matrix
-    (rows concatenated: they read the same input), 4 calls per step; random
-    device codes."""
-    shapes = [("qkv", 10240, 8192), ("o", 8192, 8192), ("gate_up", 57344, 8192), ("down", 8192, 28672)]
-    lays = [random_plan(P, torch, n, k, 128, 2, P.SDQ_TERNARY, 1234 + i) for i, (_, n, k) in enumerate(shapes)]
-    r = step_leg(P, torch, stream, lays, M, reps=50)
-    r["frac_of_hbm"] = round(r["GBps"] / hbm, 4)
-    r["groups"] = [f"{nm} {n}x{k}" for nm, n, k in shapes]
-    del lays
-    torch.cuda.empty_cache()
-    return r
-
-
-def run_sdq(args, rank, world, dist):
+def measure_decode(P, W, torch, layers, M, args, dist, dev, stream, world, hbm, sample_clocks):
+    """The decode step over ``layers`` (one sdq_linear_forward per entry):
+    graph-replayed step time, the decode kernel per launch, and the step end
+    to end with host buffers."""
     import numpy as np
-    import torch
-
-    import paper_2510_03275_gb300 as P
-    from paper_2510_03275_gb300 import workloads as W
-
-    dev = int(os.environ.get("LOCAL_RANK", "0"))
-    torch.cuda.set_device(dev)
-    hbm, tf_burst, tf_sus, peak_src = peaks()
-    cfg = W.config(4)
-    if args.linears:
-        keep = set(args.linears.split(","))
-        cfg.linears = [l for l in cfg.linears if l.name in keep]
-    M = args.m
-    layers, enc_ms = build_layer(P, W, torch, cfg)
-    if args.prefill_only:
-        return {"prefill": prefill_leg(P, W, torch, layers, torch.cuda.Stream(), tf_burst, tf_sus, peak_src),
-                "config": {"workload": "llama70b-layer prefill, M = 4096"
-                                       + (f" [only {args.linears}]" if args.linears else "")}}
     code_bytes = sum(l["code_bytes"] for l in layers)
     # per-linear inputs / outputs / workspaces; the step's x and y each live in
     # one buffer (views per linear), so a step moves them with one copy each
@@ -493,8 +487,6 @@ def run_sdq(args, rank, world, dist):
         yo += M * lin.n_out
         lay["ws"] = lay["plan"].alloc_workspace(M)
         lay["kernels"] = P.sdq_forward_kernels(lay["plan"].handle, M, lay["x"])
-
-    stream = torch.cuda.Stream()
 
     def step():
         for lay in layers:
@@ -515,9 +507,10 @@ def run_sdq(args, rank, world, dist):
         torch.cuda.synchronize()
         replay = graph.replay
 
-    sampler = ClockSampler(dev)
-    sampler.start()
-    time.sleep(0.3)
+    sampler = ClockSampler(dev) if sample_clocks else None
+    if sampler:
+        sampler.start()
+        time.sleep(0.3)
     with torch.cuda.stream(stream):
         for _ in range(max(3, args.warmup)):
             replay()
@@ -537,8 +530,10 @@ def run_sdq(args, rank, world, dist):
     if dist:
         dist.barrier()
     ms_total = ev0.elapsed_time(ev1)
-    clocks = sampler.summary(t_wall0, t_wall1)
-    sampler.stop()
+    clocks = None
+    if sampler:
+        clocks = sampler.summary(t_wall0, t_wall1)
+        sampler.stop()
     ms_total = max_over_ranks(ms_total, dist)
     ms_step = ms_total / args.steps
     value = job_rate(code_bytes, world, ms_step)
@@ -604,6 +599,41 @@ def run_sdq(args, rank, world, dist):
     torch.cuda.synchronize()
     e2e_ms = a.elapsed_time(b) / e2e_steps
     e2e_val = code_bytes * world / (e2e_ms * 1e-3) / 1e9
+    return {"code_bytes": code_bytes, "value": value, "ms_step": ms_step, "clocks": clocks,
+            "achieved": achieved, "per_lin": per_lin, "traffic": traffic, "e2e_val": e2e_val,
+            "e2e_ms": e2e_ms, "h2d": h2d, "d2h": d2h,
+            "kernels": sum(lay["kernels"] for lay in layers)}
+
+
+def run_sdq(args, rank, world, dist):
+    import numpy as np
+    import torch
+
+    import paper_2510_03275_gb300 as P
+    from paper_2510_03275_gb300 import workloads as W
+
+    dev = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(dev)
+    hbm, tf_burst, tf_sus, peak_src = peaks()
+    cfg = W.config(4)
+    if args.linears:
+        keep = set(args.linears.split(","))
+        cfg.linears = [l for l in cfg.linears if l.name in keep]
+    M = args.m
+    layers, enc_ms = build_layer(P, W, torch, cfg)
+    if args.prefill_only:
+        return {"prefill": prefill_leg(P, W, torch, layers, torch.cuda.Stream(), tf_burst, tf_sus, peak_src),
+                "config": {"workload": "llama70b-layer prefill, M = 4096"
+                                       + (f" [only {args.linears}]" if args.linears else "")}}
+    glayers = build_group_layers(P, W, torch, cfg)
+    stream = torch.cuda.Stream()
+    # headline: the step as 4 calls (q/k/v and gate/up each one plan over
+    # their rows: they read the same input); then the 7 linears one call each
+    g = measure_decode(P, W, torch, glayers, M, args, dist, dev, stream, world, hbm, sample_clocks=True)
+    pl = measure_decode(P, W, torch, layers, M, args, dist, dev, stream, world, hbm, sample_clocks=False)
+    code_bytes, value, ms_step, clocks = g["code_bytes"], g["value"], g["ms_step"], g["clocks"]
+    achieved, per_lin, traffic = g["achieved"], g["per_lin"], g["traffic"]
+    e2e_val, e2e_ms, h2d, d2h = g["e2e_val"], g["e2e_ms"], g["h2d"], g["d2h"]
 
     out = {
         "metric": METRIC, "value": round(value, 1), "unit": "GB/s",
@@ -613,6 +643,11 @@ def run_sdq(args, rank, world, dist):
         "config": {"workload": "llama70b-layer decode: q/o 8192x8192, k/v 1024x8192, "
                                "gate/up 28672x8192, down 8192x28672; OSR 2 ternary B=128"
                                + (f" [only {args.linears}]" if args.linears else ""),
+                   "calls_per_step": len(glayers),
+                   "plans": [f"{lay['lin'].name} {lay['lin'].n_out}x{lay['lin'].k_in} = "
+                             + "+".join(lay["members"]) for lay in glayers],
+                   "grouping": "linears that read the same input (q/k/v, gate/up) as one plan over their "
+                               "rows: per-row codes and alpha make each member's outputs those of its own plan",
                    "decode_batch": M, "code_bytes_per_step": code_bytes,
                    "l2": "7 code matrices (428 MB) streamed in turn > 129 MB L2",
                    "timing": ("eager launches" if args.eager else "CUDA graph of one step, replayed")
@@ -623,11 +658,11 @@ def run_sdq(args, rank, world, dist):
                 "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms, 4),
                 "how": "per step: one pinned-host -> device copy of all x, eager sdq_linear_forward "
                        "per linear, one device -> pinned-host copy of all y"},
-        "gpu_launches": sum(lay["kernels"] for lay in layers) * args.steps,
+        "gpu_launches": g["kernels"] * args.steps,
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
                      "unit": "GB/s", "frac": round(achieved / hbm, 4), "traffic": traffic,
                      "kernel": f"decode_kernel, per launch as in the step (sdq_contract_add on the prepared "
-                               f"workspace, M={M})",
+                               f"workspace, M={M}; the 4 plans of the step)",
                      "peak_source": peak_src,
                      "nominal_8tbs_frac": round(achieved / 8000.0, 4), "per_linear": per_lin},
         "roofline_per_step": {"bound": "hbm", "achieved": round(value, 1), "peak": hbm, "unit": "GB/s",
@@ -636,10 +671,17 @@ def run_sdq(args, rank, world, dist):
                                       "and the gaps between them"},
         "encode": {"ms_per_layer": round(enc_ms, 3), "what": "sdq_encode_rows + sdq_pack, 7 linears"},
     }
-    if rank == 0:
-        out["fused_groups"] = fused_groups_leg(P, torch, stream, hbm, M)
+    out["per_linear_step"] = {
+        "GBps": round(pl["value"], 1), "frac_of_hbm": round(pl["value"] / hbm, 4),
+        "ms_per_step": round(pl["ms_step"], 5), "calls": len(layers),
+        "per_launch": {"achieved": round(pl["achieved"], 1), "frac": round(pl["achieved"] / hbm, 4),
+                       "per_linear": pl["per_lin"]},
+        "e2e_GBps": round(pl["e2e_val"], 1),
+        "what": "the same layer as 7 calls, one plan per linear (each with its own Hadamard signs)"}
     if not args.no_extras and rank == 0:
-        out["decode_sweep"] = decode_sweep(P, W, torch, layers, stream, hbm, tf_burst, peak_src)
+        out["decode_sweep"] = decode_sweep(P, W, torch, glayers, stream, hbm, tf_burst, peak_src)
+        out["decode_sweep"]["values_7_calls"] = decode_sweep(P, W, torch, layers, stream, hbm, tf_burst,
+                                                             peak_src)["values"]
         out["other_configs"] = extra_configs_leg(P, W, torch, stream, hbm)
         out["prefill"] = prefill_leg(P, W, torch, layers, stream, tf_burst, tf_sus, peak_src)
         out["base3"] = base3_leg(P, torch, layers)
@@ -692,7 +734,8 @@ def decode_sweep(P, W, torch, layers, stream, hbm_gbs, tf_bf16, peak_src):
             tot_ops += 2.0 * M * lin.n_out * lay["plan"].k_eff
         res[str(M)] = round(tot_b / (tot_ms * 1e-3) / 1e9, 1)
         roof[str(M)] = sweep_roofline(tot_b, tot_ops, tot_ms, hbm_gbs, fp8)
-    return {"unit": "weight GB/s (sdq_linear_forward per linear, inputs on the device, per batch size)",
+    return {"unit": "weight GB/s (sdq_linear_forward per plan of the step, inputs on the device, per batch "
+                    "size; values_7_calls: one plan per linear)",
             "values": res, "roofline": roof,
             "peaks": {"hbm_gbs": hbm_gbs, "fp8_tflops": fp8,
                       "source": peak_src + " (fp8 = bf16 x 2, nominal ratio)"}}

@@ -126,6 +126,33 @@ def config(index: int, multiosr=None) -> Config:
     raise ValueError("config index must be 0..4")
 
 
+def shared_input_groups(cfg: Config):
+    """The linears of ``cfg`` that read the same input, as (name, [Linear])
+    groups in layer order: q/k/v (attention input) and gate/up (MLP input)
+    of each decoder layer when their OSRs agree; every other linear alone.
+    One plan over the rows of a group (rows concatenated, one Hadamard sign
+    vector) computes every member's output: alpha and codes are per row."""
+    groups, i, lins = [], 0, cfg.linears
+    while i < len(lins):
+        pre, base = lins[i].name.rpartition(".")[0], lins[i].name.rpartition(".")[2]
+        members = [lins[i]]
+        want = {"q": ("k", "v"), "gate": ("up",)}.get(base, ())
+        for j, nm in enumerate(want, 1):
+            if i + j < len(lins) and lins[i + j].name == (pre + "." if pre else "") + nm \
+                    and lins[i + j].osr == lins[i].osr and lins[i + j].k_in == lins[i].k_in:
+                members.append(lins[i + j])
+            else:
+                break
+        if len(members) != 1 + len(want):
+            members = [lins[i]]
+        name = (pre + "." if pre else "") + "_".join(m.name.rpartition(".")[2] for m in members)
+        if len(members) == 3:
+            name = (pre + "." if pre else "") + "qkv"
+        groups.append((name, members))
+        i += len(members)
+    return groups
+
+
 def _13b_shapes():
     return [("q", 5120, 5120), ("k", 5120, 5120), ("v", 5120, 5120), ("o", 5120, 5120),
             ("gate", 13824, 5120), ("up", 13824, 5120), ("down", 5120, 13824)]

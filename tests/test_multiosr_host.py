@@ -118,3 +118,14 @@ def test_cli_prints_the_map(capsys):
     out = MO.main(["--config", "3"])
     assert len(out["osr"]) == 28 and abs(out["mean_osr"] - 2.0) <= 0.02
     assert '"workload": "llama-13b-4layers"' in capsys.readouterr().out
+
+
+def test_shared_input_groups():
+    g4 = [(n, [l.name for l in ms]) for n, ms in W.shared_input_groups(W.config(4))]
+    assert g4 == [("qkv", ["q", "k", "v"]), ("o", ["o"]), ("gate_up", ["gate", "up"]), ("down", ["down"])]
+    g1 = [n for n, _ in W.shared_input_groups(W.config(1))]
+    assert g1 == ["qkv", "o", "fc1", "fc2"]
+    # under MultiOSR, members with different OSRs stay separate plans
+    g3 = W.shared_input_groups(W.config(3, multiosr=MO.allocate))
+    assert all(len({l.osr for l in ms}) == 1 for _, ms in g3)
+    assert sum(len(ms) for _, ms in g3) == 28

@@ -441,3 +441,61 @@ def test_forward_prefill_full_size_sampled(sdq, torch_cuda, ci, name, m):
                        seed=lin.seed, rows=rows)
     err = _check_forward(*lay, sdq, torch, m, seed=m + 5, rows=rows)
     assert err <= TOL, err
+
+
+def test_shared_input_group_constituents(sdq, torch_cuda):
+    """One plan over the rows of linears that read one input (q/k/v-shaped:
+    256 + 64 + 64 rows of 512 inputs, OSR 2, ternary, q's Hadamard signs):
+    every member's codes and alpha equal the oracle's encoding of that member
+    alone, bit for bit, and every member's outputs are within their bound at
+    M = 1, 8 and 130."""
+    torch = torch_cuda
+    k = 512
+    members = [W.Linear(nm, n, k, Fraction(2), "t5", 0.02, 900 + i)
+               for i, (nm, n) in enumerate([("q", 256), ("k", 64), ("v", 64)])]
+    ws = [W.weights(l) for l in members]
+    signs = W.hadamard_signs(members[0], 128)
+    wg = np.concatenate(ws)
+    d = _desc(sdq, wg.shape[0], k, 128, 2, O.TERNARY)
+    plan = sdq.Plan(d, signs)
+    codes, alpha = plan.encode(torch.from_numpy(wg).cuda())
+    torch.cuda.synchronize()
+    got = _np_u32(codes).reshape(wg.shape[0], -1)
+    al = alpha.cpu().numpy()
+    r0, per = 0, []
+    for l, w in zip(members, ws):
+        oc, oa = O.encode(w, 128, d.n_b, O.TERNARY, 0, signs, True)
+        assert np.array_equal(al[r0:r0 + l.n_out], oa), l.name
+        assert np.array_equal(got[r0:r0 + l.n_out], O.pack_plain(oc, O.TERNARY)), l.name
+        per.append(oc)
+        r0 += l.n_out
+    tiled = plan.pack(codes)
+    oc_all = np.concatenate(per)
+    for m in (1, 8, 130):
+        r0 = 0
+        for l in members:
+            rows = np.arange(r0, r0 + l.n_out)
+            err = _check_forward(plan, d, signs, oc_all[rows], al, tiled, sdq, torch, m, seed=m + 5, rows=rows)
+            assert err <= TOL, (l.name, m, err)
+            r0 += l.n_out
+
+
+@pytest.mark.parametrize("group", ["qkv", "gate_up"])
+@pytest.mark.parametrize("m", [1, 16])
+def test_forward_full_size_shared_input_groups(sdq, torch_cuda, group, m):
+    """The LLaMA-70B layer's row-concatenated q/k/v (10240 x 8192) and
+    gate/up (57344 x 8192) plans in the bench's launch shape: 16 sampled rows
+    of every member checked against the oracle."""
+    torch = torch_cuda
+    cfg = W.config(4)
+    name, members = [g for g in W.shared_input_groups(cfg) if g[0] == group][0]
+    n, k = sum(l.n_out for l in members), members[0].k_in
+    rng = np.random.default_rng(m + len(members))
+    rows, r0 = [], 0
+    for l in members:
+        rows += list(r0 + rng.choice(l.n_out, 16, replace=False))
+        r0 += l.n_out
+    rows = np.sort(np.array(rows))
+    lay = _setup_layer(sdq, torch, n, k, cfg.block, members[0].osr, cfg.quantizer, seed=members[0].seed, rows=rows)
+    err = _check_forward(*lay, sdq, torch, m, seed=m + 31, rows=rows)
+    assert err <= TOL, err
