@@ -421,22 +421,34 @@ def extra_configs_leg(P, W, torch, stream, hbm):
     out["opt125m"] = {"what": "per-linear latency of one sdq_linear_forward (prepare + contraction), L2 "
                               "flushed before each call, median of 15; binary codes, OSR 5/2",
                       "by_batch": lat}
+    def grouped(cfg):
+        # one plan per group of linears that read the same input (as the headline step)
+        return [random_plan(P, torch, sum(m.n_out for m in ms), ms[0].k_in, cfg.block, ms[0].osr, cfg.quantizer,
+                            ms[0].seed) for _, ms in W.shared_input_groups(cfg)]
+
     # LLaMA-7B
     cfg = W.config(2)
     lays = [random_plan(P, torch, l.n_out, l.k_in, cfg.block, l.osr, cfg.quantizer, l.seed) for l in cfg.linears]
+    glays = grouped(cfg)
     sweep = {}
     for M in (1, 4, 16, 64):
-        r = step_leg(P, torch, stream, lays, M, reps=30)
+        r = step_leg(P, torch, stream, glays, M, reps=30)
         r["frac_of_hbm"] = round(r["GBps"] / hbm, 4)
+        r["GBps_7_calls"] = step_leg(P, torch, stream, lays, M, reps=30)["GBps"]
         sweep[str(M)] = r
-    out["llama7b_layer"] = {"what": "decode step (7 linears, graph-replayed), weight GB/s per batch size",
+    out["llama7b_layer"] = {"what": "decode step (graph-replayed; 4 plans: q/k/v and gate/up each one plan over "
+                                    "their rows, as the headline step; GBps_7_calls: one plan per linear), "
+                                    "weight GB/s per batch size",
                             "by_batch": sweep}
-    del lays
+    del lays, glays
     # LLaMA-13B 4-layer stack, MultiOSR
     cfg = W.config(3, multiosr=allocate)
     lays = [random_plan(P, torch, l.n_out, l.k_in, cfg.block, l.osr, cfg.quantizer, l.seed) for l in cfg.linears]
-    dec = step_leg(P, torch, stream, lays, 8, reps=10)
+    glays = grouped(cfg)
+    dec = step_leg(P, torch, stream, glays, 8, reps=10)
     dec["frac_of_hbm"] = round(dec["GBps"] / hbm, 4)
+    dec["GBps_28_calls"] = step_leg(P, torch, stream, lays, 8, reps=10)["GBps"]
+    del glays
     M = 2048
     ms_k5, ms_all, flops = 0.0, 0.0, 0
     for lay, lin in zip(lays, cfg.linears):

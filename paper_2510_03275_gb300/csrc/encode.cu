@@ -55,17 +55,35 @@ __device__ __noinline__ void gptq_block_error(const EncodeParams p, int b, int r
 #pragma unroll
   for (int r = 0; r < kRW; ++r) ar[r] = __shfl_sync(0xffffffffu, alpha_row, r);
   __syncwarp();
-  for (int k = lane; k < p.B; k += 32) {
-    float sacc[kRW];
+  // 128 columns at a time (4 per lane), j outermost: every (row, column) sum
+  // still runs over j in ascending order, with 16 independent sums per lane
+  for (int kc = 0; kc < p.B; kc += 128) {
+    float sacc[kRW][4];
 #pragma unroll
-    for (int r = 0; r < kRW; ++r) sacc[r] = 0.f;
+    for (int r = 0; r < kRW; ++r)
+#pragma unroll
+      for (int q = 0; q < 4; ++q) sacc[r][q] = 0.f;
     for (int j = 0; j < p.n_b; ++j) {
-      const float gv = __ldg(p.g32 + (size_t)j * p.B + k);
+      float gv[4], xv[kRW];
 #pragma unroll
-      for (int r = 0; r < kRW; ++r) sacc[r] = __fadd_rn(sacc[r], __fmul_rn(xs[r * xs_stride + j], gv));
+      for (int q = 0; q < 4; ++q) {
+        const int k = kc + lane + 32 * q;
+        gv[q] = k < p.B ? __ldg(p.g32 + (size_t)j * p.B + k) : 0.f;
+      }
+#pragma unroll
+      for (int r = 0; r < kRW; ++r) xv[r] = xs[r * xs_stride + j];
+#pragma unroll
+      for (int r = 0; r < kRW; ++r)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) sacc[r][q] = __fadd_rn(sacc[r][q], __fmul_rn(xv[r], gv[q]));
     }
 #pragma unroll
-    for (int r = 0; r < kRW; ++r) ws[r * p.B + k] = __fsub_rn(ws[r * p.B + k], __fmul_rn(ar[r], sacc[r]));
+    for (int q = 0; q < 4; ++q) {
+      const int k = kc + lane + 32 * q;
+      if (k >= p.B) continue;
+#pragma unroll
+      for (int r = 0; r < kRW; ++r) ws[r * p.B + k] = __fsub_rn(ws[r * p.B + k], __fmul_rn(ar[r], sacc[r][q]));
+    }
   }
   const size_t ldu = (size_t)p.k_in;
   const float* uff = p.U + (size_t)b * p.B * ldu + (size_t)b * p.B;
