@@ -6,7 +6,9 @@
 // -1 -> 2) at digit j mod 5 of byte j / 5 (byte = sum_d t_d 3^d <= 242).
 // Both kernels move 80 codes per thread: 16 base-3 bytes <-> 5 plain-layout
 // words (16 two-bit fields each), with 16-byte loads / stores on the base-3
-// side.
+// side; the pack kernel stages its plain words through shared memory per
+// warp (the unpack kernel stores them directly: staging its stores measured
+// slower).
 #include "common.cuh"
 
 namespace sdq {
@@ -23,33 +25,74 @@ struct Base3Params {
 // The plain field of each trit: 0 -> 00, 1 -> 01 (+1), 2 -> 11 (-1).
 __device__ __forceinline__ uint32_t trit_field(uint32_t t) { return t == 0 ? 0u : (t == 1 ? 1u : 3u); }
 
+constexpr int kB3Threads = 256;
+
+// A warp's 32 thread groups own 160 plain words: word i of the warp (i =
+// 5 lane' + q) belongs to lane' = i / 5.  Moving them through shared memory
+// in the order of i makes consecutive lanes touch consecutive words of a row
+// (coalesced) instead of words 20 bytes apart.  Each lane finds the row and
+// word of its k-th staged word from lane' (whose row and group index it
+// reads by shuffle): ok is false past the row's words or the last group.
+__device__ __forceinline__ int64_t warp_word_addr(const Base3Params& p, int64_t row, int gi, bool valid, int k,
+                                                 bool& ok) {
+  const int i = 32 * k + (threadIdx.x & 31);
+  const int src = i / 5, q = i - 5 * src;
+  const int64_t r = __shfl_sync(0xffffffffu, row, src);
+  const int g = __shfl_sync(0xffffffffu, gi, src);
+  const bool v = __shfl_sync(0xffffffffu, valid, src);
+  const int j = 5 * g + q;
+  ok = v && j < p.wpr;
+  return r * p.wpr + j;
+}
+
 // One thread per 80 codes of a row: plain words 5 i .. 5 i + 4 -> base-3
-// bytes 16 i .. 16 i + 15.  Codes past K_eff (and the invalid pattern 10)
-// give trit 0.  gpr = bpr / 16.
-__global__ void pack_base3_kernel(const uint32_t* __restrict__ plain, uint8_t* __restrict__ out, Base3Params p) {
-  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (t >= p.total) return;
-  const int64_t row = t / p.gpr;
-  const int i = (int)(t - row * p.gpr);
-  uint32_t w[5];
-#pragma unroll
-  for (int q = 0; q < 5; ++q) {
-    const int j = 5 * i + q;
-    w[q] = j < p.wpr ? __ldg(plain + row * p.wpr + j) : 0u;
+// bytes 16 i .. 16 i + 15, through a 1024-entry table from a byte's five
+// 2-bit fields (10 bits) to its value (the invalid field 10 reads as trit
+// 0); fields of codes past K_eff are cleared first.  gpr = bpr / 16.
+__global__ void __launch_bounds__(kB3Threads) pack_base3_kernel(const uint32_t* __restrict__ plain,
+                                                                uint8_t* __restrict__ out, Base3Params p) {
+  __shared__ uint8_t lut[1024];
+  __shared__ uint32_t stage[kB3Threads / 32][160];
+  for (int v = threadIdx.x; v < 1024; v += blockDim.x) {
+    uint32_t b = 0;
+    for (int d = 4; d >= 0; --d) {
+      const uint32_t f = (v >> (2 * d)) & 3u;
+      b = 3u * b + ((f & 1u) ? (f >> 1) + 1u : 0u);
+    }
+    lut[v] = (uint8_t)b;
   }
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const bool valid = t < p.total;
+  const int64_t row = valid ? t / p.gpr : 0;
+  const int i = valid ? (int)(t - row * p.gpr) : 0;
+#pragma unroll
+  for (int k = 0; k < 5; ++k) {
+    bool ok;
+    const int64_t a = warp_word_addr(p, row, i, valid, k, ok);
+    stage[warp][32 * k + lane] = ok ? __ldg(plain + a) : 0u;
+  }
+  __syncthreads();
+  if (!valid) return;
+  uint32_t w[6];
+#pragma unroll
+  for (int q = 0; q < 5; ++q) w[q] = stage[warp][5 * lane + q];
+  w[5] = 0u;
   const int64_t c0 = (int64_t)kCodesPerThread * i;
+  if (c0 + kCodesPerThread > p.k_eff) {
+#pragma unroll
+    for (int q = 0; q < 5; ++q) {
+      const int64_t keep = p.k_eff - (c0 + 16 * q);
+      if (keep <= 0) w[q] = 0u;
+      else if (keep < 16) w[q] &= (1u << (2 * keep)) - 1u;
+    }
+  }
   uint32_t bytes[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
   for (int b = 0; b < 16; ++b) {
-    uint32_t v = 0;
-#pragma unroll
-    for (int d = 4; d >= 0; --d) {
-      const int c = 5 * b + d;
-      const uint32_t f = (w[c >> 4] >> (2 * (c & 15))) & 3u;
-      const uint32_t tr = (c0 + c < p.k_eff && (f & 1u)) ? (f >> 1) + 1u : 0u;
-      v = 3u * v + tr;
-    }
-    bytes[b >> 2] |= v << (8 * (b & 3));
+    const int bit = 10 * b, q = bit >> 5, sh = bit & 31;
+    const uint32_t v = (sh <= 22 ? (w[q] >> sh) : __funnelshift_r(w[q], w[q + 1], sh)) & 0x3FFu;
+    bytes[b >> 2] |= (uint32_t)lut[v] << (8 * (b & 3));
   }
   *reinterpret_cast<uint4*>(out + row * p.bpr + 16 * i) = make_uint4(bytes[0], bytes[1], bytes[2], bytes[3]);
 }
@@ -131,9 +174,8 @@ extern "C" int sdq_pack_base3(sdq_plan p, const uint32_t* codes_plain, uint8_t* 
   Base3Params bp;
   bp.n_out = g.n_out; bp.wpr = g.words_per_row; bp.bpr = base3_bytes_per_row(g.k_eff);
   bp.gpr = bp.bpr / 16; bp.k_eff = g.k_eff; bp.total = (int64_t)g.n_out * bp.gpr;
-  const int threads = 256;
-  const int64_t blocks = (bp.total + threads - 1) / threads;
-  pack_base3_kernel<<<(unsigned)blocks, threads, 0, (cudaStream_t)stream>>>(codes_plain, codes_base3, bp);
+  const int64_t blocks = (bp.total + kB3Threads - 1) / kB3Threads;
+  pack_base3_kernel<<<(unsigned)blocks, kB3Threads, 0, (cudaStream_t)stream>>>(codes_plain, codes_base3, bp);
   return cudaGetLastError() == cudaSuccess ? SDQ_OK : SDQ_ERR_CUDA;
 }
 
@@ -149,9 +191,8 @@ extern "C" int sdq_unpack_base3(sdq_plan p, const uint8_t* codes_base3, uint32_t
   Base3Params bp;
   bp.n_out = g.n_out; bp.wpr = g.words_per_row; bp.bpr = base3_bytes_per_row(g.k_eff);
   bp.gpr = (g.words_per_row + 4) / 5; bp.k_eff = g.k_eff; bp.total = (int64_t)g.n_out * bp.gpr;
-  const int threads = 256;
-  const int64_t blocks = (bp.total + threads - 1) / threads;
-  unpack_base3_kernel<<<(unsigned)blocks, threads, 0, (cudaStream_t)stream>>>(codes_base3, codes_plain, bad_count,
-                                                                              bp);
+  const int64_t blocks = (bp.total + kB3Threads - 1) / kB3Threads;
+  unpack_base3_kernel<<<(unsigned)blocks, kB3Threads, 0, (cudaStream_t)stream>>>(codes_base3, codes_plain,
+                                                                                  bad_count, bp);
   return cudaGetLastError() == cudaSuccess ? SDQ_OK : SDQ_ERR_CUDA;
 }
