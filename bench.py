@@ -4,14 +4,18 @@ Workload (N=1): the LLaMA-70B-shaped decoder layer (q/o 8192x8192, k/v
 1024x8192, gate/up 28672x8192, down 8192x28672), OSR 2, ternary codes, B =
 128, synthetic Student-t(5) weights (std 0.015) and N(0,1) bf16
 activations.  One step = the decode forward (prep + contraction) of all
-seven linears at batch M (default 1).  Metric: weight-HBM GB/s = packed code
-bytes of the layer / step time.  The 7 code matrices (428 MB) are streamed in
+seven linears at batch M (default 1), as 4 calls: the linears that read the
+same input (q/k/v, gate/up) are each one plan over their rows (per-row codes
+and alpha: every member's outputs are those of its own plan); the same layer
+as 7 calls is reported beside it.  Metric: weight-HBM GB/s = packed code
+bytes of the layer / step time.  The code matrices (428 MB) are streamed in
 turn, so every step reads them from HBM (L2 is 129 MB).
 
 Also reported: the decode kernel's roofline (algorithmic bytes / event-timed
 launch duration against the measured HBM copy bandwidth), the end-to-end
-figure through the C ABI with host buffers, the encoder time, the prefill
-(M = 4096) throughput when available, and the oracle's CPU time.
+figure through the C ABI with host buffers, the encoder time (also with
+GPTQ block compensation), base-3 storage, the prefill (M = 4096) throughput,
+the other workloads, and the oracle's CPU time.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
 Multi-GPU runs (torchrun, one process per GPU) are independent replicas.
