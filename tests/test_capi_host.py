@@ -179,3 +179,18 @@ def test_base3_bytes_geometry(sdq, n, k, osr, q):
         assert sdq.sdq_base3_bytes(d) == 0
     else:
         assert sdq.sdq_base3_bytes(d) == n * O.base3_bytes_per_row(sdq.sdq_k_eff(d))
+
+
+def test_header_compiles_as_c99(tmp_path):
+    """include/sdq.h is a plain C header: no C++ or torch types at the boundary."""
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("gcc not found")
+    src = tmp_path / "use.c"
+    src.write_text('#include "sdq.h"\nint main(void) { sdq_plan p = 0; (void)p; return 0; }\n')
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    r = subprocess.run([gcc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror", "-I", inc, "-c", str(src),
+                        "-o", str(tmp_path / "use.o")], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
