@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--m", type=int, default=1, help="decode batch")
     ap.add_argument("--no-extras", action="store_true", help="skip encode/prefill/sweep/cpu legs")
     ap.add_argument("--linears", default="", help="comma list of llama-70b-layer linears to run (default: all 7)")
+    ap.add_argument("--encode-only", action="store_true",
+                    help="run only the base-3 storage and GPTQ encoder legs (for their ncu captures)")
     ap.add_argument("--prefill-only", action="store_true",
                     help="time only the prefill leg (M = 4096) on the chosen linears and print its JSON "
                          "(for profiling the prefill kernels alone)")
@@ -637,6 +639,10 @@ def run_sdq(args, rank, world, dist):
         cfg.linears = [l for l in cfg.linears if l.name in keep]
     M = args.m
     layers, enc_ms = build_layer(P, W, torch, cfg)
+    if args.encode_only:
+        return {"base3": base3_leg(P, torch, layers), "encode_gptq": encode_gptq_leg(P, W, torch, cfg),
+                "config": {"workload": "llama70b-layer encode legs"
+                                       + (f" [only {args.linears}]" if args.linears else "")}}
     if args.prefill_only:
         return {"prefill": prefill_leg(P, W, torch, layers, torch.cuda.Stream(), tf_burst, tf_sus, peak_src),
                 "config": {"workload": "llama70b-layer prefill, M = 4096"
