@@ -273,19 +273,3 @@ def weights_device(lin: Linear, device="cuda"):
         rs = np.random.default_rng([lin.seed, 7777]).uniform(np.log(0.5), np.log(2.0), size=n)
         w *= torch.as_tensor(np.exp(rs), device=device, dtype=torch.float32)[:, None]
     return w
-
-
-def calibration_activations_device(k_in: int, n_tokens: int, seed: int, device="cuda"):
-    """Calibration activations with the distribution of
-    :func:`calibration_activations`, drawn on the device with torch's Philox
-    generator (different draws; for timing legs at full layer size)."""
-    import torch
-    g = torch.Generator(device=device)
-    g.manual_seed(seed)
-    z = torch.randn((n_tokens, k_in), generator=g, device=device)
-    f = torch.randn((n_tokens, 16), generator=g, device=device)
-    a = torch.randn((16, k_in), generator=g, device=device) / 4.0
-    scale = torch.exp(torch.randn((k_in,), generator=g, device=device) * 0.5)
-    idx = torch.randperm(k_in, generator=g, device=device)[:int(round(0.005 * k_in))]
-    scale[idx] *= 20.0
-    return (z + 2.0 * (f @ a)) * scale
