@@ -392,7 +392,6 @@ def extra_configs_leg(P, W, torch, stream, hbm):
     step at M = 1, 4, 16, 64; the LLaMA-13B 4-layer stack under the MultiOSR
     map: M = 8 decode step and M = 2048 prefill (contraction alone and with its
     prepare kernel)."""
-    import numpy as np
     from paper_2510_03275_gb300.multiosr import allocate
     out = {}
     flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
@@ -621,7 +620,6 @@ def measure_decode(P, W, torch, layers, M, args, dist, dev, stream, world, hbm, 
 
 
 def run_sdq(args, rank, world, dist):
-    import numpy as np
     import torch
 
     import paper_2510_03275_gb300 as P
